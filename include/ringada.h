@@ -1,0 +1,228 @@
+/*
+ * ringada.h -- C ABI of libringada: the per-batch adapter fine-tuning step of RingAda
+ * (arXiv 2502.19864) on one GB300.
+ *
+ * The step (Algorithm 1, the lines "Perform Fw propagation", "calculates the loss and
+ * updates the head", "Perform Bw propagation ending at the (L - d + 1)-th adapter"; and
+ * Section III-B.2) is:
+ *   ra_forward            forward through all L frozen transformer blocks, each with two
+ *                         Houlsby adapters h <- h + GELU(h W_down) W_up (Eq. 1), then the
+ *                         head and the mean cross-entropy loss;
+ *   ra_backward_truncated the backward from the loss down to the lowest unfrozen layer k
+ *                         (0-based, k = L - d), with activation gradients through the
+ *                         frozen weights of layers > k and weight gradients only for the
+ *                         adapters of layers >= k and the head; layers < k get no work;
+ *   ra_adapter_update     Adam on the unfrozen adapters and the trainable head;
+ *   ra_set_unfrozen_depth the top-down unfreezing schedule's depth d (Algorithm 1,
+ *                         "d = d + 1" every interval; Section III-A).
+ *
+ * Conventions
+ *   - Every pointer named *_dev is a CUDA device pointer; everything else is host memory.
+ *   - Device memory is owned by the caller (e.g. PyTorch): the library reports the sizes
+ *     it needs (ra_required_bytes) and binds caller buffers (ra_bind_memory).  It never
+ *     allocates device memory itself and never frees caller memory.
+ *   - Calls that take a cudaStream_t enqueue work on that stream and return; results
+ *     land on the device.  Caller inputs must stay valid until the stream reaches the work.
+ *     A stream of 0 is the legacy default stream.
+ *   - Errors are status codes; nothing throws or aborts.  ra_last_error(ctx) gives a
+ *     message for the last failing call on that context.  On error, no work was enqueued
+ *     by that call unless stated otherwise.
+ *   - Device waits inside kernels are bounded; a wait that runs out records a flag that
+ *     ra_sync_status reports as RA_ERR_TIMEOUT.
+ *   - Thread safety: one context must not be used from two host threads at once.
+ *   - Layout: activations are row-major [B, S, H] (token-major), B*S = T tokens.  Adapter
+ *     matrices follow Eq. 1's row-vector convention: W_down [H, m], W_up [m, H].  Frozen
+ *     linear weights are [out, in] (the product is x W^T).
+ */
+#ifndef RINGADA_H
+#define RINGADA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* ra_stream_t; /* same type as cudaStream_t */
+
+typedef enum {
+  RA_OK = 0,
+  RA_ERR_ARG = 1,         /* a null pointer, out-of-range index or size */
+  RA_ERR_STATE = 2,       /* calls out of order (no memory bound, no forward before backward...) */
+  RA_ERR_NOT_SAVED = 3,   /* backward asked to reach below the layers the forward saved */
+  RA_ERR_SHAPE = 4,       /* B > max_batch, S > max_seq, or an unsupported model shape */
+  RA_ERR_NOMEM = 5,       /* a bound buffer is smaller than required */
+  RA_ERR_CUDA = 6,        /* a CUDA runtime/driver call failed (message has the CUDA error) */
+  RA_ERR_TIMEOUT = 7,     /* a bounded device wait expired (kernel returned early) */
+  RA_ERR_UNSUPPORTED = 8  /* no sm_103 device, or a feature this build does not have */
+} ra_status;
+
+enum { RA_ENCODER_POSTLN = 0, RA_DECODER_PRENORM = 1 };
+enum { RA_F32 = 0, RA_BF16 = 1 };
+
+/* Model shape.  Encoder: post-LN blocks (LayerNorm, biased linears, exact-GELU FFN), a
+ * trainable n_out-class linear head on the token at position 0.  Decoder: pre-RMSNorm
+ * blocks, causal attention with rotate-half RoPE, SwiGLU FFN (ffn % 64 == 0), final
+ * RMSNorm and a frozen n_out-way vocabulary head over every position. */
+typedef struct {
+  int32_t arch;            /* RA_ENCODER_POSTLN | RA_DECODER_PRENORM */
+  int32_t n_layers;        /* L >= 1 */
+  int32_t hidden;          /* H, multiple of 64 */
+  int32_t n_heads;         /* H / n_heads in {64, 128} for bf16, <= 128 for f32 */
+  int32_t ffn;             /* F, multiple of 64 */
+  int32_t n_out;           /* classes (encoder) or vocabulary (decoder), multiple of 8 for decoder bf16 */
+  int32_t max_batch;       /* capacity: ra_forward accepts B <= max_batch */
+  int32_t max_seq;         /* capacity: ra_forward accepts S <= max_seq */
+  int32_t dtype;           /* RA_F32 | RA_BF16: storage of weights and activations */
+  int32_t head_trainable;  /* 1: the head is updated with the adapters (encoder); 0: frozen */
+  int32_t max_depth;       /* largest unfreezing depth that will be used (0 = L); sizes the
+                              saved-activation arena: memory falls as this falls */
+  float norm_eps;          /* LayerNorm / RMSNorm epsilon */
+  float rope_theta;        /* RoPE base (decoder) */
+} ra_model_cfg;
+
+typedef struct {
+  float lr, beta1, beta2, eps; /* Adam, no weight decay, bias-corrected */
+} ra_adam_cfg;
+
+/* Parameter ids for ra_set_weights / ra_get_grad. */
+typedef enum {
+  /* encoder block */
+  RA_P_WQKV = 0, RA_P_BQKV, RA_P_WO, RA_P_BO, RA_P_LN1_G, RA_P_LN1_B,
+  RA_P_W1, RA_P_B1, RA_P_W2, RA_P_B2, RA_P_LN2_G, RA_P_LN2_B,
+  /* adapters (both archs): attention-branch and FFN-branch, Eq. 1 */
+  RA_P_WDA, RA_P_WUA, RA_P_WDF, RA_P_WUF,
+  /* decoder block */
+  RA_P_WQ, RA_P_WK, RA_P_WV, RA_P_RMS1_G, RA_P_WG, RA_P_WU, RA_P_WD, RA_P_RMS2_G,
+  /* head (layer index -1) */
+  RA_P_HEAD_W, RA_P_HEAD_B, RA_P_RMSF_G,
+  RA_P_COUNT
+} ra_param;
+
+typedef struct {
+  int32_t layer;       /* 0..L-1, or -1 for the head */
+  int32_t param;       /* ra_param */
+  const float* data_dev; /* device, float32, row-major in the shape documented for the param;
+                            values are rounded once to the model's storage dtype */
+  int64_t numel;       /* must equal the param's element count */
+} ra_tensor_desc;
+
+typedef struct {
+  int64_t weights_bytes, trainable_bytes, workspace_bytes; /* bound sizes */
+  int64_t saved_bytes_capacity;  /* arena for max_depth layers */
+  int64_t saved_bytes_in_use;    /* activations the last forward kept (layers >= k) */
+  int32_t depth;                 /* current unfreezing depth d */
+  int32_t k_forward;             /* lowest layer the last forward saved, -1 before any */
+  int32_t k_backward;            /* lowest layer the last backward reached, -1 before any */
+  int32_t n_updates;             /* completed ra_adapter_update calls */
+  int32_t tokens;                /* B*S of the last forward */
+  int32_t num_sms;               /* SMs of the bound device */
+} ra_stats;
+
+typedef struct ra_ctx ra_ctx;
+
+/* Create a context for the model (host only; no device work).  adapter_dim = m (the
+ * bottleneck of Eq. 1), 8 <= m <= 256, multiple of 8.  *out receives the context. */
+ra_status ra_create(const ra_model_cfg* cfg, int32_t adapter_dim, ra_ctx** out);
+
+/* Bytes the caller must provide: frozen weights (and their transposed copies),
+ * trainable state (adapter/head masters, gradients, Adam moments) and workspace (saved
+ * activations for max_depth layers plus scratch).  Each buffer must be 256-byte aligned. */
+ra_status ra_required_bytes(const ra_ctx* ctx, size_t* weights, size_t* trainable,
+                            size_t* workspace);
+
+/* Bind caller-owned device buffers of at least the required sizes (sizes are given so
+ * the library can check them).  Selects the current CUDA device as the context's device;
+ * requires compute capability 10.3 (sm_103).  Zeroes gradients, moments and step counts. */
+ra_status ra_bind_memory(ra_ctx* ctx, void* weights_dev, size_t weights_bytes,
+                         void* trainable_dev, size_t trainable_bytes,
+                         void* workspace_dev, size_t workspace_bytes);
+
+/* Copy parameters in (frozen weights, initial adapters and head).  Every parameter of the
+ * model must have been set once before the first ra_forward.  Builds the transposed
+ * copies the backward reads.  Enqueued on stream. */
+ra_status ra_set_weights(ra_ctx* ctx, const ra_tensor_desc* list, int32_t n, ra_stream_t stream);
+
+/* Unfreezing depth d (1..max_depth): the next forward saves activations for layers
+ * k = L - d .. L-1 only (Section III-A: below the depth only the forward runs). */
+ra_status ra_set_unfrozen_depth(ra_ctx* ctx, int32_t d);
+
+/* Forward and loss (Algorithm 1 "Fw propagation", "calculates the loss").
+ * x_dev [B, S, H] in the model dtype; labels_dev int32 [B] (encoder) or [B, S] (decoder);
+ * loss_dev: one float (mean cross-entropy); logits_dev: nullable, float [B, n_out]
+ * (encoder) or [B*S, n_out] (decoder).  Returns RA_ERR_SHAPE if B or S exceed capacity. */
+ra_status ra_forward(ra_ctx* ctx, const void* x_dev, const int32_t* labels_dev, int32_t B,
+                     int32_t S, float* loss_dev, float* logits_dev, ra_stream_t stream);
+
+/* Backward ending at layer k (0-based; Algorithm 1 "Bw propagation ending at the
+ * (L - d + 1)-th adapter" is k = L - d).  Requires a preceding forward; k must satisfy
+ * L - d_forward <= k <= L - 1, else RA_ERR_NOT_SAVED (k too low) or RA_ERR_ARG.
+ * Writes gradients of the adapters of layers >= k and of the head (if trainable); the
+ * gradient buffers of layers < k are not touched.  Gradients are overwritten, not
+ * accumulated. */
+ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream);
+
+/* Adam step on the parameters the last backward produced gradients for (adapters of
+ * layers >= k_backward, and the head if trainable).  A parameter's step count starts at
+ * its first update.  Requires a backward since the last update, else RA_ERR_STATE. */
+ra_status ra_adapter_update(ra_ctx* ctx, const ra_adam_cfg* adam, ra_stream_t stream);
+
+/* Device pointer to a float32 gradient buffer (tests): layer 0..L-1 with RA_P_WDA..WUF,
+ * or layer -1 with RA_P_HEAD_W / RA_P_HEAD_B.  *n receives the element count.  The
+ * pointer stays valid while the memory is bound. */
+ra_status ra_get_grad(ra_ctx* ctx, int32_t layer, int32_t which, const float** dev_ptr,
+                      int64_t* n);
+
+/* Device pointer to a float32 trainable parameter (master copy), same indexing. */
+ra_status ra_get_param(ra_ctx* ctx, int32_t layer, int32_t which, const float** dev_ptr,
+                       int64_t* n);
+
+/* Checkpoint of the trainable state: masters, Adam moments, step counts and depth, as an
+ * opaque host blob of ra_trainable_state_bytes bytes.  Synchronises the device. */
+ra_status ra_trainable_state_bytes(const ra_ctx* ctx, size_t* n);
+ra_status ra_get_trainable(ra_ctx* ctx, void* host, size_t n);
+ra_status ra_set_trainable(ra_ctx* ctx, const void* host, size_t n);
+
+/* Host-side counters and sizes (no device access). */
+ra_status ra_get_stats(const ra_ctx* ctx, ra_stats* out);
+
+/* Synchronise the stream and report whether any bounded wait expired since the last
+ * call (RA_ERR_TIMEOUT), or a CUDA error occurred (RA_ERR_CUDA).  Clears the flag. */
+ra_status ra_sync_status(ra_ctx* ctx, ra_stream_t stream);
+
+/* Message of the last failing call on ctx (never null; "" if none). */
+const char* ra_last_error(const ra_ctx* ctx);
+
+/* Release the context (host memory only; bound device buffers stay the caller's). */
+void ra_destroy(ra_ctx* ctx);
+
+/* ---------------------------------------------------------------------------------------
+ * Stand-alone kernels, for testing each piece of the step in isolation.  No context.
+ * ------------------------------------------------------------------------------------- */
+
+/* C[M, N] = A[M, K] B[N, K]^T (+ bias[N]) on the tensor cores: bf16 operands, fp32
+ * accumulation, bf16 output.  Row-major, leading dimensions equal the row lengths.
+ * K % 8 == 0, N % 8 == 0 (16-byte rows).  bias_dev nullable (float).  gelu_out_dev
+ * nullable: if given, also writes GELU(C) there (the FFN-up epilogue of the frozen
+ * forward).  Returns RA_ERR_UNSUPPORTED on a device that is not sm_103. */
+ra_status ra_gemm_bf16(const void* A_dev, const void* B_dev, void* C_dev, int32_t M, int32_t N,
+                       int32_t K, const float* bias_dev, void* gelu_out_dev, ra_stream_t stream);
+
+/* Adapter backward of Eq. 1 for T rows (the in-kernel weight-gradient reduction of the
+ * step), float32 throughout.  g_dev [T, H] = dLoss/d(adapter output); h_dev [T, H] the
+ * adapter input; z_dev [T, m] = h W_down saved by the forward; W_down [H, m], W_up [m, H].
+ * Writes dW_down [H, m], dW_up [m, H] and, if dh_dev is not null, dh [T, H].
+ * scratch_dev: caller scratch of ra_adapter_backward_scratch_bytes(T, H, m) bytes.
+ * The result is deterministic (fixed reduction order). */
+ra_status ra_adapter_backward(const float* g_dev, const float* h_dev, const float* z_dev,
+                              const float* W_down_dev, const float* W_up_dev, int32_t T,
+                              int32_t H, int32_t m, float* dW_down_dev, float* dW_up_dev,
+                              float* dh_dev, void* scratch_dev, size_t scratch_bytes,
+                              ra_stream_t stream);
+size_t ra_adapter_backward_scratch_bytes(int32_t T, int32_t H, int32_t m);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* RINGADA_H */

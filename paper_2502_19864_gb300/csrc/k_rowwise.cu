@@ -1,0 +1,740 @@
+// k_rowwise.cu -- row-wise fused kernels of the step: adapters (Eq. 1) fused with the
+// residual add and the block's normalisation, the adapter backward with its in-kernel
+// deterministic weight-gradient reduction, LayerNorm / RMSNorm, the heads and their
+// cross-entropy, and Adam.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace ra {
+namespace {
+
+template <typename T>
+__device__ __forceinline__ float ldf(const void* p, int64_t i) {
+  return to_f(reinterpret_cast<const T*>(p)[i]);
+}
+template <typename T>
+__device__ __forceinline__ void stf(void* p, int64_t i, float v) {
+  reinterpret_cast<T*>(p)[i] = from_f<T>(v);
+}
+
+constexpr int WARPS = 8;
+constexpr int RPW = 2;             // rows per warp in the adapter row kernels
+constexpr int ROWS = WARPS * RPW;  // rows per CTA
+constexpr int MAXM = 128;          // adapter bottleneck upper bound
+constexpr int MC = MAXM / 32;      // bottleneck columns per lane
+
+// ---------------------------------------------------------------------------------------
+// Adapter forward (Eq. 1) + residual + norm.  Warp w owns rows (blockIdx*ROWS + w*RPW + r).
+// smem: rows [ROWS][H] f32 (adapter input, then the pre-norm sum), s [ROWS][m] f32.
+// ---------------------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(WARPS * 32) adapter_fwd_kernel(AdapterFwdArgs a) {
+  extern __shared__ float sm[];
+  const int H = a.H, m = a.m;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float* rows = sm + (size_t)warp * RPW * H;
+  float* sv = sm + (size_t)ROWS * H + warp * RPW * MAXM;
+  const int t0 = blockIdx.x * ROWS + warp * RPW;
+
+  for (int r = 0; r < RPW; ++r) {
+    int t = t0 + r;
+    for (int i = lane; i < H; i += 32) rows[r * H + i] = t < a.T ? ldf<T>(a.a, (int64_t)t * H + i) : 0.f;
+  }
+  __syncwarp();
+  // z = a W_down  (lanes over bottleneck columns j = lane + 32c)
+  float z[RPW][MC];
+#pragma unroll
+  for (int r = 0; r < RPW; ++r)
+#pragma unroll
+    for (int c = 0; c < MC; ++c) z[r][c] = 0.f;
+  for (int i = 0; i < H; ++i) {
+    float w[MC];
+#pragma unroll
+    for (int c = 0; c < MC; ++c) {
+      int j = lane + 32 * c;
+      w[c] = j < m ? a.Wd[(int64_t)i * m + j] : 0.f;
+    }
+#pragma unroll
+    for (int r = 0; r < RPW; ++r) {
+      float x = rows[r * H + i];
+#pragma unroll
+      for (int c = 0; c < MC; ++c) z[r][c] = fmaf(x, w[c], z[r][c]);
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < RPW; ++r) {
+    int t = t0 + r;
+#pragma unroll
+    for (int c = 0; c < MC; ++c) {
+      int j = lane + 32 * c;
+      if (j < m) {
+        sv[r * MAXM + j] = gelu_f(z[r][c]);
+        if (a.z && t < a.T) a.z[(int64_t)t * m + j] = z[r][c];
+      }
+    }
+  }
+  __syncwarp();
+  // out = a + GELU(z) W_up, in chunks of 256 columns (lanes over i = i0 + lane + 32cc)
+  for (int i0 = 0; i0 < H; i0 += 256) {
+    float acc[RPW][8];
+#pragma unroll
+    for (int r = 0; r < RPW; ++r)
+#pragma unroll
+      for (int cc = 0; cc < 8; ++cc) acc[r][cc] = 0.f;
+    for (int j = 0; j < m; ++j) {
+      float w[8];
+#pragma unroll
+      for (int cc = 0; cc < 8; ++cc) {
+        int i = i0 + lane + 32 * cc;
+        w[cc] = i < H ? a.Wu[(int64_t)j * H + i] : 0.f;
+      }
+#pragma unroll
+      for (int r = 0; r < RPW; ++r) {
+        float s = sv[r * MAXM + j];
+#pragma unroll
+        for (int cc = 0; cc < 8; ++cc) acc[r][cc] = fmaf(s, w[cc], acc[r][cc]);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < RPW; ++r) {
+      int t = t0 + r;
+#pragma unroll
+      for (int cc = 0; cc < 8; ++cc) {
+        int i = i0 + lane + 32 * cc;
+        if (i < H) {
+          float res = 0.f;
+          if (t < a.T)
+            res = a.decoder ? reinterpret_cast<const float*>(a.resid)[(int64_t)t * H + i]
+                            : ldf<T>(a.resid, (int64_t)t * H + i);
+          rows[r * H + i] = res + rows[r * H + i] + acc[r][cc];
+        }
+      }
+    }
+  }
+  __syncwarp();
+  // normalisation of the residual sum
+  for (int r = 0; r < RPW; ++r) {
+    int t = t0 + r;
+    if (t >= a.T) break;
+    float* v = rows + r * H;
+    if (!a.decoder) {
+      float s = 0.f;
+      for (int i = lane; i < H; i += 32) s += v[i];
+      float mu = warp_sum(s) / H;
+      float q = 0.f;
+      for (int i = lane; i < H; i += 32) { float d = v[i] - mu; q += d * d; }
+      float rstd = rsqrtf(warp_sum(q) / H + a.eps);
+      for (int i = lane; i < H; i += 32) {
+        float xh = (v[i] - mu) * rstd;
+        stf<T>(a.y, (int64_t)t * H + i, xh * a.gamma[i] + a.beta[i]);
+        if (a.xhat) stf<T>(a.xhat, (int64_t)t * H + i, xh);
+      }
+      if (a.rstd && lane == 0) a.rstd[t] = rstd;
+    } else {
+      float q = 0.f;
+      for (int i = lane; i < H; i += 32) q += v[i] * v[i];
+      float rstd = rsqrtf(warp_sum(q) / H + a.eps);
+      for (int i = lane; i < H; i += 32) {
+        a.x_out[(int64_t)t * H + i] = v[i];
+        stf<T>(a.y, (int64_t)t * H + i, v[i] * rstd * a.gamma[i]);
+      }
+      if (a.rstd && lane == 0) a.rstd[t] = rstd;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------------------
+// Adapter backward, row part: dz = (g W_up^T) * GELU'(z), dh = g + dz W_down^T
+// ---------------------------------------------------------------------------------------
+template <typename TO>
+__global__ void __launch_bounds__(WARPS * 32) adapter_bwd_rows_kernel(AdapterBwdArgs a) {
+  extern __shared__ float sm[];
+  const int H = a.H, m = a.m;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float* rows = sm + (size_t)warp * RPW * H;
+  float* dzs = sm + (size_t)ROWS * H + warp * RPW * MAXM;
+  const int t0 = blockIdx.x * ROWS + warp * RPW;
+  for (int r = 0; r < RPW; ++r) {
+    int t = t0 + r;
+    for (int i = lane; i < H; i += 32) rows[r * H + i] = t < a.T ? a.g[(int64_t)t * H + i] : 0.f;
+  }
+  __syncwarp();
+  float ds[RPW][MC];
+#pragma unroll
+  for (int r = 0; r < RPW; ++r)
+#pragma unroll
+    for (int c = 0; c < MC; ++c) ds[r][c] = 0.f;
+  for (int i = 0; i < H; ++i) {
+    float w[MC];
+#pragma unroll
+    for (int c = 0; c < MC; ++c) {
+      int j = lane + 32 * c;
+      w[c] = j < m ? a.WuT[(int64_t)i * m + j] : 0.f;
+    }
+#pragma unroll
+    for (int r = 0; r < RPW; ++r) {
+      float x = rows[r * H + i];
+#pragma unroll
+      for (int c = 0; c < MC; ++c) ds[r][c] = fmaf(x, w[c], ds[r][c]);
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < RPW; ++r) {
+    int t = t0 + r;
+#pragma unroll
+    for (int c = 0; c < MC; ++c) {
+      int j = lane + 32 * c;
+      if (j < m) {
+        float dz = 0.f;
+        if (t < a.T) {
+          dz = ds[r][c] * gelu_grad_f(a.z[(int64_t)t * m + j]);
+          a.dz[(int64_t)t * m + j] = dz;
+        }
+        dzs[r * MAXM + j] = dz;
+      }
+    }
+  }
+  __syncwarp();
+  if (!a.dh) return;
+  for (int i0 = 0; i0 < H; i0 += 256) {
+    float acc[RPW][8];
+#pragma unroll
+    for (int r = 0; r < RPW; ++r)
+#pragma unroll
+      for (int cc = 0; cc < 8; ++cc) acc[r][cc] = 0.f;
+    for (int j = 0; j < m; ++j) {
+      float w[8];
+#pragma unroll
+      for (int cc = 0; cc < 8; ++cc) {
+        int i = i0 + lane + 32 * cc;
+        w[cc] = i < H ? a.WdT[(int64_t)j * H + i] : 0.f;
+      }
+#pragma unroll
+      for (int r = 0; r < RPW; ++r) {
+        float d = dzs[r * MAXM + j];
+#pragma unroll
+        for (int cc = 0; cc < 8; ++cc) acc[r][cc] = fmaf(d, w[cc], acc[r][cc]);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < RPW; ++r) {
+      int t = t0 + r;
+      if (t >= a.T) continue;
+#pragma unroll
+      for (int cc = 0; cc < 8; ++cc) {
+        int i = i0 + lane + 32 * cc;
+        if (i < H) stf<TO>(a.dh, (int64_t)t * H + i, rows[r * H + i] + acc[r][cc]);
+      }
+    }
+  }
+}
+
+// Weight-gradient partials over a chunk of rows:
+//   pWu[c][j][i]  = sum_{t in chunk c} GELU(z[t, j]) g[t, i]          (dW_up  = GELU(z)^T g)
+//   pWdT[c][j][i] = sum_{t in chunk c} h[t, i] dz[t, j]                (dW_down^T = dz^T h)
+// CTA: 64 columns i x all m; thread owns i = tid % 64, j = tid/64 + 4c.
+constexpr int DW_COLS = 64, DW_ROWS = 16;
+template <typename T>
+__global__ void __launch_bounds__(256) adapter_dw_partial_kernel(AdapterBwdArgs a, int chunk) {
+  __shared__ float gS[DW_ROWS][DW_COLS], hS[DW_ROWS][DW_COLS];
+  __shared__ float sS[DW_ROWS][MAXM], dzS[DW_ROWS][MAXM];
+  const int H = a.H, m = a.m;
+  const int i0 = blockIdx.x * DW_COLS, c = blockIdx.y;
+  const int tid = threadIdx.x, il = tid % DW_COLS, jg = tid / DW_COLS;
+  const int tb = c * chunk, te = min(a.T, tb + chunk);
+  float aWu[MAXM / 4], aWd[MAXM / 4];
+#pragma unroll
+  for (int q = 0; q < MAXM / 4; ++q) { aWu[q] = 0.f; aWd[q] = 0.f; }
+  for (int t0 = tb; t0 < te; t0 += DW_ROWS) {
+    __syncthreads();
+    for (int e = tid; e < DW_ROWS * DW_COLS; e += 256) {
+      int r = e / DW_COLS, i = e % DW_COLS, t = t0 + r;
+      bool in = t < te && i0 + i < H;
+      gS[r][i] = in ? a.g[(int64_t)t * H + i0 + i] : 0.f;
+      hS[r][i] = in ? ldf<T>(a.h, (int64_t)t * H + i0 + i) : 0.f;
+    }
+    for (int e = tid; e < DW_ROWS * MAXM; e += 256) {
+      int r = e / MAXM, j = e % MAXM, t = t0 + r;
+      bool in = t < te && j < m;
+      sS[r][j] = in ? gelu_f(a.z[(int64_t)t * m + j]) : 0.f;
+      dzS[r][j] = in ? a.dz[(int64_t)t * m + j] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll 4
+    for (int r = 0; r < DW_ROWS; ++r) {
+      float gv = gS[r][il], hv = hS[r][il];
+#pragma unroll
+      for (int q = 0; q < MAXM / 4; ++q) {
+        int j = jg + 4 * q;
+        aWu[q] = fmaf(sS[r][j], gv, aWu[q]);
+        aWd[q] = fmaf(dzS[r][j], hv, aWd[q]);
+      }
+    }
+  }
+  if (i0 + il >= H) return;
+  float* pWu = a.partials + (size_t)c * 2 * H * m;
+  float* pWdT = pWu + (size_t)H * m;
+#pragma unroll
+  for (int q = 0; q < MAXM / 4; ++q) {
+    int j = jg + 4 * q;
+    if (j < m) {
+      pWu[(size_t)j * H + i0 + il] = aWu[q];
+      pWdT[(size_t)j * H + i0 + il] = aWd[q];
+    }
+  }
+}
+
+// Fixed-order sum of the partials: dW_up[j][i] and dW_down[i][j].
+__global__ void adapter_dw_reduce_kernel(const float* partials, int nchunk, int H, int m,
+                                         float* dWd, float* dWu) {
+  int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  int64_t n = (int64_t)H * m;
+  if (e >= 2 * n) return;
+  bool up = e < n;
+  int64_t idx = up ? e : e - n;  // index into [m][H]
+  float s = 0.f;
+  for (int c = 0; c < nchunk; ++c) s += partials[(size_t)c * 2 * n + (up ? 0 : n) + idx];
+  if (up) dWu[idx] = s;
+  else {
+    int j = (int)(idx / H), i = (int)(idx % H);
+    dWd[(int64_t)i * m + j] = s;
+  }
+}
+
+// Chunk count of the weight-gradient reduction: a pure function of (T, H), so the scratch
+// size planned on the host and the grid launched on any device agree, and the reduction
+// order (hence the bits of the result) does not depend on the device.
+constexpr int kDwTargetCtas = 304;
+int dw_chunks(int T, int H) {
+  int colblocks = (H + DW_COLS - 1) / DW_COLS;
+  int want = (kDwTargetCtas + colblocks - 1) / colblocks;
+  int maxc = (T + DW_ROWS - 1) / DW_ROWS;
+  return max(1, min(min(want, 64), maxc));
+}
+
+// ---------------------------------------------------------------------------------------
+// Norms
+// ---------------------------------------------------------------------------------------
+template <typename T>
+__global__ void layernorm_bwd_kernel(const float* dy, const void* xhat, const float* rstd,
+                                     const float* gamma, float* ds, int Tn, int H) {
+  int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (t >= Tn) return;
+  float s1 = 0.f, s2 = 0.f;
+  for (int i = lane; i < H; i += 32) {
+    float gy = dy[(int64_t)t * H + i] * gamma[i];
+    float xh = ldf<T>(xhat, (int64_t)t * H + i);
+    s1 += gy;
+    s2 += gy * xh;
+  }
+  s1 = warp_sum(s1) / H;
+  s2 = warp_sum(s2) / H;
+  float r = rstd[t];
+  for (int i = lane; i < H; i += 32) {
+    float gy = dy[(int64_t)t * H + i] * gamma[i];
+    float xh = ldf<T>(xhat, (int64_t)t * H + i);
+    ds[(int64_t)t * H + i] = r * (gy - s1 - xh * s2);
+  }
+}
+
+template <typename TX, typename TN>
+__global__ void rmsnorm_fwd_kernel(const void* x, const float* gamma, float eps, void* n,
+                                   float* rstd, float* xf, int Tn, int H) {
+  int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (t >= Tn) return;
+  float q = 0.f;
+  for (int i = lane; i < H; i += 32) { float v = ldf<TX>(x, (int64_t)t * H + i); q += v * v; }
+  float r = rsqrtf(warp_sum(q) / H + eps);
+  for (int i = lane; i < H; i += 32) {
+    float v = ldf<TX>(x, (int64_t)t * H + i);
+    stf<TN>(n, (int64_t)t * H + i, v * r * gamma[i]);
+    if (xf) xf[(int64_t)t * H + i] = v;
+  }
+  if (rstd && lane == 0) rstd[t] = r;
+}
+
+__global__ void rmsnorm_bwd_kernel(const float* dy, const float* x, const float* rstd,
+                                   const float* gamma, const float* resid, float* dx, int Tn,
+                                   int H) {
+  int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (t >= Tn) return;
+  float s = 0.f;
+  for (int i = lane; i < H; i += 32) s += dy[(int64_t)t * H + i] * gamma[i] * x[(int64_t)t * H + i];
+  s = warp_sum(s) / H;
+  float r = rstd[t];
+  for (int i = lane; i < H; i += 32) {
+    int64_t e = (int64_t)t * H + i;
+    float v = r * dy[e] * gamma[i] - x[e] * r * r * r * s;
+    dx[e] = (resid ? resid[e] : 0.f) + v;
+  }
+}
+
+// ---------------------------------------------------------------------------------------
+// Heads
+// ---------------------------------------------------------------------------------------
+constexpr int MAXC = 32, MAXB = 256;
+// forward: logits = y[b, 0, :] Wh^T + bh, mean CE, dlogits = (softmax - onehot) / B
+template <typename T>
+__global__ void __launch_bounds__(256) encoder_head_fwd_kernel(const void* y, const float* Wh,
+    const float* bh, const int32_t* labels, int B, int S, int H, int C, float* loss,
+    float* logits_out, float* dlogits, unsigned* err) {
+  __shared__ float lg[MAXB * MAXC];
+  __shared__ float red[MAXB];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int pc = warp; pc < B * C; pc += 8) {
+    int b = pc / C, c = pc % C;
+    float s = 0.f;
+    for (int i = lane; i < H; i += 32) s += ldf<T>(y, (int64_t)b * S * H + i) * Wh[(int64_t)c * H + i];
+    s = warp_sum(s);
+    if (lane == 0) lg[b * C + c] = s + bh[c];
+  }
+  __syncthreads();
+  for (int b = threadIdx.x; b < B; b += blockDim.x) {
+    float mx = -INFINITY;
+    for (int c = 0; c < C; ++c) mx = fmaxf(mx, lg[b * C + c]);
+    float se = 0.f;
+    for (int c = 0; c < C; ++c) se += expf(lg[b * C + c] - mx);
+    float lse = mx + logf(se);
+    int lab = labels[b];
+    if (lab < 0 || lab >= C) { set_dev_error(err, RA_DEVERR_BOUNDS); lab = 0; }
+    red[b] = lse - lg[b * C + lab];
+    for (int c = 0; c < C; ++c) {
+      if (logits_out) logits_out[b * C + c] = lg[b * C + c];
+      float p = expf(lg[b * C + c] - lse);
+      dlogits[b * C + c] = (p - (c == lab ? 1.f : 0.f)) / B;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+    for (int b = 0; b < B; ++b) s += red[b];
+    *loss = s / B;
+  }
+}
+
+// backward: dWh = dlogits^T cls, dbh = sum_b dlogits, dy[b, 0, :] = dlogits Wh
+template <typename T>
+__global__ void __launch_bounds__(256) encoder_head_bwd_kernel(const void* y, const float* Wh,
+    const float* dlogits, int B, int S, int H, int C, float* dWh, float* dbh, float* dy) {
+  __shared__ float lg[MAXB * MAXC];
+  for (int e = threadIdx.x; e < B * C; e += blockDim.x) lg[e] = dlogits[e];
+  __syncthreads();
+  int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < H) {
+    for (int c = 0; c < C; ++c) {
+      float s = 0.f;
+      for (int b = 0; b < B; ++b) s += lg[b * C + c] * ldf<T>(y, (int64_t)b * S * H + i);
+      if (dWh) dWh[(int64_t)c * H + i] = s;
+    }
+    for (int b = 0; b < B; ++b) {
+      float s = 0.f;
+      for (int c = 0; c < C; ++c) s += lg[b * C + c] * Wh[(int64_t)c * H + i];
+      dy[(int64_t)b * S * H + i] = s;
+    }
+  }
+  if (dbh && blockIdx.x == 0 && threadIdx.x < C) {
+    float s = 0.f;
+    for (int b = 0; b < B; ++b) s += lg[b * C + threadIdx.x];
+    dbh[threadIdx.x] = s;
+  }
+}
+
+// one CTA per row: in-place dlogits = (softmax - onehot) / T
+template <typename T>
+__global__ void __launch_bounds__(256) vocab_ce_kernel(void* logits, int ld,
+    const int32_t* labels, int Tn, int V, float* row_loss, float* logits_out, unsigned* err) {
+  __shared__ float red[8];
+  const int t = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  T* row = reinterpret_cast<T*>(logits) + (int64_t)t * ld;
+  float mx = -INFINITY;
+  for (int j = threadIdx.x; j < V; j += 256) {
+    float v = to_f(row[j]);
+    mx = fmaxf(mx, v);
+    if (logits_out) logits_out[(int64_t)t * V + j] = v;
+  }
+  mx = warp_max(mx);
+  if (lane == 0) red[warp] = mx;
+  __syncthreads();
+  mx = red[0];
+  for (int w = 1; w < 8; ++w) mx = fmaxf(mx, red[w]);
+  __syncthreads();
+  float se = 0.f;
+  for (int j = threadIdx.x; j < V; j += 256) se += expf(to_f(row[j]) - mx);
+  se = warp_sum(se);
+  if (lane == 0) red[warp] = se;
+  __syncthreads();
+  se = 0.f;
+  for (int w = 0; w < 8; ++w) se += red[w];
+  float lse = mx + logf(se);
+  int lab = labels[t];
+  if (lab < 0 || lab >= V) {
+    if (threadIdx.x == 0) set_dev_error(err, RA_DEVERR_BOUNDS);
+    lab = 0;
+  }
+  float zl = to_f(row[lab]);
+  __syncthreads();
+  if (threadIdx.x == 0) row_loss[t] = lse - zl;
+  float invT = 1.f / Tn;
+  for (int j = threadIdx.x; j < V; j += 256) {
+    float p = expf(to_f(row[j]) - lse);
+    row[j] = from_f<T>((p - (j == lab ? 1.f : 0.f)) * invT);
+  }
+}
+
+__global__ void __launch_bounds__(256) mean_kernel(const float* v, int n, float* out) {
+  __shared__ float red[256];
+  float s = 0.f;
+  for (int i = threadIdx.x; i < n; i += 256) s += v[i];
+  red[threadIdx.x] = s;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *out = red[0] / n;
+}
+
+// ---------------------------------------------------------------------------------------
+// Adam
+// ---------------------------------------------------------------------------------------
+__global__ void adam_kernel(AdamArgs a) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= a.n) return;
+  int s = (int)(i / a.seg_len);
+  if (s >= a.n_seg) s = a.n_seg - 1;
+  float t = (float)(a.steps[s] + 1);
+  float g = a.g[i];
+  float m = a.beta1 * a.m[i] + (1.f - a.beta1) * g;
+  float v = a.beta2 * a.v[i] + (1.f - a.beta2) * g * g;
+  a.m[i] = m;
+  a.v[i] = v;
+  float bc1 = 1.f - powf(a.beta1, t);
+  float bc2 = 1.f - powf(a.beta2, t);
+  float denom = sqrtf(v) / sqrtf(bc2) + a.eps;
+  a.p[i] -= (a.lr / bc1) * m / denom;
+}
+
+__global__ void bump_kernel(int32_t* steps, int n) {
+  int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) steps[i] += 1;
+}
+
+// ---------------------------------------------------------------------------------------
+// utilities
+// ---------------------------------------------------------------------------------------
+template <typename T>
+__global__ void convert_kernel(const float* src, void* dst, int64_t n) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) stf<T>(dst, i, src[i]);
+}
+
+template <typename T>
+__global__ void transpose_kernel(const float* src, void* dst, int rows, int cols, int ld_dst) {
+  __shared__ float tile[32][33];
+  int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  for (int y = threadIdx.y; y < 32; y += 8) {
+    int r = r0 + y, c = c0 + threadIdx.x;
+    tile[y][threadIdx.x] = (r < rows && c < cols) ? src[(int64_t)r * cols + c] : 0.f;
+  }
+  __syncthreads();
+  for (int y = threadIdx.y; y < 32; y += 8) {
+    int c = c0 + y, r = r0 + threadIdx.x;
+    if (c < cols && r < rows) stf<T>(dst, (int64_t)c * ld_dst + r, tile[threadIdx.x][y]);
+  }
+}
+
+// packed gate/up row of source row r of part (0 = gate, 1 = up): 64-row blocks alternate
+__device__ __forceinline__ int64_t packed_row(int r, int part) {
+  return (int64_t)(r >> 6) * 128 + part * 64 + (r & 63);
+}
+template <typename T>
+__global__ void pack_rows_kernel(const float* src, void* dst, int R, int C, int part, int transposed) {
+  int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= (int64_t)R * C) return;
+  int r = (int)(e / C), c = (int)(e % C);
+  int64_t pr = packed_row(r, part);
+  if (transposed) stf<T>(dst, (int64_t)c * (2 * R) + pr, src[e]);
+  else stf<T>(dst, pr * C + c, src[e]);
+}
+
+// transposed copies of the adapter matrices of layers [l0, l1): for each layer the four
+// matrices WdA [H,m], WuA [m,H], WdF [H,m], WuF [m,H] (contiguous, 4Hm per layer) go to
+// WdT [m,H], WuT [H,m], ... at the same offsets of PT.
+__global__ void adapter_transpose_kernel(const float* P, float* PT, int H, int m) {
+  int layer = blockIdx.z >> 2, mat = blockIdx.z & 3;
+  int64_t base = (int64_t)layer * 4 * H * m + (int64_t)mat * H * m;
+  int rows = (mat & 1) ? m : H, cols = (mat & 1) ? H : m;
+  int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= (int64_t)rows * cols) return;
+  int r = (int)(e / cols), c = (int)(e % cols);
+  PT[base + (int64_t)c * rows + r] = P[base + e];
+}
+
+__global__ void fill_kernel(float* dst, float v, int64_t n) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) dst[i] = v;
+}
+
+inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1) / per); }
+
+}  // namespace
+
+// =========================================================================================
+cudaError_t adapter_fwd(const AdapterFwdArgs& a, cudaStream_t st) {
+  if (a.m > MAXM || a.m <= 0) return cudaErrorInvalidValue;
+  size_t smem = ((size_t)ROWS * a.H + ROWS * MAXM) * sizeof(float);
+  unsigned grid = blocks_for(a.T, ROWS);
+  if (a.dtype == DT_BF16) {
+    cudaFuncSetAttribute(adapter_fwd_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    adapter_fwd_kernel<bf16><<<grid, WARPS * 32, smem, st>>>(a);
+  } else {
+    cudaFuncSetAttribute(adapter_fwd_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    adapter_fwd_kernel<float><<<grid, WARPS * 32, smem, st>>>(a);
+  }
+  return cudaGetLastError();
+}
+
+size_t adapter_bwd_partials_floats(int T, int H, int m) {
+  return (size_t)dw_chunks(T, H) * 2 * H * m;
+}
+
+cudaError_t adapter_bwd(const AdapterBwdArgs& a, cudaStream_t st) {
+  if (a.m > MAXM || a.m <= 0) return cudaErrorInvalidValue;
+  size_t smem = ((size_t)ROWS * a.H + ROWS * MAXM) * sizeof(float);
+  unsigned grid = blocks_for(a.T, ROWS);
+  if (a.dh_dtype == DT_BF16) {
+    cudaFuncSetAttribute(adapter_bwd_rows_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    adapter_bwd_rows_kernel<bf16><<<grid, WARPS * 32, smem, st>>>(a);
+  } else {
+    cudaFuncSetAttribute(adapter_bwd_rows_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    adapter_bwd_rows_kernel<float><<<grid, WARPS * 32, smem, st>>>(a);
+  }
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  int nchunk = dw_chunks(a.T, a.H);
+  int chunk = (a.T + nchunk - 1) / nchunk;
+  dim3 g2((a.H + DW_COLS - 1) / DW_COLS, nchunk);
+  if (a.dtype == DT_BF16) adapter_dw_partial_kernel<bf16><<<g2, 256, 0, st>>>(a, chunk);
+  else adapter_dw_partial_kernel<float><<<g2, 256, 0, st>>>(a, chunk);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  int64_t n = 2LL * a.H * a.m;
+  adapter_dw_reduce_kernel<<<blocks_for(n, 256), 256, 0, st>>>(a.partials, nchunk, a.H, a.m, a.dWd, a.dWu);
+  return cudaGetLastError();
+}
+
+cudaError_t layernorm_bwd(const float* dy, const void* xhat, const float* rstd,
+                          const float* gamma, float* ds, int T, int H, int dtype,
+                          cudaStream_t st) {
+  unsigned grid = blocks_for((int64_t)T * 32, 256);
+  if (dtype == DT_BF16) layernorm_bwd_kernel<bf16><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H);
+  else layernorm_bwd_kernel<float><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H);
+  return cudaGetLastError();
+}
+
+cudaError_t rmsnorm_fwd(const void* x, int x_dtype, const float* gamma, float eps, void* n,
+                        int n_dtype, float* rstd, float* x_f32_out, int T, int H,
+                        cudaStream_t st) {
+  unsigned grid = blocks_for((int64_t)T * 32, 256);
+  if (x_dtype == DT_BF16 && n_dtype == DT_BF16)
+    rmsnorm_fwd_kernel<bf16, bf16><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H);
+  else if (x_dtype == DT_F32 && n_dtype == DT_BF16)
+    rmsnorm_fwd_kernel<float, bf16><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H);
+  else if (x_dtype == DT_BF16)
+    rmsnorm_fwd_kernel<bf16, float><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H);
+  else
+    rmsnorm_fwd_kernel<float, float><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H);
+  return cudaGetLastError();
+}
+
+cudaError_t rmsnorm_bwd(const float* dy, const float* x, const float* rstd, const float* gamma,
+                        const float* resid, float* dx, int T, int H, cudaStream_t st) {
+  rmsnorm_bwd_kernel<<<blocks_for((int64_t)T * 32, 256), 256, 0, st>>>(dy, x, rstd, gamma, resid, dx, T, H);
+  return cudaGetLastError();
+}
+
+cudaError_t encoder_head_fwd(const void* y, int dtype, const float* Wh, const float* bh,
+                             const int32_t* labels, int B, int S, int H, int C, float* loss,
+                             float* logits_out, float* dlogits, unsigned* err, cudaStream_t st) {
+  if (C > MAXC || B > MAXB) return cudaErrorInvalidValue;
+  if (dtype == DT_BF16)
+    encoder_head_fwd_kernel<bf16><<<1, 256, 0, st>>>(y, Wh, bh, labels, B, S, H, C, loss, logits_out, dlogits, err);
+  else
+    encoder_head_fwd_kernel<float><<<1, 256, 0, st>>>(y, Wh, bh, labels, B, S, H, C, loss, logits_out, dlogits, err);
+  return cudaGetLastError();
+}
+
+cudaError_t encoder_head_bwd(const void* y, int dtype, const float* Wh, const float* dlogits,
+                             int B, int S, int H, int C, float* dWh, float* dbh, float* dy,
+                             cudaStream_t st) {
+  if (C > MAXC || B > MAXB) return cudaErrorInvalidValue;
+  unsigned grid = blocks_for(H, 256);
+  if (dtype == DT_BF16)
+    encoder_head_bwd_kernel<bf16><<<grid, 256, 0, st>>>(y, Wh, dlogits, B, S, H, C, dWh, dbh, dy);
+  else
+    encoder_head_bwd_kernel<float><<<grid, 256, 0, st>>>(y, Wh, dlogits, B, S, H, C, dWh, dbh, dy);
+  return cudaGetLastError();
+}
+
+cudaError_t vocab_ce(void* logits, int dtype, int ld, const int32_t* labels, int T, int V,
+                     float* row_loss, float* loss, float* logits_out, unsigned* err,
+                     cudaStream_t st) {
+  if (dtype == DT_BF16)
+    vocab_ce_kernel<bf16><<<T, 256, 0, st>>>(logits, ld, labels, T, V, row_loss, logits_out, err);
+  else
+    vocab_ce_kernel<float><<<T, 256, 0, st>>>(logits, ld, labels, T, V, row_loss, logits_out, err);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  mean_kernel<<<1, 256, 0, st>>>(row_loss, T, loss);
+  return cudaGetLastError();
+}
+
+cudaError_t adam_update(const AdamArgs& a, cudaStream_t st) {
+  if (a.n <= 0) return cudaSuccess;
+  adam_kernel<<<blocks_for(a.n, 256), 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t adam_bump(int32_t* steps, int n, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  bump_kernel<<<blocks_for(n, 128), 128, 0, st>>>(steps, n);
+  return cudaGetLastError();
+}
+
+cudaError_t convert_f32(const float* src, void* dst, int dst_dtype, int64_t n, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  if (dst_dtype == DT_BF16) convert_kernel<bf16><<<blocks_for(n, 256), 256, 0, st>>>(src, dst, n);
+  else convert_kernel<float><<<blocks_for(n, 256), 256, 0, st>>>(src, dst, n);
+  return cudaGetLastError();
+}
+
+cudaError_t transpose_f32(const float* src, void* dst, int dst_dtype, int rows, int cols,
+                          int ld_dst, cudaStream_t st) {
+  dim3 grid((cols + 31) / 32, (rows + 31) / 32), blk(32, 8);
+  if (dst_dtype == DT_BF16) transpose_kernel<bf16><<<grid, blk, 0, st>>>(src, dst, rows, cols, ld_dst);
+  else transpose_kernel<float><<<grid, blk, 0, st>>>(src, dst, rows, cols, ld_dst);
+  return cudaGetLastError();
+}
+
+cudaError_t pack_rows(const float* src, void* dst, int dst_dtype, int R, int C, int part,
+                      bool transposed, cudaStream_t st) {
+  int64_t n = (int64_t)R * C;
+  if (dst_dtype == DT_BF16) pack_rows_kernel<bf16><<<blocks_for(n, 256), 256, 0, st>>>(src, dst, R, C, part, transposed);
+  else pack_rows_kernel<float><<<blocks_for(n, 256), 256, 0, st>>>(src, dst, R, C, part, transposed);
+  return cudaGetLastError();
+}
+
+cudaError_t adapter_transpose(const float* P, float* PT, int n_layers, int H, int m, cudaStream_t st) {
+  if (n_layers <= 0) return cudaSuccess;
+  dim3 grid(blocks_for((int64_t)H * m, 256), 1, 4 * n_layers);
+  adapter_transpose_kernel<<<grid, 256, 0, st>>>(P, PT, H, m);
+  return cudaGetLastError();
+}
+
+cudaError_t fill_f32(float* dst, float v, int64_t n, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  fill_kernel<<<blocks_for(n, 256), 256, 0, st>>>(dst, v, n);
+  return cudaGetLastError();
+}
+
+}  // namespace ra

@@ -1,0 +1,174 @@
+// kernels.h -- host-side launchers of the libringada kernels (internal, not ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace ra {
+
+enum DType : int { DT_F32 = 0, DT_BF16 = 1 };
+
+inline size_t dtype_size(int dt) { return dt == DT_BF16 ? 2 : 4; }
+
+// ---------------------------------------------------------------------------------------
+// GEMM  C[M, N] = A[M, K] * B[N, K]^T with a fused epilogue.  A and B share a dtype and are
+// K-major (row-major, K contiguous).  The accumulator is fp32.
+// ---------------------------------------------------------------------------------------
+enum EpiKind : int {
+  EPI_STORE = 0,     // C = acc (+ bias)
+  EPI_BIAS_GELU,     // C = acc + bias (pre-activation u, optional), C2 = GELU(u)
+  EPI_DGELU,         // C = acc * GELU'(aux)           (aux = saved u)
+  EPI_RESID,         // C = acc + aux                  (aux = fp32 residual)
+  EPI_DSWIGLU,       // N = F: acc is d(h) at col j; aux = packed [gate|up] [M, 2F];
+                     // C (width 2F, packed like aux) gets d(gate), d(up)
+  EPI_SWIGLU,        // N = 2F packed [gate|up]: C = packed pre-activations (optional),
+                     // C2 [M, F] = silu(gate) * up
+};
+
+struct GemmArgs {
+  const void* A = nullptr; int lda = 0;
+  const void* B = nullptr; int ldb = 0;
+  int M = 0, N = 0, K = 0;
+  int in_dtype = DT_F32;
+  int epi = EPI_STORE;
+  void* C = nullptr; int ldc = 0; int c_dtype = DT_F32;
+  const float* bias = nullptr;
+  void* C2 = nullptr; int ldc2 = 0; int c2_dtype = DT_F32;
+  const void* aux = nullptr; int ldaux = 0; int aux_dtype = DT_F32;
+  unsigned* err = nullptr;
+};
+
+// Returns a cudaError_t from the launch (cudaSuccess if enqueued).
+cudaError_t gemm(const GemmArgs& a, cudaStream_t st);
+// tcgen05 path; returns cudaErrorNotSupported if the shape/dtype is not handled.
+cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st);
+cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st);
+// Whether the tcgen05 path is usable on the current device (sm_103).
+bool tc_available();
+int device_sm_count();
+
+// ---------------------------------------------------------------------------------------
+// Attention (per (batch, head); token t = b*S + s; head hh at columns hh*dh of q/k/v).
+// ---------------------------------------------------------------------------------------
+struct AttnArgs {
+  const void* qkv = nullptr;  // [T, 3H]: q | k | v
+  int B = 0, S = 0, n_heads = 0, head_dim = 0;
+  int dtype = DT_F32;
+  bool causal = false;
+  bool rope = false;          // rotate-half RoPE on q and k inside the kernel
+  float rope_theta = 10000.f;
+  float scale = 1.f;
+  void* O = nullptr;          // [T, H]
+  float* lse = nullptr;       // [B, heads, S] (natural log, scaled scores) or null
+  // backward
+  const void* dO = nullptr;   // [T, H]
+  float* Dscratch = nullptr;  // [B, heads, S]
+  void* dqkv = nullptr;       // [T, 3H]
+  unsigned* err = nullptr;
+};
+cudaError_t attention_fwd(const AttnArgs& a, cudaStream_t st);
+cudaError_t attention_bwd(const AttnArgs& a, cudaStream_t st);
+
+// ---------------------------------------------------------------------------------------
+// Row-wise fused kernels
+// ---------------------------------------------------------------------------------------
+// Adapter forward (Eq. 1) fused with the residual add and the block's normalisation.
+//   out_pre = a + GELU(a Wd) Wu, z = a Wd (saved if z != null)
+//   encoder: y = LN(resid + out_pre) * g + b ; xhat, rstd saved (if non-null)
+//   decoder: x_out(f32) = resid(f32) + out_pre ; n = RMSNorm(x_out) * g (act), rstd
+struct AdapterFwdArgs {
+  int T = 0, H = 0, m = 0, dtype = DT_F32;
+  bool decoder = false;
+  const void* a = nullptr;      // [T, H] act
+  const float* Wd = nullptr;    // [H, m]
+  const float* Wu = nullptr;    // [m, H]
+  float* z = nullptr;           // [T, m] or null
+  const void* resid = nullptr;  // encoder: act [T, H]; decoder: f32 [T, H]
+  const float* gamma = nullptr;
+  const float* beta = nullptr;  // encoder only
+  float eps = 1e-12f;
+  void* y = nullptr;            // encoder: act [T, H] (LN output); decoder: act n
+  float* x_out = nullptr;       // decoder: f32 residual stream out
+  void* xhat = nullptr;         // encoder: act [T, H] or null
+  float* rstd = nullptr;        // [T] or null
+};
+cudaError_t adapter_fwd(const AdapterFwdArgs& a, cudaStream_t st);
+
+// Adapter backward, row part: dz = (g Wu^T) * GELU'(z) -> dz (f32 [T, m]);
+// dh = g + dz Wd^T -> dh (act) if non-null.  WuT [H, m] and WdT [m, H] are transposed copies.
+struct AdapterBwdArgs {
+  int T = 0, H = 0, m = 0, dtype = DT_F32;
+  const float* g = nullptr;     // [T, H] f32
+  const void* h = nullptr;      // [T, H] act (adapter input)
+  const float* z = nullptr;     // [T, m]
+  const float* WuT = nullptr;   // [H, m]
+  const float* WdT = nullptr;   // [m, H]
+  float* dz = nullptr;          // [T, m] scratch
+  void* dh = nullptr;           // [T, H] act or null
+  int dh_dtype = DT_F32;
+  float* dWd = nullptr;         // [H, m]
+  float* dWu = nullptr;         // [m, H]
+  float* partials = nullptr;    // scratch, adapter_bwd_partials_floats(T, H, m)
+};
+size_t adapter_bwd_partials_floats(int T, int H, int m);
+cudaError_t adapter_bwd(const AdapterBwdArgs& a, cudaStream_t st);
+
+// LayerNorm backward with frozen gamma: ds = rstd * (gy - mean(gy) - xhat mean(gy xhat)),
+// gy = dy * gamma.  dy f32, xhat act, ds f32.
+cudaError_t layernorm_bwd(const float* dy, const void* xhat, const float* rstd,
+                          const float* gamma, float* ds, int T, int H, int dtype,
+                          cudaStream_t st);
+// RMSNorm forward: n = x * rstd * gamma; x given as act (x_act) or f32 (x_f32);
+// optionally copies x into x_f32_out (f32 residual stream).
+cudaError_t rmsnorm_fwd(const void* x, int x_dtype, const float* gamma, float eps, void* n,
+                        int n_dtype, float* rstd, float* x_f32_out, int T, int H,
+                        cudaStream_t st);
+// RMSNorm backward: dx = resid + rstd * gy - x rstd^3 mean(gy x), gy = dy * gamma.
+cudaError_t rmsnorm_bwd(const float* dy, const float* x, const float* rstd, const float* gamma,
+                        const float* resid, float* dx, int T, int H, cudaStream_t st);
+
+// Encoder head forward: logits = y[b, 0, :] Wh^T + bh; mean CE -> loss; logits_out
+// (optional); dlogits [B, C] = (softmax - onehot) / B.
+cudaError_t encoder_head_fwd(const void* y, int dtype, const float* Wh, const float* bh,
+                             const int32_t* labels, int B, int S, int H, int C, float* loss,
+                             float* logits_out, float* dlogits, unsigned* err, cudaStream_t st);
+// Encoder head backward: dWh, dbh (nullable), and dy rows at position 0 (dy pre-zeroed).
+cudaError_t encoder_head_bwd(const void* y, int dtype, const float* Wh, const float* dlogits,
+                             int B, int S, int H, int C, float* dWh, float* dbh, float* dy,
+                             cudaStream_t st);
+// Decoder cross-entropy over T rows of V logits (act), in place: logits <- dLoss/dlogits
+// (mean over T).  Per-row losses in row_loss, then loss = mean (fixed order).
+// Labels outside [0, V) set RA_DEVERR_BOUNDS in *err and are read as 0.
+cudaError_t vocab_ce(void* logits, int dtype, int ld, const int32_t* labels, int T, int V,
+                     float* row_loss, float* loss, float* logits_out, unsigned* err,
+                     cudaStream_t st);
+
+// Adam on a flat fp32 range [0, n): segment s covers [s*seg_len, ...) capped by n; each
+// segment has its own step counter steps[s] (incremented by adam_bump).  Also refreshes
+// transposed copies through the optional callback-free map below.
+struct AdamArgs {
+  float* p = nullptr; const float* g = nullptr; float* m = nullptr; float* v = nullptr;
+  int64_t n = 0;
+  int64_t seg_len = 0;         // elements per segment (one layer's adapters)
+  int n_seg = 0;
+  const int32_t* steps = nullptr; // [n_seg] completed steps before this update
+  float lr = 1e-4f, beta1 = 0.9f, beta2 = 0.999f, eps = 1e-8f;
+};
+cudaError_t adam_update(const AdamArgs& a, cudaStream_t st);
+cudaError_t adam_bump(int32_t* steps, int n, cudaStream_t st);
+
+// Utilities
+cudaError_t convert_f32(const float* src, void* dst, int dst_dtype, int64_t n, cudaStream_t st);
+// dst[c * ld_dst + r] = src[r, c] (src rows x cols, f32) converted to dst_dtype
+cudaError_t transpose_f32(const float* src, void* dst, int dst_dtype, int rows, int cols,
+                          int ld_dst, cudaStream_t st);
+// Decoder FFN gate/up packing: rows of a part (0 gate, 1 up) [R = F, C = H] go to the packed
+// [2F, H] matrix in 64-row blocks alternating gate and up (or to its transpose [H, 2F]).
+cudaError_t pack_rows(const float* src, void* dst, int dst_dtype, int R, int C, int part,
+                      bool transposed, cudaStream_t st);
+// Transposed f32 copies of the adapter matrices of n_layers consecutive layers.
+cudaError_t adapter_transpose(const float* P, float* PT, int n_layers, int H, int m, cudaStream_t st);
+cudaError_t fill_f32(float* dst, float v, int64_t n, cudaStream_t st);
+
+}  // namespace ra

@@ -66,7 +66,7 @@ CONFIGS: Dict[str, ModelCfg] = {
     "large": _enc(24, 1024, 16, 4096, 64, 32, 256, "bf16"),
     "llama": _dec(16, 2048, 16, 5632, 128, 32000, 8, 1024, "bf16"),
     # small parity cases: several tiles plus ragged tails
-    "tiny_dec": _dec(2, 128, 2, 352, 16, 101, 2, 48, "f32"),
+    "tiny_dec": _dec(2, 128, 2, 320, 16, 101, 2, 48, "f32"),
     "small_enc_bf16": _enc(3, 256, 4, 1024, 32, 3, 100, "bf16"),
     "small_dec_bf16": _dec(3, 256, 2, 704, 32, 1000, 2, 200, "bf16"),
     "mid_enc_f32": _enc(3, 192, 3, 768, 24, 5, 77, "f32"),

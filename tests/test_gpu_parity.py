@@ -1,0 +1,222 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle, and the north-star
+invariants on the GPU: truncated gradients equal full-backprop gradients, nothing below k
+is written, frozen weights never change, the step is deterministic, checkpoints resume."""
+import numpy as np
+import pytest
+
+import synth
+from oracle import ringada_oracle as O
+from paper_2502_19864_gb300 import ringada as R
+from gpu_helpers import GpuRun, check_step, oracle_full
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def _parity_all_depths(name, depths=None, seed=0):
+    cfg = synth.CONFIGS[name]
+    w = synth.make_workload(cfg, seed)
+    ref = oracle_full(cfg, w)
+    run = GpuRun(cfg, w)
+    reports = {}
+    try:
+        for d in depths or range(1, cfg.n_layers + 1):
+            k = cfg.n_layers - d
+            loss = run.step(d)
+            logits = run.logits.double().cpu().numpy()
+            reports[d] = check_step(cfg, loss, logits, run.grads(k), run.head_grads(), ref, k)
+    finally:
+        run.close()
+    return reports
+
+
+@pytest.mark.parametrize("name", ["tiny", "mid_enc_f32", "tiny_dec"])
+def test_fp32_parity_every_depth(name):
+    _parity_all_depths(name)
+
+
+@pytest.mark.parametrize("name", ["small_enc_bf16", "small_dec_bf16"])
+def test_bf16_parity_every_depth(name):
+    _parity_all_depths(name)
+
+
+def test_truncated_equals_full_and_nothing_below_k():
+    import torch
+    cfg = synth.CONFIGS["mid_enc_f32"]
+    w = synth.make_workload(cfg, 3)
+    run = GpuRun(cfg, w)
+    try:
+        run.step(cfg.n_layers)
+        full = run.grads(0)
+        for d in range(1, cfg.n_layers):
+            k = cfg.n_layers - d
+            # sentinel in every gradient buffer below k
+            for l in range(k):
+                for key in synth.ADAPTER_KEYS:
+                    ptr, n = R.ra_get_grad(run.ctx, l, R.P[R.KEY_TO_PARAM[key]])
+                    base = run.model.buffers[1]
+                    off = ptr - base.data_ptr()
+                    base[off:off + 4 * n].view(torch.float32).fill_(float("nan"))
+            run.step(d)
+            g = run.grads(k)
+            for l in range(k, cfg.n_layers):
+                for key in synth.ADAPTER_KEYS:
+                    np.testing.assert_array_equal(g[l][key], full[l][key])
+            below = run.grads(0)
+            for l in range(k):
+                for key in synth.ADAPTER_KEYS:
+                    assert np.isnan(below[l][key]).all(), (d, l, key)
+    finally:
+        run.close()
+
+
+def test_backward_below_saved_depth_and_shape_errors():
+    cfg = synth.CONFIGS["tiny"]
+    run = GpuRun(cfg, synth.make_workload(cfg, 0))
+    try:
+        run.forward(1)
+        with pytest.raises(R.RingAdaError) as e:
+            R.ra_backward_truncated(run.ctx, 0)
+        assert e.value.status == R.RA_ERR_NOT_SAVED
+        with pytest.raises(R.RingAdaError) as e:
+            R.ra_forward(run.ctx, run.x.data_ptr(), run.labels.data_ptr(), cfg.batch + 1, cfg.seq,
+                         run.loss.data_ptr())
+        assert e.value.status == R.RA_ERR_SHAPE
+        R.ra_backward_truncated(run.ctx, cfg.n_layers - 1)
+        R.ra_adapter_update(run.ctx)
+        with pytest.raises(R.RingAdaError) as e:
+            R.ra_adapter_update(run.ctx)          # no backward since the last update
+        assert e.value.status == R.RA_ERR_STATE
+        st = R.ra_get_stats(run.ctx)
+        assert st["k_forward"] == cfg.n_layers - 1 and st["n_updates"] == 1
+        R.ra_sync_status(run.ctx)
+    finally:
+        run.close()
+
+
+def test_frozen_weights_unchanged_and_only_unfrozen_updated():
+    cfg = synth.CONFIGS["small_enc_bf16"]
+    w = synth.make_workload(cfg, 0)
+    run = GpuRun(cfg, w)
+    try:
+        wbuf = run.model.buffers[0].clone()
+        before = {l: {key: run.model.param(l, key).cpu() for key in synth.ADAPTER_KEYS}
+                  for l in range(cfg.n_layers)}
+        run.step(1, update=True)
+        run.step(2, update=True)
+        assert bool((run.model.buffers[0] == wbuf).all())
+        for l in range(cfg.n_layers):
+            for key in synth.ADAPTER_KEYS:
+                same = bool((run.model.param(l, key).cpu() == before[l][key]).all())
+                assert same == (l < cfg.n_layers - 2), (l, key)
+    finally:
+        run.close()
+
+
+def test_step_is_deterministic():
+    cfg = synth.CONFIGS["small_dec_bf16"]
+    w = synth.make_workload(cfg, 0)
+    a = GpuRun(cfg, w)
+    b = GpuRun(cfg, w)
+    try:
+        la, lb = a.step(2), b.step(2)
+        assert la == lb
+        ga, gb = a.grads(cfg.n_layers - 2), b.grads(cfg.n_layers - 2)
+        for l in ga:
+            for key in ga[l]:
+                np.testing.assert_array_equal(ga[l][key], gb[l][key])
+    finally:
+        a.close()
+        b.close()
+
+
+def test_checkpoint_resume_is_bitwise():
+    cfg = synth.CONFIGS["tiny"]
+    w = synth.make_workload(cfg, 0)
+    batches = [synth.make_batch(cfg, 100 + s) for s in range(5)]
+    depths = [1, 1, 2, 2, 2]
+    a = GpuRun(cfg, w)
+    b = GpuRun(cfg, w)
+    try:
+        for (x, y), d in zip(batches, depths):
+            a.set_batch(x, y)
+            a.step(d, update=True)
+        for (x, y), d in zip(batches[:3], depths[:3]):
+            b.set_batch(x, y)
+            b.step(d, update=True)
+        blob = R.ra_get_trainable(b.ctx)
+        b.close()
+        c = GpuRun(cfg, w)
+        R.ra_set_trainable(c.ctx, blob)
+        for (x, y), d in zip(batches[3:], depths[3:]):
+            c.set_batch(x, y)
+            c.step(d, update=True)
+        for l in range(cfg.n_layers):
+            for key in synth.ADAPTER_KEYS:
+                assert bool((a.model.param(l, key) == c.model.param(l, key)).all()), (l, key)
+        c.close()
+    finally:
+        a.close()
+
+
+def test_adam_trajectory_matches_oracle_tiny():
+    """Five steps of the depth schedule (d grows every 2 steps here) with Adam on the tiny
+    fp32 model: losses and parameters follow the oracle's trajectory."""
+    cfg = synth.CONFIGS["tiny"]
+    w = synth.make_workload(cfg, 0)
+    batches = [synth.make_batch(cfg, 200 + s) for s in range(5)]
+    depths = [R.schedule_depth(s, interval=2, d0=1, d_max=cfg.n_layers) for s in range(5)]
+    run = GpuRun(cfg, w)
+    layers, head = O.to_f64_params(w["layers"], w["head"])
+    opt = O.Adam(lr=1e-4)
+    ref_losses = O.train(cfg, layers, head, batches, depths, opt)
+    try:
+        for (x, y), d, rl in zip(batches, depths, ref_losses):
+            run.set_batch(x, y)
+            loss = run.step(d, update=True)
+            assert abs(loss - rl) <= 1e-4 * abs(rl)
+        for l in range(cfg.n_layers):
+            for key in synth.ADAPTER_KEYS:
+                p = run.model.param(l, key).double().cpu().numpy().reshape(layers[l][key].shape)
+                delta_ref = layers[l][key] - w["layers"][l][key]
+                delta_gpu = p - w["layers"][l][key]
+                if np.abs(delta_ref).max() == 0:
+                    assert np.abs(delta_gpu).max() == 0
+                else:
+                    assert np.linalg.norm(delta_gpu - delta_ref) / np.linalg.norm(delta_ref) < 1e-3
+    finally:
+        run.close()
+
+
+def test_adapter_backward_entry_point_vs_oracle():
+    import torch
+    rng = np.random.default_rng(0)
+    T, H, m = 300, 192, 24
+    g, h = rng.normal(size=(T, H)), rng.normal(size=(T, H))
+    Wd, Wu = rng.normal(size=(H, m)) * 0.05, rng.normal(size=(m, H)) * 0.05
+    z = h @ Wd
+    dh_ref, dWd_ref, dWu_ref = O.adapter_backward(g, h, z, Wd, Wu)
+    dev = lambda a: torch.tensor(a, dtype=torch.float32, device="cuda")
+    tg, th, tz, tWd, tWu = map(dev, (g, h, z, Wd, Wu))
+    dWd = torch.empty(H, m, dtype=torch.float32, device="cuda")
+    dWu = torch.empty(m, H, dtype=torch.float32, device="cuda")
+    dh = torch.empty(T, H, dtype=torch.float32, device="cuda")
+    nb = R.ra_adapter_backward_scratch_bytes(T, H, m)
+    scratch = torch.empty(nb, dtype=torch.uint8, device="cuda")
+    R.ra_adapter_backward(tg.data_ptr(), th.data_ptr(), tz.data_ptr(), tWd.data_ptr(), tWu.data_ptr(),
+                          T, H, m, dWd.data_ptr(), dWu.data_ptr(), dh.data_ptr(), scratch.data_ptr(), nb)
+    torch.cuda.synchronize()
+    for got, ref in ((dWd, dWd_ref), (dWu, dWu_ref), (dh, dh_ref)):
+        err = np.abs(got.double().cpu().numpy() - ref).max() / np.abs(ref).max()
+        assert err < 1e-5, err
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name,depths", [("base", [1, 3, 6, 12])])
+def test_full_size_parity_base(name, depths):
+    _parity_all_depths(name, depths)

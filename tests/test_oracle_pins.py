@@ -17,11 +17,10 @@ import synth
 from oracle import ringada_oracle as O
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
-torch.set_default_dtype(torch.float64)
 
 
 def T(a, grad=False):
-    t = torch.tensor(np.asarray(a, dtype=np.float64))
+    t = torch.tensor(np.asarray(a, dtype=np.float64), dtype=torch.float64)
     return t.requires_grad_(grad)
 
 
