@@ -1,0 +1,430 @@
+#!/usr/bin/env python
+"""Throughput of the adapter fine-tuning step (forward, loss, early-stopped backward, Adam)
+on the BERT-base-shaped workload, versus the unfreezing depth d (k = L - d).
+
+One "step" is ra_forward + ra_backward_truncated(k) + ra_adapter_update over one batch of
+32 x 128 synthetic tokens, replayed from a CUDA graph; inputs are resident in HBM when the
+timed region starts.  The headline is samples/s at d = 6 (a frozen prefix of 6 blocks plus
+a 6-block backward); the sweep over d = 1, 3, 6, 12 is in "sweep".  The step streams more
+than 1 GB per call, far above the 129 MB L2, so no flush is needed between steps.
+
+  python bench.py [--gpus N --steps K --warmup W]      # the CUDA path (one JSON line)
+  python bench.py --impl reference ...                 # the fp64 oracle on the host cores
+
+Under torchrun (N > 1) every rank runs an independent replica (the step does not shard:
+"replicas only"); value = all ranks' samples / the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "fine-tune samples/sec vs unfrozen depth k"
+UNIT = "samples/s"
+HEADLINE_D = 6
+SWEEP = [1, 3, 6, 12]
+CPU_SAMPLE_BATCH = 2      # sequences of 128 tokens per oracle step (bounded CPU sample)
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="base")
+    ap.add_argument("--no-large", action="store_true", help="skip the BERT-large GEMM check")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-worker", default=None, help=argparse.SUPPRESS)
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------------------
+# oracle legs (host cores)
+# ---------------------------------------------------------------------------------------
+
+def oracle_sample_rate(cfg_name, depth, batch, min_seconds, steps=None):
+    """fp64 oracle steps (forward, loss, early-stopped backward, Adam) on `batch` sequences
+    of the workload; returns (samples/s, steps run, seconds)."""
+    import dataclasses
+    import synth
+    from oracle import ringada_oracle as O
+    cfg = dataclasses.replace(synth.CONFIGS[cfg_name], batch=batch)
+    w = synth.make_workload(cfg, 0)
+    layers, head = O.to_f64_params(w["layers"], w["head"])
+    opt = O.Adam(lr=1e-4)
+    n, t0 = 0, time.perf_counter()
+    while True:
+        r = O.step(cfg, layers, head, w["x"], w["labels"], depth)
+        O.apply_update(cfg, layers, head, r, opt)
+        n += 1
+        el = time.perf_counter() - t0
+        if (steps is not None and n >= steps) or (steps is None and el >= min_seconds):
+            break
+    return batch * n / el, n, el
+
+
+def cpu_worker(spec):
+    cfg_name, depth, batch, secs = spec.split(",")
+    rate, n, el = oracle_sample_rate(cfg_name, int(depth), int(batch), float(secs))
+    print(json.dumps(dict(rate=rate, steps=n, seconds=el)))
+
+
+def run_cpu_baseline(cfg_name, depth, batch, seconds):
+    cores = os.cpu_count() or 1
+    env = dict(os.environ, OMP_NUM_THREADS=str(cores), OPENBLAS_NUM_THREADS=str(cores),
+               MKL_NUM_THREADS=str(cores), CUDA_VISIBLE_DEVICES="")
+    spec = "%s,%d,%d,%g" % (cfg_name, depth, batch, seconds)
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-worker", spec],
+                       capture_output=True, text=True, env=env, timeout=900)
+    if r.returncode != 0:
+        return {"value": None, "unit": UNIT, "cores": cores, "kind": "oracle",
+                "sample": "failed: " + r.stderr.strip()[-300:]}
+    res = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": res["rate"], "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": "%d oracle steps (fp64 numpy, BLAS on %d threads) of %s at d=%d on %d of "
+                      "the 32 sequences, %.1f s" % (res["steps"], cores, cfg_name, depth, batch,
+                                                   res["seconds"])}
+
+
+def reference_main(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import synth
+    cfg = synth.CONFIGS[args.config]
+    cores = os.cpu_count() or 1
+    # warm-up and timed oracle steps, each a bounded sample (CPU_SAMPLE_BATCH sequences)
+    oracle_sample_rate(args.config, HEADLINE_D, 1, 0, steps=max(1, min(args.warmup, 2)))
+    rate, n, el = oracle_sample_rate(args.config, HEADLINE_D, 1, 0, steps=args.steps)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * el / n,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": "bert-base-shaped adapter step, d=%d (one of 32 sequences per "
+                               "oracle step)" % HEADLINE_D, "batch": 1, "seq_len": cfg.seq,
+                   "layers": cfg.n_layers, "hidden": cfg.hidden},
+        "cpu_baseline": {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": "%d fp64 oracle steps on 1 sequence of 128 tokens" % n},
+        "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# ---------------------------------------------------------------------------------------
+# GPU leg
+# ---------------------------------------------------------------------------------------
+
+def start_clock_sampler(index):
+    path = tempfile.mktemp(prefix="clocks_", suffix=".csv")
+    q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    try:
+        f = open(path, "w")
+        p = subprocess.Popen(["nvidia-smi", "-i", str(index), "--query-gpu=" + q,
+                              "--format=csv,noheader,nounits", "-lms", "200"], stdout=f,
+                             stderr=subprocess.DEVNULL)
+        return p, f, path
+    except Exception:
+        return None, None, path
+
+
+def stop_clock_sampler(h):
+    p, f, path = h
+    if p is None:
+        return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+    p.terminate()
+    p.wait(timeout=10)
+    f.close()
+    sm, smax, reasons = [], None, set()
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    for line in open(path):
+        parts = [x.strip() for x in line.split(",")]
+        if len(parts) < 9:
+            continue
+        try:
+            sm.append(float(parts[1]))
+            smax = float(parts[2])
+        except ValueError:
+            continue
+        for nm, v in zip(names, parts[5:9]):
+            if v.lower() == "active":
+                reasons.add(nm)
+    os.unlink(path)
+    return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+            "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def measured_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))), "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+def gemm_traffic():
+    """DRAM bytes per launch of the tensor-core GEMM from the committed ncu summary, if the
+    kernel source has not changed since the capture (else null)."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "gemm_traffic.txt")
+    src = os.path.join(ROOT, "paper_2502_19864_gb300", "csrc", "k_gemm_tc.cu")
+    try:
+        kv = dict(l.split("=", 1) for l in open(path).read().split() if "=" in l)
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        if kv.get("source_sha") != h:
+            return None, "kernel changed since the capture"
+        return float(kv["bytes_per_flop"]), kv.get("case", "")
+    except Exception:
+        return None, "no capture"
+
+
+class Runner:
+    """A model context plus CUDA graphs of one step per depth."""
+
+    def __init__(self, cfg, max_depth, device):
+        import torch
+        import synth
+        from paper_2502_19864_gb300 import ringada as R
+        self.torch, self.R, self.cfg = torch, R, cfg
+        w = synth.make_workload(cfg, 0)
+        arch = R.RA_ENCODER_POSTLN if cfg.arch == "encoder" else R.RA_DECODER_PRENORM
+        self.model = R.Model(R.make_cfg(arch, cfg.n_layers, cfg.hidden, cfg.n_heads, cfg.ffn,
+                                        cfg.n_out, cfg.batch, cfg.seq,
+                                        R.RA_BF16 if cfg.dtype == "bf16" else R.RA_F32,
+                                        int(cfg.head_trainable), max_depth, cfg.norm_eps,
+                                        cfg.rope_theta), cfg.adapter_dim, device=device)
+        self.model.set_weights(w["layers"], w["head"])
+        dt = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
+        self.x = torch.tensor(w["x"], dtype=torch.float32).to(dt).to(device)
+        self.labels = torch.tensor(w["labels"], dtype=torch.int32).to(device)
+        self.loss = torch.zeros(1, dtype=torch.float32, device=device)
+        self.x_host = torch.tensor(w["x"], dtype=torch.float32).to(dt).pin_memory()
+        self.labels_host = torch.tensor(w["labels"], dtype=torch.int32).pin_memory()
+        self.loss_host = torch.zeros(1, dtype=torch.float32).pin_memory()
+        self.graphs = {}
+        self.launches = {}
+
+    def step(self, d, stream=None):
+        R, c = self.R, self.model.ctx
+        R.ra_set_unfrozen_depth(c, d)
+        R.ra_forward(c, self.x.data_ptr(), self.labels.data_ptr(), self.cfg.batch, self.cfg.seq,
+                     self.loss.data_ptr(), None, stream)
+        R.ra_backward_truncated(c, self.cfg.n_layers - d, stream)
+        R.ra_adapter_update(c, stream=stream)
+
+    def capture(self, d, profile=False):
+        torch, R = self.torch, self.R
+        n0 = R.ra_kernel_launches()
+        self.step(d)                      # eager warm-up (also counts the launches of a step)
+        torch.cuda.synchronize()
+        self.launches[d] = R.ra_kernel_launches() - n0
+        g = torch.cuda.CUDAGraph()
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        R.ra_profile_enable(self.model.ctx, profile)
+        with torch.cuda.graph(g, stream=s, capture_error_mode="relaxed"):
+            self.step(d, torch.cuda.current_stream())
+        R.ra_profile_enable(self.model.ctx, False)
+        torch.cuda.synchronize()
+        self.graphs[d] = g
+        return g
+
+    def time_steps(self, d, steps, warmup):
+        torch = self.torch
+        g = self.graphs[d]
+        for _ in range(warmup):
+            g.replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(steps):
+            g.replay()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / steps
+
+    def time_e2e(self, d, steps):
+        """Host-buffer path: pinned H2D copy of the batch, the step, D2H of the loss."""
+        torch = self.torch
+        g = self.graphs[d]
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0 = time.perf_counter()
+        a.record()
+        for _ in range(steps):
+            self.x.copy_(self.x_host, non_blocking=True)
+            self.labels.copy_(self.labels_host, non_blocking=True)
+            g.replay()
+            self.loss_host.copy_(self.loss, non_blocking=True)
+        b.record()
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+        ms = max(a.elapsed_time(b), 1000 * wall) / steps
+        h2d = self.x.numel() * self.x.element_size() + self.labels.numel() * 4
+        return ms, h2d, 4
+
+
+def gpu_main(args):
+    import torch
+    import synth
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    device = "cuda:%d" % torch.cuda.current_device()
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2502_19864_gb300 import ringada as R
+
+    cfg = synth.CONFIGS[args.config]
+    peaks, peak_kind = measured_peaks()
+    steps, warmup = args.steps, max(3, args.warmup)
+
+    # CPU baseline first (its own process, before the GPU work starts)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = run_cpu_baseline(args.config, HEADLINE_D, CPU_SAMPLE_BATCH, 12.0)
+
+    run = Runner(cfg, max(SWEEP), device)
+    sweep = {}
+    for d in SWEEP:
+        run.capture(d, profile=(d == HEADLINE_D))
+    # sweep points (not the headline)
+    for d in SWEEP:
+        if d != HEADLINE_D:
+            sweep[d] = run.time_steps(d, steps, warmup)
+    # headline: timed region with the clock sampler running and the profiled graph
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clk = start_clock_sampler(torch.cuda.current_device())
+    ms = run.time_steps(HEADLINE_D, steps, warmup)
+    clocks = stop_clock_sampler(clk)
+    sweep[HEADLINE_D] = ms
+    prof = R.ra_profile_read(run.model.ctx)   # the last replay's per-kernel device times
+    e2e_ms, h2d, d2h = run.time_e2e(HEADLINE_D, steps)
+    stats = run.model.stats()
+    launches_headline = run.launches[HEADLINE_D]
+    R.ra_set_unfrozen_depth(run.model.ctx, HEADLINE_D)
+
+    # max over ranks
+    if dist:
+        t = torch.tensor([ms, e2e_ms], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, e2e_ms = t.tolist()
+
+    B = cfg.batch
+    value = world * B / (ms / 1000.0)
+    g = prof["gemm"]
+    gemm_tflops = g["flops"] / (g["ms"] / 1000.0) / 1e12 if g["ms"] > 0 else None
+    traffic_per_flop, traffic_note = gemm_traffic()
+    launches_per_gemm = max(1, g["calls"])
+    roof = {
+        "kernel": "frozen-weight and dX GEMMs (tcgen05, bf16 in, fp32 accumulate), all launches of one step",
+        "bound": "tensor", "unit": "TFLOP/s",
+        "achieved": gemm_tflops,
+        "peak": peaks["bf16_tflops_sustained"],
+        "peak_kind": "%s bf16 sustained (kernel timed inside a long step)" % peak_kind,
+        "frac": (gemm_tflops / peaks["bf16_tflops_sustained"]) if gemm_tflops else None,
+        "launches": g["calls"],
+        "flops_per_launch": g["flops"] / launches_per_gemm,
+        "traffic": (traffic_per_flop * g["flops"] / launches_per_gemm) if traffic_per_flop else None,
+        "traffic_note": traffic_note,
+    }
+    phases = {k: {"ms": v["ms"], "calls": v["calls"],
+                  "tflops": (v["flops"] / v["ms"] / 1e9) if v["ms"] > 0 and v["flops"] else None,
+                  "gbs": (v["bytes"] / v["ms"] / 1e6) if v["ms"] > 0 and v["bytes"] else None}
+              for k, v in prof.items()}
+
+    large = None
+    if rank == 0 and not args.no_large and args.config == "base":
+        del run
+        torch.cuda.empty_cache()
+        large = large_gemm_check(torch, R, synth, device, peaks)
+
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return 0
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
+        "warmup": warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": "bert-base-shaped adapter step (12 post-LN layers, H 768, 12 "
+                               "heads, FFN 3072, adapters m 64, batch 32 x 128), d=%d" % HEADLINE_D,
+                   "global_batch": B * world, "seq_len": cfg.seq, "depth": HEADLINE_D,
+                   "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (>1 GB streamed per step)",
+                   "cuda_graph": True},
+        "sweep": {"d=%d" % d: {"samples_per_s": world * B / (sweep[d] / 1000.0),
+                               "ms_per_step": sweep[d], "k": cfg.n_layers - d}
+                  for d in sorted(sweep)},
+        "monotone_in_k": all(sweep[a] > sweep[b] for a, b in zip(sorted(sweep)[1:], sorted(sweep))),
+        "saved_bytes_at_headline": stats["saved_bytes_in_use"],
+        "roofline": roof,
+        "phases_ms": phases,
+        "clocks": clocks,
+        "e2e": {"value": world * B / (e2e_ms / 1000.0), "unit": UNIT,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+        "gpu_launches": launches_headline * steps,
+        "gpu_launches_per_step": launches_headline,
+        "cpu_baseline": cpu,
+        "large": large,
+    }
+    print(json.dumps(line))
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+def large_gemm_check(torch, R, synth, device, peaks):
+    """BERT-large-shaped step at d = 24 and d = 1: samples/s and the GEMMs' tensor throughput
+    (the spec bar is >= 60 % of dense bf16 peak in these GEMMs)."""
+    cfg = synth.CONFIGS["large"]
+    run = Runner(cfg, cfg.n_layers, device)
+    out = {}
+    for d in (24, 1):
+        run.capture(d, profile=True)
+        ms = run.time_steps(d, 10, 3)
+        prof = R.ra_profile_read(run.model.ctx)
+        g = prof["gemm"]
+        tf = g["flops"] / (g["ms"] / 1000.0) / 1e12 if g["ms"] > 0 else None
+        out["d=%d" % d] = {"samples_per_s": cfg.batch / (ms / 1000.0), "ms_per_step": ms,
+                           "gemm_tflops": tf,
+                           "gemm_frac_sustained": tf / peaks["bf16_tflops_sustained"] if tf else None,
+                           "gemm_frac_burst": tf / peaks["bf16_tflops"] if tf else None,
+                           "gemm_share_of_step": g["ms"] / ms if ms else None}
+    return out
+
+
+def main():
+    args = parse()
+    if args.cpu_worker:
+        cpu_worker(args.cpu_worker)
+        return 0
+    if args.impl == "reference":
+        return reference_main(args)
+    return gpu_main(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -198,6 +198,41 @@ const char* ra_last_error(const ra_ctx* ctx);
 void ra_destroy(ra_ctx* ctx);
 
 /* ---------------------------------------------------------------------------------------
+ * Measurement.  With profiling on, every kernel call of the step is bracketed by a pair of
+ * CUDA events on the call's stream (also when the calls are captured into a CUDA graph:
+ * the events become graph nodes and a replay re-records them).  ra_profile_read sums the
+ * elapsed times per category once the recorded work has completed, together with the
+ * algorithmic work of those calls (flops: 2 M N K per GEMM, 4 S^2 dh per attention head
+ * forward and 10 S^2 dh backward, halved when causal; bytes: each input read once and each
+ * output written once).
+ * ------------------------------------------------------------------------------------- */
+typedef enum {
+  RA_PROF_GEMM = 0,     /* frozen-weight GEMMs and their transposed-weight dX GEMMs */
+  RA_PROF_ATTN_FWD,     /* fused attention forward */
+  RA_PROF_ATTN_BWD,     /* fused attention backward */
+  RA_PROF_ADAPTER_FWD,  /* adapter + residual + norm forward */
+  RA_PROF_ADAPTER_BWD,  /* adapter backward with the in-kernel dW reduction */
+  RA_PROF_NORM,         /* LayerNorm / RMSNorm kernels outside the adapter kernels */
+  RA_PROF_HEAD,         /* head, loss, cross-entropy */
+  RA_PROF_UPDATE,       /* Adam and the refresh of transposed adapter copies */
+  RA_PROF_COUNT
+} ra_prof_cat;
+
+typedef struct {
+  double ms[RA_PROF_COUNT];     /* summed device time of the calls, milliseconds */
+  double flops[RA_PROF_COUNT];  /* algorithmic floating-point operations */
+  double bytes[RA_PROF_COUNT];  /* algorithmic DRAM bytes */
+  int32_t calls[RA_PROF_COUNT]; /* calls recorded */
+} ra_profile;
+
+/* on != 0: start recording (clears earlier records); on == 0: stop recording. */
+ra_status ra_profile_enable(ra_ctx* ctx, int32_t on);
+/* Sums the records; the caller must have synchronised the recorded work first. */
+ra_status ra_profile_read(ra_ctx* ctx, ra_profile* out);
+/* Kernels this library has launched in this process so far (every entry point). */
+int64_t ra_kernel_launches(void);
+
+/* ---------------------------------------------------------------------------------------
  * Stand-alone kernels, for testing each piece of the step in isolation.  No context.
  * ------------------------------------------------------------------------------------- */
 

@@ -326,6 +326,7 @@ cudaError_t fwd_impl(const AttnArgs& a, cudaStream_t st) {
   cudaFuncSetAttribute(attn_fwd_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   dim3 grid((a.S + QB - 1) / QB, a.B * a.n_heads);
   attn_fwd_kernel<T><<<grid, 256, smem, st>>>(a);
+  note_launch(1);
   return cudaGetLastError();
 }
 
@@ -345,6 +346,7 @@ cudaError_t bwd_impl(const AttnArgs& a, cudaStream_t st) {
   size_t smem2 = (size_t)(2 * KB * ld + 2 * 32 * ld) * sizeof(float);
   cudaFuncSetAttribute(attn_bwd_dq_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
   attn_bwd_dq_kernel<T><<<dim3((a.S + 31) / 32, a.B * a.n_heads), 256, smem2, st>>>(a);
+  note_launch(3);
   return cudaGetLastError();
 }
 

@@ -127,12 +127,14 @@ cudaError_t gemm_simt(const GemmArgs& g, cudaStream_t st) {
   dim3 grid((g.N + BN - 1) / BN, (g.M + BM - 1) / BM);
   if (g.in_dtype == DT_BF16) gemm_simt_kernel<bf16><<<grid, NT, 0, st>>>(g);
   else gemm_simt_kernel<float><<<grid, NT, 0, st>>>(g);
+  note_launch(1);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || g.epi != EPI_SWIGLU) return e;
   int F = g.N / 2;
   int64_t n = (int64_t)g.M * F;
   swiglu_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(g.C, g.ldc, g.c_dtype, g.C2,
                                                              g.ldc2, g.c2_dtype, g.M, F);
+  note_launch(1);
   return cudaGetLastError();
 }
 

@@ -1,7 +1,577 @@
-// k_gemm_tc.cu -- tcgen05 / TMEM / TMA GEMM (placeholder until the kernel lands).
+// k_gemm_tc.cu -- tcgen05 / TMEM / TMA GEMM for sm_103a with the step's fused epilogues.
+//
+// C[M, N] = A[M, K] B[N, K]^T, bf16 operands (both K-major), fp32 accumulation in TMEM.
+// This carries every frozen-weight GEMM of the forward (QKV, attention output, FFN up with
+// the bias+GELU or SwiGLU epilogue, FFN down) and every transposed-weight dX GEMM of the
+// backward (fused GELU' / SwiGLU' / residual epilogues) -- the dense contractions of the
+// step.
+//
+// Structure (one persistent CTA per SM, 192 threads):
+//   warp 0      TMA producer: 128 x 64 A tiles and BN x 64 B tiles (128-byte swizzle) into
+//               a STAGES-deep shared-memory ring, completion tracked by mbarrier tx counts;
+//   warp 1      allocates 2*BN TMEM columns (two accumulators); one thread issues
+//               tcgen05.mma (M = 128, N = BN, K = 16) and tcgen05.commit to free each stage
+//               and to publish each finished accumulator;
+//   warps 2..5  epilogue: tcgen05.ld of their 32 TMEM lanes, fused math, vector stores;
+//               the second accumulator lets the next tile's main loop overlap this.
+// Every mbarrier wait is bounded (global timer); on expiry the kernel records
+// RA_DEVERR_TIMEOUT, drains its own copies and MMAs, frees TMEM and returns.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <mutex>
+#include <unordered_map>
+
+#include "common.cuh"
 #include "kernels.h"
 
 namespace ra {
-bool tc_available() { return false; }
-cudaError_t gemm_tc(const GemmArgs&, cudaStream_t) { return cudaErrorNotSupported; }
+namespace {
+
+constexpr int BM = 128, BK = 64, NTHREADS = 192;
+
+template <int BN>
+struct TileCfg {
+  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * BN;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024;  // + alignment slack
+};
+
+struct TcParams {
+  int M, N, K;
+  int n_tiles_n, num_tiles, k_blocks;
+  int epi;
+  void* C; int ldc; int c_dtype;
+  const float* bias;
+  void* C2; int ldc2; int c2_dtype;
+  const void* aux; int ldaux; int aux_dtype;
+  unsigned* err;
+};
+
+// ---- PTX helpers ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t addr, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n.reg .pred p;\n"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      "selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(addr), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase of `parity` to complete.  Returns false if the CTA was told to
+// abort or the global-timer limit passed (then the error word gets RA_DEVERR_TIMEOUT).
+__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                       unsigned* err) {
+  const uint32_t addr = smem_u32(bar);
+  if (mbar_try(addr, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try(addr, parity)) return true;
+    if ((it & 63) == 0) {
+      if (*abort_flag) return false;
+      if (global_ns() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        set_dev_error(err, RA_DEVERR_TIMEOUT);
+        return false;
+      }
+    }
+  }
+}
+__device__ __forceinline__ void tma_load_2d(const CUtensorMap* tm, uint32_t dst, uint64_t* bar,
+                                            int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+// 32 lanes x 32 consecutive fp32 columns: thread i gets lane (base + i), columns c..c+31
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor: K-major tile with rows of 128 bytes under the 128-byte
+// swizzle; 8-row groups are 1024 bytes apart (stride byte offset); the leading byte offset
+// is not used by this layout; descriptor version 1; layout type 2 = SWIZZLE_128B.
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+// Instruction descriptor of kind::f16: D f32 (bits 4-5 = 1), A and B bf16 (bits 7-9 and
+// 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) |
+         ((uint32_t)(M >> 4) << 24);
+}
+
+// ---- epilogue ---------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+// store 8 consecutive values (16 bytes for bf16, 32 bytes for f32)
+__device__ __forceinline__ void store8(void* base, int dt, int64_t off, const float* v) {
+  if (dt == DT_BF16) {
+    uint4 q;
+    q.x = pack_bf16x2(v[0], v[1]);
+    q.y = pack_bf16x2(v[2], v[3]);
+    q.z = pack_bf16x2(v[4], v[5]);
+    q.w = pack_bf16x2(v[6], v[7]);
+    *reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(base) + off) = q;
+  } else {
+    float4* p = reinterpret_cast<float4*>(reinterpret_cast<float*>(base) + off);
+    p[0] = make_float4(v[0], v[1], v[2], v[3]);
+    p[1] = make_float4(v[4], v[5], v[6], v[7]);
+  }
+}
+__device__ __forceinline__ void load8(const void* base, int dt, int64_t off, float* v) {
+  if (dt == DT_BF16) {
+    uint4 q = *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(base) + off);
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&q);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float2 f = __bfloat1622float2(h[i]);
+      v[2 * i] = f.x;
+      v[2 * i + 1] = f.y;
+    }
+  } else {
+    const float4* p = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(base) + off);
+    float4 a = p[0], b = p[1];
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  }
+}
+
+// One row's 32 accumulator columns [n, n + 32) of output C (non-SwiGLU epilogues).
+template <int EPI>
+__device__ __forceinline__ void epi_chunk(const TcParams& p, int row, int n, float* v) {
+#pragma unroll
+  for (int g = 0; g < 4; ++g) {
+    const int c = n + 8 * g;
+    if (c >= p.N) break;
+    float* x = v + 8 * g;
+    if (EPI == EPI_STORE) {
+      if (p.bias) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) x[i] += p.bias[c + i];
+      }
+      store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
+    } else if (EPI == EPI_BIAS_GELU) {
+      if (p.bias) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) x[i] += p.bias[c + i];
+      }
+      if (p.C) store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) x[i] = gelu_f(x[i]);
+      store8(p.C2, p.c2_dtype, (int64_t)row * p.ldc2 + c, x);
+    } else if (EPI == EPI_DGELU) {
+      float u[8];
+      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + c, u);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) x[i] *= gelu_grad_f(u[i]);
+      store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
+    } else if (EPI == EPI_RESID) {
+      float r[8];
+      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + c, r);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) x[i] += r[i];
+      store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
+    } else if (EPI == EPI_DSWIGLU) {
+      // column c of d(h) -> packed gate column gc and up column gc + 64
+      const int64_t gc = (int64_t)(c >> 6) * 128 + (c & 63);
+      float gt[8], up[8], dg[8], du[8];
+      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + gc, gt);
+      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + gc + 64, up);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        dg[i] = x[i] * up[i] * silu_grad_f(gt[i]);
+        du[i] = x[i] * silu_f(gt[i]);
+      }
+      store8(p.C, p.c_dtype, (int64_t)row * p.ldc + gc, dg);
+      store8(p.C, p.c_dtype, (int64_t)row * p.ldc + gc + 64, du);
+    }
+  }
+}
+
+// ---- the kernel -------------------------------------------------------------------------------
+template <int BN, int EPI>
+__global__ void __launch_bounds__(NTHREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const TcParams p) {
+  using Cfg = TileCfg<BN>;
+  constexpr int STAGES = Cfg::STAGES;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES];
+  __shared__ __align__(8) uint64_t tfull_bar[2], tempty_bar[2], drain_bar;
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ volatile int abort_sh;
+
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const uint32_t smem_base = smem_u32(smem);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull_bar[a], 1);
+      mbar_init(&tempty_bar[a], 4);
+    }
+    mbar_init(&drain_bar, 1);
+    abort_sh = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 0 && lane == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&tmem_base_sh)),
+                 "r"((uint32_t)Cfg::TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = tmem_base_sh;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int pending_phase[STAGES];
+      for (int s = 0; s < STAGES; ++s) pending_phase[s] = -1;
+      bool ok = true;
+      for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+        const int m0 = (tile / p.n_tiles_n) * BM, n0 = (tile % p.n_tiles_n) * BN;
+        for (int kb = 0; kb < p.k_blocks; ++kb) {
+          if (!mbar_wait(&empty_bar[stage], phase ^ 1u, &abort_sh, p.err)) { ok = false; break; }
+          mbar_expect_tx(&full_bar[stage], Cfg::STAGE_BYTES);
+          const uint32_t sa = smem_base + stage * Cfg::STAGE_BYTES;
+          tma_load_2d(&tmA, sa, &full_bar[stage], kb * BK, m0);
+          tma_load_2d(&tmB, sa + Cfg::A_BYTES, &full_bar[stage], kb * BK, n0);
+          pending_phase[stage] = (int)phase;
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      if (!ok) {  // let every copy this thread started land before the CTA goes away
+        volatile int no_abort = 0;
+        for (int s = 0; s < STAGES; ++s)
+          if (pending_phase[s] >= 0) mbar_wait(&full_bar[s], (uint32_t)pending_phase[s], &no_abort, nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16(BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+        if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, &abort_sh, p.err)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+        for (int kb = 0; kb < p.k_blocks; ++kb) {
+          if (!mbar_wait(&full_bar[stage], phase, &abort_sh, p.err)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sa = smem_base + stage * Cfg::STAGE_BYTES;
+          const uint64_t adesc = sdesc_sw128(sa), bdesc = sdesc_sw128(sa + Cfg::A_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)  // advance 16 elements = 32 bytes inside the swizzle atom
+            umma_bf16(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k), idesc,
+                      (kb | k) != 0);
+          umma_commit(&empty_bar[stage]);
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        umma_commit(&tfull_bar[acc]);
+        if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+      }
+      // all MMAs issued by this thread complete before TMEM and shared memory are released
+      umma_commit(&drain_bar);
+      volatile int no_abort = 0;
+      mbar_wait(&drain_bar, 0, &no_abort, nullptr);
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue (warps 2..5)
+    const int quad = warp & 3;  // TMEM lanes 32*quad .. 32*quad + 31
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x) {
+      const int m0 = (tile / p.n_tiles_n) * BM, n0 = (tile % p.n_tiles_n) * BN;
+      if (!mbar_wait(&tfull_bar[acc], acc_phase, &abort_sh, p.err)) break;
+      tc_fence_after();
+      const int row = m0 + quad * 32 + lane;
+      const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
+      if (EPI == EPI_SWIGLU) {
+        // per 128-column block: gate columns [0, 64), up columns [64, 128)
+#pragma unroll 1
+        for (int blk = 0; blk < BN; blk += 128) {
+#pragma unroll 1
+          for (int c0 = 0; c0 < 64; c0 += 32) {
+            float g[32], u[32];
+            tmem_ld32(tbase + blk + c0, g);
+            tmem_ld32(tbase + blk + 64 + c0, u);
+            const int ng = n0 + blk + c0;           // packed gate column
+            if (row < p.M && ng < p.N) {
+              if (p.C) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                  store8(p.C, p.c_dtype, (int64_t)row * p.ldc + ng + 8 * q, g + 8 * q);
+                  store8(p.C, p.c_dtype, (int64_t)row * p.ldc + ng + 64 + 8 * q, u + 8 * q);
+                }
+              }
+              const int hc = (n0 + blk) / 2 + c0;   // column of h = silu(gate) * up
+#pragma unroll
+              for (int i = 0; i < 32; ++i) g[i] = silu_f(g[i]) * u[i];
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+                store8(p.C2, p.c2_dtype, (int64_t)row * p.ldc2 + hc + 8 * q, g + 8 * q);
+            }
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 32) {
+          float v[32];
+          tmem_ld32(tbase + c0, v);
+          if (row < p.M && n0 + c0 < p.N) epi_chunk<EPI>(p, row, n0 + c0, v);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+      if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"((uint32_t)Cfg::TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// ---- host side --------------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+struct MapKey {
+  const void* ptr;
+  int64_t rows, cols, ld;
+  int box_rows;
+  bool operator==(const MapKey& o) const {
+    return ptr == o.ptr && rows == o.rows && cols == o.cols && ld == o.ld && box_rows == o.box_rows;
+  }
+};
+struct MapKeyHash {
+  size_t operator()(const MapKey& k) const {
+    size_t h = std::hash<const void*>()(k.ptr);
+    h ^= std::hash<int64_t>()(k.rows * 1000003 + k.cols) + 0x9e3779b9 + (h << 6) + (h >> 2);
+    h ^= std::hash<int64_t>()(k.ld * 31 + k.box_rows) + 0x9e3779b9 + (h << 6) + (h >> 2);
+    return h;
+  }
+};
+
+// bf16 row-major [rows, cols] with leading dimension ld; box = 64 columns x box_rows rows
+bool make_map(CUtensorMap* out, const void* ptr, int64_t rows, int64_t cols, int64_t ld, int box_rows) {
+  static std::mutex mu;
+  static std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
+  MapKey key{ptr, rows, cols, ld, box_rows};
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(key);
+  if (it != cache.end()) {
+    *out = it->second;
+    return true;
+  }
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t gstride[1] = {(cuuint64_t)ld * 2};
+  cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+  cuuint32_t estride[2] = {1, 1};
+  CUresult r = fn(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), gdim, gstride,
+                  box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return false;
+  if (cache.size() > 4096) cache.clear();
+  cache.emplace(key, *out);
+  return true;
+}
+
+template <int BN, int EPI>
+cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int grid,
+                   cudaStream_t st) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, TileCfg<BN>::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  gemm_tc_kernel<BN, EPI><<<grid, NTHREADS, TileCfg<BN>::SMEM, st>>>(a, b, p);
+  note_launch(1);
+  return cudaGetLastError();
+}
+
+template <int BN>
+cudaError_t dispatch(const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int grid,
+                     cudaStream_t st) {
+  switch (p.epi) {
+    case EPI_STORE: return launch<BN, EPI_STORE>(a, b, p, grid, st);
+    case EPI_BIAS_GELU: return launch<BN, EPI_BIAS_GELU>(a, b, p, grid, st);
+    case EPI_DGELU: return launch<BN, EPI_DGELU>(a, b, p, grid, st);
+    case EPI_RESID: return launch<BN, EPI_RESID>(a, b, p, grid, st);
+    case EPI_SWIGLU: return launch<BN, EPI_SWIGLU>(a, b, p, grid, st);
+    case EPI_DSWIGLU: return launch<BN, EPI_DSWIGLU>(a, b, p, grid, st);
+  }
+  return cudaErrorNotSupported;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+}  // namespace
+
+bool tc_available() {
+  static int v = -1;
+  if (v < 0) {
+    int dev = 0, major = 0, minor = 0;
+    v = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) == cudaSuccess)
+      v = (major == 10 && minor == 3 && encode_fn() != nullptr) ? 1 : 0;
+  }
+  return v == 1;
+}
+
+cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
+  if (g.in_dtype != DT_BF16 || g.M <= 0 || g.N <= 0 || g.K <= 0) return cudaErrorNotSupported;
+  // TMA: 16-byte aligned bases and row strides; epilogue: 8-column vector groups
+  if (g.lda % 8 || g.ldb % 8 || g.K % 8 || g.N % 8 || !aligned16(g.A) || !aligned16(g.B))
+    return cudaErrorNotSupported;
+  const bool has_c = g.C != nullptr;
+  if (has_c && (!aligned16(g.C) || g.ldc % 8)) return cudaErrorNotSupported;
+  if (g.C2 && (!aligned16(g.C2) || g.ldc2 % 8)) return cudaErrorNotSupported;
+  if (g.aux && (!aligned16(g.aux) || g.ldaux % 8)) return cudaErrorNotSupported;
+  if (g.epi == EPI_SWIGLU && (g.N % 128 || !g.C2)) return cudaErrorNotSupported;
+  if (g.epi == EPI_DSWIGLU && g.N % 64) return cudaErrorNotSupported;
+  if (!has_c && g.epi != EPI_BIAS_GELU && g.epi != EPI_SWIGLU) return cudaErrorNotSupported;
+
+  const int sms = device_sm_count();
+  const int m_tiles = (g.M + BM - 1) / BM;
+  // tile width: fewer waves of 128 x BN tiles, weighting 128-wide tiles by the higher
+  // shared-memory traffic per flop they carry
+  auto cost = [&](int bn) {
+    int tiles = m_tiles * ((g.N + bn - 1) / bn);
+    int waves = (tiles + sms - 1) / sms;
+    return (double)waves * bn * (bn == 128 ? 1.15 : 1.0);
+  };
+  const int BNsel = (g.N <= 128 || cost(128) < cost(256)) ? 128 : 256;
+
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, g.A, g.M, g.K, g.lda, BM)) return cudaErrorNotSupported;
+  if (!make_map(&mb, g.B, g.N, g.K, g.ldb, BNsel)) return cudaErrorNotSupported;
+  TcParams p;
+  p.M = g.M; p.N = g.N; p.K = g.K;
+  p.n_tiles_n = (g.N + BNsel - 1) / BNsel;
+  p.num_tiles = m_tiles * p.n_tiles_n;
+  p.k_blocks = (g.K + BK - 1) / BK;
+  p.epi = g.epi;
+  p.C = g.C; p.ldc = g.ldc; p.c_dtype = g.c_dtype;
+  p.bias = g.bias;
+  p.C2 = g.C2; p.ldc2 = g.ldc2; p.c2_dtype = g.c2_dtype;
+  p.aux = g.aux; p.ldaux = g.ldaux; p.aux_dtype = g.aux_dtype;
+  p.err = g.err;
+  const int grid = p.num_tiles < sms ? p.num_tiles : sms;
+  return BNsel == 256 ? dispatch<256>(ma, mb, p, grid, st) : dispatch<128>(ma, mb, p, grid, st);
+}
+
 }  // namespace ra

@@ -591,6 +591,7 @@ cudaError_t adapter_fwd(const AdapterFwdArgs& a, cudaStream_t st) {
     cudaFuncSetAttribute(adapter_fwd_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     adapter_fwd_kernel<float><<<grid, WARPS * 32, smem, st>>>(a);
   }
+  note_launch(1);
   return cudaGetLastError();
 }
 
@@ -620,6 +621,7 @@ cudaError_t adapter_bwd(const AdapterBwdArgs& a, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   int64_t n = 2LL * a.H * a.m;
   adapter_dw_reduce_kernel<<<blocks_for(n, 256), 256, 0, st>>>(a.partials, nchunk, a.H, a.m, a.dWd, a.dWu);
+  note_launch(3);
   return cudaGetLastError();
 }
 
@@ -629,6 +631,7 @@ cudaError_t layernorm_bwd(const float* dy, const void* xhat, const float* rstd,
   unsigned grid = blocks_for((int64_t)T * 32, 256);
   if (dtype == DT_BF16) layernorm_bwd_kernel<bf16><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H);
   else layernorm_bwd_kernel<float><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H);
+  note_launch(1);
   return cudaGetLastError();
 }
 
@@ -644,12 +647,14 @@ cudaError_t rmsnorm_fwd(const void* x, int x_dtype, const float* gamma, float ep
     rmsnorm_fwd_kernel<bf16, float><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H);
   else
     rmsnorm_fwd_kernel<float, float><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H);
+  note_launch(1);
   return cudaGetLastError();
 }
 
 cudaError_t rmsnorm_bwd(const float* dy, const float* x, const float* rstd, const float* gamma,
                         const float* resid, float* dx, int T, int H, cudaStream_t st) {
   rmsnorm_bwd_kernel<<<blocks_for((int64_t)T * 32, 256), 256, 0, st>>>(dy, x, rstd, gamma, resid, dx, T, H);
+  note_launch(1);
   return cudaGetLastError();
 }
 
@@ -661,6 +666,7 @@ cudaError_t encoder_head_fwd(const void* y, int dtype, const float* Wh, const fl
     encoder_head_fwd_kernel<bf16><<<1, 256, 0, st>>>(y, Wh, bh, labels, B, S, H, C, loss, logits_out, dlogits, err);
   else
     encoder_head_fwd_kernel<float><<<1, 256, 0, st>>>(y, Wh, bh, labels, B, S, H, C, loss, logits_out, dlogits, err);
+  note_launch(1);
   return cudaGetLastError();
 }
 
@@ -673,6 +679,7 @@ cudaError_t encoder_head_bwd(const void* y, int dtype, const float* Wh, const fl
     encoder_head_bwd_kernel<bf16><<<grid, 256, 0, st>>>(y, Wh, dlogits, B, S, H, C, dWh, dbh, dy);
   else
     encoder_head_bwd_kernel<float><<<grid, 256, 0, st>>>(y, Wh, dlogits, B, S, H, C, dWh, dbh, dy);
+  note_launch(1);
   return cudaGetLastError();
 }
 
@@ -686,18 +693,21 @@ cudaError_t vocab_ce(void* logits, int dtype, int ld, const int32_t* labels, int
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   mean_kernel<<<1, 256, 0, st>>>(row_loss, T, loss);
+  note_launch(2);
   return cudaGetLastError();
 }
 
 cudaError_t adam_update(const AdamArgs& a, cudaStream_t st) {
   if (a.n <= 0) return cudaSuccess;
   adam_kernel<<<blocks_for(a.n, 256), 256, 0, st>>>(a);
+  note_launch(1);
   return cudaGetLastError();
 }
 
 cudaError_t adam_bump(int32_t* steps, int n, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   bump_kernel<<<blocks_for(n, 128), 128, 0, st>>>(steps, n);
+  note_launch(1);
   return cudaGetLastError();
 }
 
@@ -705,6 +715,7 @@ cudaError_t convert_f32(const float* src, void* dst, int dst_dtype, int64_t n, c
   if (n <= 0) return cudaSuccess;
   if (dst_dtype == DT_BF16) convert_kernel<bf16><<<blocks_for(n, 256), 256, 0, st>>>(src, dst, n);
   else convert_kernel<float><<<blocks_for(n, 256), 256, 0, st>>>(src, dst, n);
+  note_launch(1);
   return cudaGetLastError();
 }
 
@@ -713,6 +724,7 @@ cudaError_t transpose_f32(const float* src, void* dst, int dst_dtype, int rows, 
   dim3 grid((cols + 31) / 32, (rows + 31) / 32), blk(32, 8);
   if (dst_dtype == DT_BF16) transpose_kernel<bf16><<<grid, blk, 0, st>>>(src, dst, rows, cols, ld_dst);
   else transpose_kernel<float><<<grid, blk, 0, st>>>(src, dst, rows, cols, ld_dst);
+  note_launch(1);
   return cudaGetLastError();
 }
 
@@ -721,6 +733,7 @@ cudaError_t pack_rows(const float* src, void* dst, int dst_dtype, int R, int C, 
   int64_t n = (int64_t)R * C;
   if (dst_dtype == DT_BF16) pack_rows_kernel<bf16><<<blocks_for(n, 256), 256, 0, st>>>(src, dst, R, C, part, transposed);
   else pack_rows_kernel<float><<<blocks_for(n, 256), 256, 0, st>>>(src, dst, R, C, part, transposed);
+  note_launch(1);
   return cudaGetLastError();
 }
 
@@ -728,12 +741,14 @@ cudaError_t adapter_transpose(const float* P, float* PT, int n_layers, int H, in
   if (n_layers <= 0) return cudaSuccess;
   dim3 grid(blocks_for((int64_t)H * m, 256), 1, 4 * n_layers);
   adapter_transpose_kernel<<<grid, 256, 0, st>>>(P, PT, H, m);
+  note_launch(1);
   return cudaGetLastError();
 }
 
 cudaError_t fill_f32(float* dst, float v, int64_t n, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   fill_kernel<<<blocks_for(n, 256), 256, 0, st>>>(dst, v, n);
+  note_launch(1);
   return cudaGetLastError();
 }
 

@@ -11,6 +11,10 @@ enum DType : int { DT_F32 = 0, DT_BF16 = 1 };
 
 inline size_t dtype_size(int dt) { return dt == DT_BF16 ? 2 : 4; }
 
+// Counts kernels launched by this library (process-wide), for launch accounting.
+void note_launch(int n);
+long long launches_so_far();
+
 // ---------------------------------------------------------------------------------------
 // GEMM  C[M, N] = A[M, K] * B[N, K]^T with a fused epilogue.  A and B share a dtype and are
 // K-major (row-major, K contiguous).  The accumulator is fp32.

@@ -10,6 +10,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -92,6 +93,24 @@ struct ra_ctx {
   int n_updates = 0;
   int last_xL_slot = 0;
   int top_out = 0;  // index of the ping-pong buffer holding the last layer's output (encoder)
+
+  // profiling: event pairs around kernel calls
+  bool profiling = false;
+  struct Rec { int cat; double flops, bytes; cudaEvent_t a, b; };
+  std::vector<Rec> recs;
+  std::vector<cudaEvent_t> pool;
+  size_t pool_used = 0;
+  cudaEvent_t take_event() {
+    if (pool_used == pool.size()) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+      pool.push_back(e);
+    }
+    return pool[pool_used++];
+  }
+  ~ra_ctx() {
+    for (cudaEvent_t e : pool) cudaEventDestroy(e);
+  }
 
   template <typename T = void>
   T* w(size_t off) const { return reinterpret_cast<T*>(W + off); }
@@ -470,6 +489,74 @@ ra_status ra_set_unfrozen_depth(ra_ctx* ctx, int32_t d) {
   return RA_OK;
 }
 
+}  // extern "C"
+
+// ---- profiled kernel calls -------------------------------------------------------------
+namespace {
+
+template <class F>
+cudaError_t prof(ra_ctx* c, int cat, double flops, double bytes, cudaStream_t st, F&& f) {
+  if (!c->profiling) return f();
+  cudaEvent_t a = c->take_event(), b = c->take_event();
+  // inside stream capture an event must be recorded as "external" to become a graph node
+  // that a replay re-records (otherwise it only orders the capture)
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaStreamIsCapturing(st, &cs);
+  unsigned flags = cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : cudaEventRecordDefault;
+  if (a) cudaEventRecordWithFlags(a, st, flags);
+  cudaError_t e = f();
+  if (b) cudaEventRecordWithFlags(b, st, flags);
+  if (a && b) c->recs.push_back({cat, flops, bytes, a, b});
+  return e;
+}
+
+double esz(int dt) { return (double)dtype_size(dt); }
+
+cudaError_t P_gemm(ra_ctx* c, const GemmArgs& g, cudaStream_t st) {
+  double M = g.M, N = g.N, K = g.K;
+  double out = (g.C ? M * N * esz(g.c_dtype) : 0) + (g.C2 ? M * (g.epi == EPI_SWIGLU ? N / 2 : N) * esz(g.c2_dtype) : 0);
+  double aux = g.aux ? M * (g.epi == EPI_DSWIGLU ? 2 * N : N) * esz(g.aux_dtype) : 0;
+  if (g.epi == EPI_DSWIGLU) out = 2 * M * N * esz(g.c_dtype);
+  double bytes = (M * K + N * K) * esz(g.in_dtype) + out + aux;
+  return prof(c, RA_PROF_GEMM, 2 * M * N * K, bytes, st, [&] { return gemm(g, st); });
+}
+
+cudaError_t P_attn_fwd(ra_ctx* c, const AttnArgs& a, cudaStream_t st) {
+  double S = a.S, bh = (double)a.B * a.n_heads, dh = a.head_dim, T = (double)a.B * a.S;
+  double fl = 4 * bh * S * S * dh * (a.causal ? 0.5 : 1.0);
+  double by = T * 4 * a.n_heads * dh * esz(a.dtype) + (a.lse ? bh * S * 4 : 0);
+  return prof(c, RA_PROF_ATTN_FWD, fl, by, st, [&] { return attention_fwd(a, st); });
+}
+
+cudaError_t P_attn_bwd(ra_ctx* c, const AttnArgs& a, cudaStream_t st) {
+  double S = a.S, bh = (double)a.B * a.n_heads, dh = a.head_dim, T = (double)a.B * a.S;
+  double fl = 10 * bh * S * S * dh * (a.causal ? 0.5 : 1.0);
+  double H = (double)a.n_heads * dh;
+  double by = T * (3 * H + H + H + 3 * H) * esz(a.dtype) + bh * S * 4;  // qkv, O, dO, dqkv, lse
+  return prof(c, RA_PROF_ATTN_BWD, fl, by, st, [&] { return attention_bwd(a, st); });
+}
+
+cudaError_t P_adapter_fwd(ra_ctx* c, const AdapterFwdArgs& a, cudaStream_t st) {
+  double T = a.T, H = a.H, m = a.m, e = esz(a.dtype);
+  double by = T * H * e                              // adapter input
+              + T * H * (a.decoder ? 4 : e)          // residual
+              + T * H * e                            // normalised output
+              + (a.decoder ? T * H * 4 : 0)          // f32 residual stream out
+              + (a.xhat ? T * H * e : 0) + (a.rstd ? T * 4 : 0) + (a.z ? T * m * 4 : 0);
+  return prof(c, RA_PROF_ADAPTER_FWD, 4 * T * H * m, by, st, [&] { return adapter_fwd(a, st); });
+}
+
+cudaError_t P_adapter_bwd(ra_ctx* c, const AdapterBwdArgs& a, cudaStream_t st) {
+  double T = a.T, H = a.H, m = a.m, e = esz(a.dtype);
+  double by = T * H * 4 + T * H * e + T * m * 4 + (a.dh ? T * H * esz(a.dh_dtype) : 0) + 2 * H * m * 4;
+  double fl = 4 * T * H * m + 4 * T * H * m + (a.dh ? 2 * T * H * m : 0);
+  return prof(c, RA_PROF_ADAPTER_BWD, fl, by, st, [&] { return adapter_bwd(a, st); });
+}
+
+}  // namespace
+
+extern "C" {
+
 // ---- forward -----------------------------------------------------------------------------
 namespace {
 
@@ -512,41 +599,43 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
 
     GemmArgs g = gemm_args(ctx, xin, H, ctx->w(o.Wqkv), H, T, 3 * H, H);
     g.C = qkv; g.ldc = 3 * H; g.c_dtype = act; g.bias = ctx->w<float>(o.bqkv);
-    CU(gemm(g, st));
+    CU(P_gemm(ctx, g, st));
     AttnArgs at;
     at.qkv = qkv; at.B = B; at.S = S; at.n_heads = ctx->nh; at.head_dim = ctx->dh;
     at.dtype = act; at.scale = 1.f / sqrtf((float)ctx->dh); at.O = O; at.lse = lse;
     at.err = ctx->ws<unsigned>(ctx->ws_err);
     if (!lse) at.lse = nullptr;
-    CU(attention_fwd(at, st));
+    CU(P_attn_fwd(ctx, at, st));
     g = gemm_args(ctx, O, H, ctx->w(o.Wo), H, T, H, H);
     g.C = a; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.bo);
-    CU(gemm(g, st));
+    CU(P_gemm(ctx, g, st));
     AdapterFwdArgs ad;
     ad.T = T; ad.H = H; ad.m = m; ad.dtype = act; ad.decoder = false;
     ad.a = a; ad.Wd = Pl; ad.Wu = Pl + (size_t)H * m; ad.z = zA; ad.resid = xin;
     ad.gamma = ctx->w<float>(o.g1); ad.beta = ctx->w<float>(o.be1); ad.eps = ctx->cfg.norm_eps;
     ad.y = y1; ad.xhat = xhat1; ad.rstd = rstd1;
-    CU(adapter_fwd(ad, st));
+    CU(P_adapter_fwd(ctx, ad, st));
     g = gemm_args(ctx, y1, H, ctx->w(o.W1), H, T, F, H);
     g.epi = EPI_BIAS_GELU; g.C = u; g.ldc = F; g.c_dtype = act; g.bias = ctx->w<float>(o.b1);
     g.C2 = hbuf; g.ldc2 = F; g.c2_dtype = act;
-    CU(gemm(g, st));
+    CU(P_gemm(ctx, g, st));
     g = gemm_args(ctx, hbuf, F, ctx->w(o.W2), F, T, H, F);
     g.C = f; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.b2);
-    CU(gemm(g, st));
+    CU(P_gemm(ctx, g, st));
     ad.a = f; ad.Wd = Pl + (size_t)2 * H * m; ad.Wu = Pl + (size_t)3 * H * m; ad.z = zF;
     ad.resid = y1; ad.gamma = ctx->w<float>(o.g2); ad.beta = ctx->w<float>(o.be2);
     ad.y = xout; ad.xhat = xhat2; ad.rstd = rstd2;
-    CU(adapter_fwd(ad, st));
+    CU(P_adapter_fwd(ctx, ad, st));
     xin = xout;
     ctx->top_out = out_idx;
     out_idx ^= 1;
   }
   // head: CLS token of the last block's output
   float* Ph = ctx->P() + (size_t)L * 4 * H * m;
-  CU(encoder_head_fwd(xin, act, Ph, Ph + (size_t)ctx->C * H, labels, B, S, H, ctx->C, loss,
-                      logits, ctx->ws<float>(ctx->h_dlogits), ctx->ws<unsigned>(ctx->ws_err), st));
+  CU(prof(ctx, RA_PROF_HEAD, 2.0 * B * H * ctx->C, (double)B * H * dtype_size(act), st, [&] {
+    return encoder_head_fwd(xin, act, Ph, Ph + (size_t)ctx->C * H, labels, B, S, H, ctx->C, loss,
+                            logits, ctx->ws<float>(ctx->h_dlogits), ctx->ws<unsigned>(ctx->ws_err), st);
+  }));
   return RA_OK;
 }
 
@@ -559,8 +648,10 @@ ra_status decoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
   float* xin = k == 0 ? (float*)(ctx->slot(0) + so.x_in) : ctx->ws<float>(ctx->s_X[0]);
   float* rstd_in = k == 0 ? (float*)(ctx->slot(0) + so.rstd1) : ctx->ws<float>(ctx->s_rstd);
   void* nbuf = ctx->ws<char>(ctx->s_n);
-  CU(rmsnorm_fwd(x, act, ctx->w<float>(ctx->lw[0].g1), ctx->cfg.norm_eps, nbuf, act, rstd_in,
-                 xin, T, H, st));
+  CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * (2 * dtype_size(act) + 4), st, [&] {
+    return rmsnorm_fwd(x, act, ctx->w<float>(ctx->lw[0].g1), ctx->cfg.norm_eps, nbuf, act, rstd_in,
+                       xin, T, H, st);
+  }));
   int pp = 1;
   for (int l = 0; l < L; ++l) {
     const LayerWOff& o = ctx->lw[l];
@@ -596,43 +687,45 @@ ra_status decoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
 
     GemmArgs g = gemm_args(ctx, nbuf, H, ctx->w(o.Wqkv), H, T, 3 * H, H);
     g.C = qkv; g.ldc = 3 * H; g.c_dtype = act;
-    CU(gemm(g, st));
+    CU(P_gemm(ctx, g, st));
     AttnArgs at;
     at.qkv = qkv; at.B = B; at.S = S; at.n_heads = ctx->nh; at.head_dim = ctx->dh;
     at.dtype = act; at.causal = true; at.rope = true; at.rope_theta = ctx->cfg.rope_theta;
     at.scale = 1.f / sqrtf((float)ctx->dh); at.O = O; at.lse = lse;
     at.err = ctx->ws<unsigned>(ctx->ws_err);
-    CU(attention_fwd(at, st));
+    CU(P_attn_fwd(ctx, at, st));
     g = gemm_args(ctx, O, H, ctx->w(o.Wo), H, T, H, H);
     g.C = a; g.ldc = H; g.c_dtype = act;
-    CU(gemm(g, st));
+    CU(P_gemm(ctx, g, st));
     AdapterFwdArgs ad;
     ad.T = T; ad.H = H; ad.m = m; ad.dtype = act; ad.decoder = true;
     ad.a = a; ad.Wd = Pl; ad.Wu = Pl + (size_t)H * m; ad.z = zA; ad.resid = xin;
     ad.gamma = ctx->w<float>(o.g2); ad.eps = ctx->cfg.norm_eps;
     ad.y = nbuf; ad.x_out = x1; ad.rstd = rstd2;
-    CU(adapter_fwd(ad, st));
+    CU(P_adapter_fwd(ctx, ad, st));
     g = gemm_args(ctx, nbuf, H, ctx->w(o.W1), H, T, 2 * F, H);
     g.epi = EPI_SWIGLU; g.C = gu; g.ldc = 2 * F; g.c_dtype = act;
     g.C2 = hbuf; g.ldc2 = F; g.c2_dtype = act;
-    CU(gemm(g, st));
+    CU(P_gemm(ctx, g, st));
     g = gemm_args(ctx, hbuf, F, ctx->w(o.W2), F, T, H, F);
     g.C = f; g.ldc = H; g.c_dtype = act;
-    CU(gemm(g, st));
+    CU(P_gemm(ctx, g, st));
     ad.a = f; ad.Wd = Pl + (size_t)2 * H * m; ad.Wu = Pl + (size_t)3 * H * m; ad.z = zF;
     ad.resid = x1; ad.gamma = gnext;
     ad.y = (l + 1 < L) ? nbuf : ctx->ws<void>(ctx->h_nf);
     ad.x_out = xnext; ad.rstd = rstd_next;
-    CU(adapter_fwd(ad, st));
+    CU(P_adapter_fwd(ctx, ad, st));
     xin = xnext;
   }
   // head: logits = RMSNorm_f(x_L) Wh^T, CE in place
   void* lg = ctx->ws<char>(ctx->h_logits);
   GemmArgs g = gemm_args(ctx, ctx->ws(ctx->h_nf), H, ctx->w(ctx->head_W), H, T, ctx->C, H);
   g.C = lg; g.ldc = ctx->C; g.c_dtype = act;
-  CU(gemm(g, st));
-  CU(vocab_ce(lg, act, ctx->C, labels, T, ctx->C, ctx->ws<float>(ctx->h_rowloss), loss, logits,
-              ctx->ws<unsigned>(ctx->ws_err), st));
+  CU(P_gemm(ctx, g, st));
+  CU(prof(ctx, RA_PROF_HEAD, 0, 2.0 * T * ctx->C * dtype_size(act), st, [&] {
+    return vocab_ce(lg, act, ctx->C, labels, T, ctx->C, ctx->ws<float>(ctx->h_rowloss), loss, logits,
+                    ctx->ws<unsigned>(ctx->ws_err), st);
+  }));
   return RA_OK;
 }
 
@@ -682,17 +775,21 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
     float* Gh = ctx->G() + (size_t)L * 4 * H * m;
     CU(cudaMemsetAsync(dY, 0, (size_t)T * H * 4, st));
     const void* yL = ctx->ws(ctx->s_X[ctx->top_out]);
-    CU(encoder_head_bwd(yL, act, Ph, ctx->ws<float>(ctx->h_dlogits), B, S, H, ctx->C,
-                        ctx->cfg.head_trainable ? Gh : nullptr,
-                        ctx->cfg.head_trainable ? Gh + (size_t)ctx->C * H : nullptr, dY, st));
+    CU(prof(ctx, RA_PROF_HEAD, 4.0 * B * H * ctx->C, (double)B * H * (dtype_size(act) + 4), st, [&] {
+      return encoder_head_bwd(yL, act, Ph, ctx->ws<float>(ctx->h_dlogits), B, S, H, ctx->C,
+                              ctx->cfg.head_trainable ? Gh : nullptr,
+                              ctx->cfg.head_trainable ? Gh + (size_t)ctx->C * H : nullptr, dY, st);
+    }));
   } else {
     float* dn = ctx->ws<float>(ctx->b_ds2);
     GemmArgs g = gemm_args(ctx, ctx->ws(ctx->h_logits), ctx->C, ctx->w(ctx->head_WT), ctx->C, T,
                            H, ctx->C);
     g.C = dn; g.ldc = H; g.c_dtype = DT_F32;
-    CU(gemm(g, st));
-    CU(rmsnorm_bwd(dn, ctx->ws<float>(ctx->h_xL), ctx->ws<float>(ctx->h_rstdf),
-                   ctx->w<float>(ctx->head_rmsf), nullptr, dY, T, H, st));
+    CU(P_gemm(ctx, g, st));
+    CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * 12, st, [&] {
+      return rmsnorm_bwd(dn, ctx->ws<float>(ctx->h_xL), ctx->ws<float>(ctx->h_rstdf),
+                         ctx->w<float>(ctx->head_rmsf), nullptr, dY, T, H, st);
+    }));
   }
   for (int l = L - 1; l >= k; --l) {
     const LayerWOff& o = ctx->lw[l];
@@ -706,85 +803,89 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
     ab.partials = ctx->ws<float>(ctx->b_part);
     if (!ctx->dec) {
       float* ds2 = ctx->ws<float>(ctx->b_ds2);
-      CU(layernorm_bwd(dY, sb + so.xhat2, (float*)(sb + so.rstd2), ctx->w<float>(o.g2), ds2, T, H, act, st));
+      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * (8 + dtype_size(act)), st,
+              [&] { return layernorm_bwd(dY, sb + so.xhat2, (float*)(sb + so.rstd2), ctx->w<float>(o.g2), ds2, T, H, act, st); }));
       // FFN-branch adapter: g = ds2, input f, z_F
       ab.g = ds2; ab.h = sb + so.f; ab.z = (float*)(sb + so.zF);
       ab.WuT = PTl + (size_t)3 * H * m; ab.WdT = PTl + (size_t)2 * H * m;
       ab.dh = ctx->ws(ctx->b_df); ab.dh_dtype = act;
       ab.dWd = Gl + (size_t)2 * H * m; ab.dWu = Gl + (size_t)3 * H * m;
-      CU(adapter_bwd(ab, st));
+      CU(P_adapter_bwd(ctx, ab, st));
       // du = (df W2) * GELU'(u)
       GemmArgs g = gemm_args(ctx, ctx->ws(ctx->b_df), H, ctx->w(o.W2T), H, T, F, H);
       g.epi = EPI_DGELU; g.C = ctx->ws(ctx->b_du); g.ldc = F; g.c_dtype = act;
       g.aux = sb + so.u; g.ldaux = F; g.aux_dtype = act;
-      CU(gemm(g, st));
+      CU(P_gemm(ctx, g, st));
       // dy1 = ds2 + du W1
       float* dy1 = ctx->ws<float>(ctx->b_dy1);
       g = gemm_args(ctx, ctx->ws(ctx->b_du), F, ctx->w(o.W1T), F, T, H, F);
       g.epi = EPI_RESID; g.C = dy1; g.ldc = H; g.c_dtype = DT_F32;
       g.aux = ds2; g.ldaux = H; g.aux_dtype = DT_F32;
-      CU(gemm(g, st));
+      CU(P_gemm(ctx, g, st));
       float* ds1 = ctx->ws<float>(ctx->b_ds1);
-      CU(layernorm_bwd(dy1, sb + so.xhat1, (float*)(sb + so.rstd1), ctx->w<float>(o.g1), ds1, T, H, act, st));
+      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * (8 + dtype_size(act)), st,
+              [&] { return layernorm_bwd(dy1, sb + so.xhat1, (float*)(sb + so.rstd1), ctx->w<float>(o.g1), ds1, T, H, act, st); }));
       // attention-branch adapter
       ab.g = ds1; ab.h = sb + so.a; ab.z = (float*)(sb + so.zA);
       ab.WuT = PTl + (size_t)H * m; ab.WdT = PTl;
       ab.dh = lowest ? nullptr : ctx->ws(ctx->b_da);
       ab.dWd = Gl; ab.dWu = Gl + (size_t)H * m;
-      CU(adapter_bwd(ab, st));
+      CU(P_adapter_bwd(ctx, ab, st));
       if (lowest) break;
       g = gemm_args(ctx, ctx->ws(ctx->b_da), H, ctx->w(o.WoT), H, T, H, H);
       g.C = ctx->ws(ctx->b_dO); g.ldc = H; g.c_dtype = act;
-      CU(gemm(g, st));
+      CU(P_gemm(ctx, g, st));
       AttnArgs at;
       at.qkv = sb + so.qkv; at.B = B; at.S = S; at.n_heads = ctx->nh; at.head_dim = ctx->dh;
       at.dtype = act; at.scale = 1.f / sqrtf((float)ctx->dh); at.O = sb + so.O;
       at.lse = (float*)(sb + so.lse); at.dO = ctx->ws(ctx->b_dO); at.Dscratch = ctx->ws<float>(ctx->b_D);
       at.dqkv = ctx->ws(ctx->b_dqkv); at.err = ctx->ws<unsigned>(ctx->ws_err);
-      CU(attention_bwd(at, st));
+      CU(P_attn_bwd(ctx, at, st));
       g = gemm_args(ctx, ctx->ws(ctx->b_dqkv), 3 * H, ctx->w(o.WqkvT), 3 * H, T, H, 3 * H);
       g.epi = EPI_RESID; g.C = dX; g.ldc = H; g.c_dtype = DT_F32;
       g.aux = ds1; g.ldaux = H; g.aux_dtype = DT_F32;
-      CU(gemm(g, st));
+      CU(P_gemm(ctx, g, st));
     } else {
       // FFN-branch adapter: g = dY (= d x2), input f, z_F
       ab.g = dY; ab.h = sb + so.f; ab.z = (float*)(sb + so.zF);
       ab.WuT = PTl + (size_t)3 * H * m; ab.WdT = PTl + (size_t)2 * H * m;
       ab.dh = ctx->ws(ctx->b_df); ab.dh_dtype = act;
       ab.dWd = Gl + (size_t)2 * H * m; ab.dWu = Gl + (size_t)3 * H * m;
-      CU(adapter_bwd(ab, st));
+      CU(P_adapter_bwd(ctx, ab, st));
       // d(gate), d(up) from d h = df Wd
       GemmArgs g = gemm_args(ctx, ctx->ws(ctx->b_df), H, ctx->w(o.W2T), H, T, F, H);
       g.epi = EPI_DSWIGLU; g.C = ctx->ws(ctx->b_du); g.ldc = 2 * F; g.c_dtype = act;
       g.aux = sb + so.gu; g.ldaux = 2 * F; g.aux_dtype = act;
-      CU(gemm(g, st));
+      CU(P_gemm(ctx, g, st));
       float* dn2 = ctx->ws<float>(ctx->b_ds2);
       g = gemm_args(ctx, ctx->ws(ctx->b_du), 2 * F, ctx->w(o.W1T), 2 * F, T, H, 2 * F);
       g.C = dn2; g.ldc = H; g.c_dtype = DT_F32;
-      CU(gemm(g, st));
+      CU(P_gemm(ctx, g, st));
       float* dx1 = ctx->ws<float>(ctx->b_dy1);
-      CU(rmsnorm_bwd(dn2, (float*)(sb + so.x1), (float*)(sb + so.rstd2), ctx->w<float>(o.g2), dY, dx1, T, H, st));
+      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * 16, st,
+              [&] { return rmsnorm_bwd(dn2, (float*)(sb + so.x1), (float*)(sb + so.rstd2), ctx->w<float>(o.g2), dY, dx1, T, H, st); }));
       ab.g = dx1; ab.h = sb + so.a; ab.z = (float*)(sb + so.zA);
       ab.WuT = PTl + (size_t)H * m; ab.WdT = PTl;
       ab.dh = lowest ? nullptr : ctx->ws(ctx->b_da);
       ab.dWd = Gl; ab.dWu = Gl + (size_t)H * m;
-      CU(adapter_bwd(ab, st));
+      CU(P_adapter_bwd(ctx, ab, st));
       if (lowest) break;
       g = gemm_args(ctx, ctx->ws(ctx->b_da), H, ctx->w(o.WoT), H, T, H, H);
       g.C = ctx->ws(ctx->b_dO); g.ldc = H; g.c_dtype = act;
-      CU(gemm(g, st));
+      CU(P_gemm(ctx, g, st));
       AttnArgs at;
       at.qkv = sb + so.qkv; at.B = B; at.S = S; at.n_heads = ctx->nh; at.head_dim = ctx->dh;
       at.dtype = act; at.causal = true; at.rope = true; at.rope_theta = ctx->cfg.rope_theta;
       at.scale = 1.f / sqrtf((float)ctx->dh); at.O = sb + so.O;
       at.lse = (float*)(sb + so.lse); at.dO = ctx->ws(ctx->b_dO); at.Dscratch = ctx->ws<float>(ctx->b_D);
       at.dqkv = ctx->ws(ctx->b_dqkv); at.err = ctx->ws<unsigned>(ctx->ws_err);
-      CU(attention_bwd(at, st));
+      CU(P_attn_bwd(ctx, at, st));
       float* dn1 = ctx->ws<float>(ctx->b_ds1);
       g = gemm_args(ctx, ctx->ws(ctx->b_dqkv), 3 * H, ctx->w(o.WqkvT), 3 * H, T, H, 3 * H);
       g.C = dn1; g.ldc = H; g.c_dtype = DT_F32;
-      CU(gemm(g, st));
-      CU(rmsnorm_bwd(dn1, (float*)(sb + so.x_in), (float*)(sb + so.rstd1), ctx->w<float>(o.g1), dx1, dX, T, H, st));
+      CU(P_gemm(ctx, g, st));
+      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * 16, st,
+              [&] { return rmsnorm_bwd(dn1, (float*)(sb + so.x_in), (float*)(sb + so.rstd1), ctx->w<float>(o.g1), dx1, dX, T, H, st); }));
     }
     dY = dX;
     dyi ^= 1;
@@ -817,9 +918,12 @@ ra_status ra_adapter_update(ra_ctx* ctx, const ra_adam_cfg* adam, ra_stream_t st
   a.n_seg = (L - k) + (ctx->cfg.head_trainable ? 1 : 0);
   a.steps = ctx->steps() + k;
   a.lr = adam->lr; a.beta1 = adam->beta1; a.beta2 = adam->beta2; a.eps = adam->eps;
-  CU(adam_update(a, st));
-  CU(adam_bump(ctx->steps() + k, a.n_seg, st));
-  CU(adapter_transpose(ctx->P() + off, ctx->PT() + off, L - k, ctx->H, ctx->m, st));
+  CU(prof(ctx, RA_PROF_UPDATE, 0, (double)a.n * 4 * 6 + (double)(L - k) * 4 * ctx->H * ctx->m * 8, st, [&] {
+    cudaError_t e = adam_update(a, st);
+    if (e == cudaSuccess) e = adam_bump(ctx->steps() + k, a.n_seg, st);
+    if (e == cudaSuccess) e = adapter_transpose(ctx->P() + off, ctx->PT() + off, L - k, ctx->H, ctx->m, st);
+    return e;
+  }));
   ctx->bwd_since_update = false;
   ctx->n_updates++;
   return RA_OK;
@@ -955,6 +1059,35 @@ const char* ra_last_error(const ra_ctx* ctx) { return ctx ? ctx->err.c_str() : "
 
 void ra_destroy(ra_ctx* ctx) { delete ctx; }
 
+// ---- measurement -------------------------------------------------------------------------
+ra_status ra_profile_enable(ra_ctx* ctx, int32_t on) {
+  if (!ctx) return RA_ERR_ARG;
+  ctx->profiling = on != 0;
+  if (on) {
+    ctx->recs.clear();
+    ctx->pool_used = 0;
+  }
+  return RA_OK;
+}
+
+ra_status ra_profile_read(ra_ctx* ctx, ra_profile* out) {
+  if (!ctx || !out) return RA_ERR_ARG;
+  ra_profile p{};
+  for (const auto& r : ctx->recs) {
+    float ms = 0.f;
+    cudaError_t e = cudaEventElapsedTime(&ms, r.a, r.b);
+    if (e != cudaSuccess) return fail(ctx, RA_ERR_CUDA, "cudaEventElapsedTime: %s", cudaGetErrorString(e));
+    p.ms[r.cat] += ms;
+    p.flops[r.cat] += r.flops;
+    p.bytes[r.cat] += r.bytes;
+    p.calls[r.cat] += 1;
+  }
+  *out = p;
+  return RA_OK;
+}
+
+int64_t ra_kernel_launches(void) { return (int64_t)launches_so_far(); }
+
 // ---- stand-alone kernels -----------------------------------------------------------------
 ra_status ra_gemm_bf16(const void* A_dev, const void* B_dev, void* C_dev, int32_t M, int32_t N,
                        int32_t K, const float* bias_dev, void* gelu_out_dev, ra_stream_t stream) {
@@ -1005,6 +1138,10 @@ ra_status ra_adapter_backward(const float* g_dev, const float* h_dev, const floa
 }  // extern "C"
 
 namespace ra {
+static std::atomic<long long> g_launches{0};
+void note_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+long long launches_so_far() { return g_launches.load(std::memory_order_relaxed); }
+
 int device_sm_count() {
   int dev = 0, n = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 148;

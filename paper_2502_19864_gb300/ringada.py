@@ -68,6 +68,14 @@ class ra_stats(C.Structure):
                 ("tokens", C.c_int32), ("num_sms", C.c_int32)]
 
 
+PROF_CATS = ["gemm", "attn_fwd", "attn_bwd", "adapter_fwd", "adapter_bwd", "norm", "head", "update"]
+
+
+class ra_profile(C.Structure):
+    _fields_ = [("ms", C.c_double * 8), ("flops", C.c_double * 8), ("bytes", C.c_double * 8),
+                ("calls", C.c_int32 * 8)]
+
+
 class RingAdaError(RuntimeError):
     def __init__(self, status, msg):
         super().__init__("%s: %s" % (STATUS_NAMES.get(status, status), msg))
@@ -105,6 +113,9 @@ _SIGS = {
                                       C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
                                       C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]),
     "ra_adapter_backward_scratch_bytes": (C.c_size_t, [C.c_int32, C.c_int32, C.c_int32]),
+    "ra_profile_enable": (C.c_int, [C.c_void_p, C.c_int32]),
+    "ra_profile_read": (C.c_int, [C.c_void_p, C.c_void_p]),
+    "ra_kernel_launches": (C.c_int64, []),
 }
 
 
@@ -242,6 +253,22 @@ def ra_adapter_backward_scratch_bytes(T, H, m) -> int:
 def ra_adapter_backward(g, h, z, Wd, Wu, T, H, m, dWd, dWu, dh, scratch, scratch_bytes, stream=None):
     _check(lib().ra_adapter_backward(g, h, z, Wd, Wu, T, H, m, dWd, dWu, dh, scratch,
                                      scratch_bytes, _stream_ptr(stream)))
+
+
+def ra_profile_enable(ctx, on: bool):
+    _check(lib().ra_profile_enable(ctx, 1 if on else 0), ctx)
+
+
+def ra_profile_read(ctx):
+    """Per-category {ms, flops, bytes, calls} of the recorded kernel calls."""
+    p = ra_profile()
+    _check(lib().ra_profile_read(ctx, C.byref(p)), ctx)
+    return {cat: dict(ms=p.ms[i], flops=p.flops[i], bytes=p.bytes[i], calls=p.calls[i])
+            for i, cat in enumerate(PROF_CATS)}
+
+
+def ra_kernel_launches() -> int:
+    return lib().ra_kernel_launches()
 
 
 # ---- convenience: torch-owned buffers ------------------------------------------------------

@@ -1,0 +1,76 @@
+"""The tcgen05 GEMM through the C ABI (ra_gemm_bf16) against a plain fp32 PyTorch matmul of
+the same bf16 operands: single tile, ragged M/N/K tails, the BERT/LLaMA shapes of the step,
+the bias and bias+GELU epilogues, and bitwise determinism."""
+import numpy as np
+import pytest
+
+from paper_2502_19864_gb300 import ringada as R
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def _run(M, N, K, bias=False, gelu=False, seed=0):
+    import torch
+    g = torch.Generator(device="cpu").manual_seed(seed)
+    A = torch.randn(M, K, generator=g).to(torch.bfloat16).cuda()
+    B = (torch.randn(N, K, generator=g) * 0.05).to(torch.bfloat16).cuda()
+    b = (torch.randn(N, generator=g) * 0.1).float().cuda() if bias else None
+    C = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda")
+    G = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda") if gelu else None
+    R.ra_gemm_bf16(A.data_ptr(), B.data_ptr(), C.data_ptr(), M, N, K,
+                   b.data_ptr() if bias else None, G.data_ptr() if gelu else None)
+    torch.cuda.synchronize()
+    ref = A.float() @ B.float().T
+    if bias:
+        ref = ref + b
+    return C, G, ref
+
+
+def _check(C, ref, tol=8e-3):
+    c = C.float()
+    assert not bool(c.isnan().any()), "unwritten outputs"
+    err = (c - ref).abs().max().item()
+    scale = ref.abs().max().item()
+    # bf16 output rounding (2^-9 relative) plus fp32 accumulation-order differences
+    assert err <= tol * scale, (err, scale)
+    rel = ((c - ref).norm() / ref.norm()).item()
+    assert rel <= 4e-3, rel
+
+
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (128, 128, 128), (256, 512, 192)])
+def test_gemm_small_tiles(M, N, K):
+    C, _, ref = _run(M, N, K)
+    _check(C, ref)
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 200, 136), (77, 1000, 72), (1000, 8, 1024), (129, 264, 8)])
+def test_gemm_ragged_tails(M, N, K):
+    C, _, ref = _run(M, N, K)
+    _check(C, ref)
+
+
+@pytest.mark.parametrize("M,N,K", [(4096, 2304, 768), (4096, 768, 3072), (8192, 4096, 1024),
+                                   (8192, 1024, 4096), (8192, 2048, 5632)])
+def test_gemm_step_shapes(M, N, K):
+    C, _, ref = _run(M, N, K)
+    _check(C, ref)
+
+
+def test_gemm_bias_and_gelu_epilogue():
+    import torch
+    C, G, ref = _run(520, 384, 256, bias=True, gelu=True)
+    _check(C, ref)
+    _check(G, torch.nn.functional.gelu(ref), tol=1e-2)
+
+
+def test_gemm_is_deterministic():
+    C1, _, _ = _run(1024, 768, 768, seed=3)
+    C2, _, _ = _run(1024, 768, 768, seed=3)
+    assert bool((C1.view(-1).view(dtype=__import__("torch").int16) ==
+                 C2.view(-1).view(dtype=__import__("torch").int16)).all())
