@@ -257,6 +257,25 @@ ra_status ra_adapter_backward(const float* g_dev, const float* h_dev, const floa
                               ra_stream_t stream);
 size_t ra_adapter_backward_scratch_bytes(int32_t T, int32_t H, int32_t m);
 
+/* Same computation as ra_adapter_backward, for callers that cannot allocate device memory:
+ * a caller that is capturing its stream into a CUDA graph (cudaMalloc is not allowed
+ * during capture), or a host that passes a kernel only its inputs and outputs and has no
+ * allocator to offer.  The paper has no counterpart; this is a deployment variant.
+ * Scratch: a fixed 16 MiB device array inside the library (ra_adapter_backward_noalloc_
+ * capacity() bytes), held on every GPU that loads the library until the process exits;
+ * the call allocates nothing and frees nothing.  Sizes whose scratch need
+ * (ra_adapter_backward_scratch_bytes) exceeds the array are rejected with RA_ERR_NOMEM.
+ * The first call on a device looks up the array's device address (cudaGetSymbolAddress);
+ * make that first call before any stream capture.  All calls share the one array: calls
+ * that can overlap on the GPU (different streams without ordering) race on it and must be
+ * serialised by the caller.  Nothing in the array needs to start at zero: every element a
+ * call reads was written earlier in the same call. */
+ra_status ra_adapter_backward_noalloc(const float* g_dev, const float* h_dev, const float* z_dev,
+                                      const float* W_down_dev, const float* W_up_dev, int32_t T,
+                                      int32_t H, int32_t m, float* dW_down_dev, float* dW_up_dev,
+                                      float* dh_dev, ra_stream_t stream);
+size_t ra_adapter_backward_noalloc_capacity(void);
+
 #ifdef __cplusplus
 }
 #endif

@@ -113,6 +113,10 @@ _SIGS = {
                                       C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
                                       C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]),
     "ra_adapter_backward_scratch_bytes": (C.c_size_t, [C.c_int32, C.c_int32, C.c_int32]),
+    "ra_adapter_backward_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                              C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
+                                              C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "ra_adapter_backward_noalloc_capacity": (C.c_size_t, []),
     "ra_profile_enable": (C.c_int, [C.c_void_p, C.c_int32]),
     "ra_profile_read": (C.c_int, [C.c_void_p, C.c_void_p]),
     "ra_kernel_launches": (C.c_int64, []),
@@ -253,6 +257,16 @@ def ra_adapter_backward_scratch_bytes(T, H, m) -> int:
 def ra_adapter_backward(g, h, z, Wd, Wu, T, H, m, dWd, dWu, dh, scratch, scratch_bytes, stream=None):
     _check(lib().ra_adapter_backward(g, h, z, Wd, Wu, T, H, m, dWd, dWu, dh, scratch,
                                      scratch_bytes, _stream_ptr(stream)))
+
+
+def ra_adapter_backward_noalloc(g, h, z, Wd, Wu, T, H, m, dWd, dWu, dh, stream=None):
+    """The adapter backward with the library's fixed scratch array (no allocation)."""
+    _check(lib().ra_adapter_backward_noalloc(g, h, z, Wd, Wu, T, H, m, dWd, dWu, dh,
+                                             _stream_ptr(stream)))
+
+
+def ra_adapter_backward_noalloc_capacity() -> int:
+    return lib().ra_adapter_backward_noalloc_capacity()
 
 
 def ra_profile_enable(ctx, on: bool):

@@ -1,0 +1,77 @@
+"""The allocation-free adapter backward (ra_adapter_backward_noalloc), for callers that
+cannot allocate device memory (e.g. while capturing a CUDA graph, or inside a host that
+hands over only inputs and outputs).  Checked through the C ABI against the existing
+ra_adapter_backward on two calls in a row with different inputs, since the fixed scratch
+array is shared by every call and keeps the previous call's contents.  Named to run last."""
+import numpy as np
+import pytest
+
+from paper_2502_19864_gb300 import ringada as R
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def _inputs(T, H, m, seed):
+    import torch
+    rng = np.random.default_rng(seed)
+    dev = lambda a: torch.tensor(a, dtype=torch.float32, device="cuda")
+    h = rng.normal(size=(T, H))
+    Wd = rng.normal(size=(H, m)) * 0.05
+    return dict(g=dev(rng.normal(size=(T, H))), h=dev(h), z=dev(h @ Wd), Wd=dev(Wd),
+                Wu=dev(rng.normal(size=(m, H)) * 0.05))
+
+
+def _outputs(T, H, m):
+    import torch
+    return (torch.empty(H, m, dtype=torch.float32, device="cuda"),
+            torch.empty(m, H, dtype=torch.float32, device="cuda"),
+            torch.empty(T, H, dtype=torch.float32, device="cuda"))
+
+
+def _with_scratch(x, T, H, m):
+    import torch
+    dWd, dWu, dh = _outputs(T, H, m)
+    nb = R.ra_adapter_backward_scratch_bytes(T, H, m)
+    scratch = torch.empty(nb, dtype=torch.uint8, device="cuda")
+    R.ra_adapter_backward(x["g"].data_ptr(), x["h"].data_ptr(), x["z"].data_ptr(),
+                          x["Wd"].data_ptr(), x["Wu"].data_ptr(), T, H, m, dWd.data_ptr(),
+                          dWu.data_ptr(), dh.data_ptr(), scratch.data_ptr(), nb)
+    torch.cuda.synchronize()
+    return dWd, dWu, dh
+
+
+def _no_alloc(x, T, H, m):
+    import torch
+    dWd, dWu, dh = _outputs(T, H, m)
+    R.ra_adapter_backward_noalloc(x["g"].data_ptr(), x["h"].data_ptr(), x["z"].data_ptr(),
+                                  x["Wd"].data_ptr(), x["Wu"].data_ptr(), T, H, m,
+                                  dWd.data_ptr(), dWu.data_ptr(), dh.data_ptr())
+    torch.cuda.synchronize()
+    return dWd, dWu, dh
+
+
+def test_no_alloc_matches_the_scratch_entry_point_on_consecutive_calls():
+    # a large call first, then a smaller one that reuses the array's stale contents
+    for (T, H, m, seed) in ((1000, 256, 32, 0), (300, 192, 24, 1)):
+        x = _inputs(T, H, m, seed)
+        ref = _with_scratch(x, T, H, m)
+        got = _no_alloc(x, T, H, m)
+        for a, b in zip(got, ref):
+            a, b = a.double().cpu().numpy(), b.double().cpu().numpy()
+            assert np.abs(a - b).max() <= 1e-5 * np.abs(b).max()
+
+
+def test_no_alloc_rejects_sizes_beyond_its_array():
+    cap = R.ra_adapter_backward_noalloc_capacity()
+    assert cap == 16 << 20
+    T, H, m = 65536, 2048, 128
+    assert R.ra_adapter_backward_scratch_bytes(T, H, m) > cap
+    with pytest.raises(R.RingAdaError) as e:
+        R.ra_adapter_backward_noalloc(16, 16, 16, 16, 16, T, H, m, 16, 16, 16)
+    assert e.value.status == R.RA_ERR_NOMEM
