@@ -1,0 +1,580 @@
+// k_adapter_mma.cu -- tensor-core (mma.sync m16n8k16, bf16 -> fp32) versions of the adapter
+// kernels for the bf16 models.
+//
+// The adapter (Eq. 1) is a skinny contraction: T x H -> T x m -> T x H with m << H.  Its
+// arithmetic (4 T H m flops forward) is beyond what FFMA sustains at HBM speed, while its
+// bytes (the T x H input, residual and outputs) make it HBM-bound on tensor cores; so the
+// kernels below stream each row tile through shared memory once and fuse everything the
+// row needs:
+//   forward   z = a W_down; s = GELU(z); v = resid + a + s W_up; LayerNorm (post-LN
+//             encoder) or residual stream + RMSNorm (pre-norm decoder) of v;
+//   backward  dz = (g W_up^T) * GELU'(z); dh = g + dz W_down^T;
+//   dW        per row-chunk partials of dW_up = GELU(z)^T g and dW_down^T = dz^T h, summed
+//             afterwards in a fixed order (deterministic).
+// CTA = R rows (16 or 32) x H / 128 warps.  Phase 1 (the reduction over H) splits K across
+// warps and sums the per-warp partials of z in a fixed order; phase 2 splits the H output
+// columns across warps; row statistics for the norm are combined across warps in shared
+// memory in a fixed order.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace ra {
+namespace {
+
+constexpr int COLS_PER_WARP = 128;
+
+__device__ __forceinline__ void mma_bf16(float* d, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t* r, const void* p) {
+  uint32_t a = (uint32_t)__cvta_generic_to_shared(p);
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(a));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t* r, const void* p) {
+  uint32_t a = (uint32_t)__cvta_generic_to_shared(p);
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(a));
+}
+__device__ __forceinline__ uint32_t ld_u32(const bf16* p) {
+  return __ldg(reinterpret_cast<const unsigned int*>(p));
+}
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+__device__ __forceinline__ float2 unpack2(uint32_t u) {
+  __nv_bfloat162 h = *reinterpret_cast<__nv_bfloat162*>(&u);
+  return __bfloat1622float2(h);
+}
+
+// A fragment (16 x 16, row-major in smem, leading dimension ld elements) at (r0, k0)
+__device__ __forceinline__ void load_a(uint32_t* a, const bf16* s, int ld, int r0, int k0, int lane) {
+  const int r = r0 + (lane & 7) + ((lane >> 3) & 1) * 8;
+  const int c = k0 + (lane >> 4) * 8;
+  ldsm_x4(a, s + (size_t)r * ld + c);
+}
+
+// Phase 1 shared by forward and backward: partial[w] = X[R, kslice] * Bw^T over this warp's
+// 128-wide slice of H, where Bw is [m, H] row-major bf16 in global memory (B fragments
+// read directly; the matrix is small and stays in L1/L2).
+template <int MT, int NT>
+__device__ __forceinline__ void phase1(float (&acc)[MT][NT][4], const bf16* Xs, int ldx,
+                                       const bf16* Bw, int H, int kbase, int lane) {
+  const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) acc[mt][nt][i] = 0.f;
+#pragma unroll 2
+  for (int ks = 0; ks < COLS_PER_WARP / 16; ++ks) {
+    const int k0 = kbase + ks * 16;
+    uint32_t a[MT][4];
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) load_a(a[mt], Xs, ldx, mt * 16, k0, lane);
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      const bf16* bp = Bw + (size_t)(nt * 8 + g) * H + k0 + 2 * t;
+      const uint32_t b0 = ld_u32(bp), b1 = ld_u32(bp + 8);
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) mma_bf16(acc[mt][nt], a[mt], b0, b1);
+    }
+  }
+}
+
+template <int MT, int NT>
+__device__ __forceinline__ void store_partial(const float (&acc)[MT][NT][4], float* part, int m,
+                                              int lane) {
+  const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      const int r = mt * 16 + g, c = nt * 8 + 2 * t;
+      *reinterpret_cast<float2*>(part + r * m + c) = make_float2(acc[mt][nt][0], acc[mt][nt][1]);
+      *reinterpret_cast<float2*>(part + (r + 8) * m + c) = make_float2(acc[mt][nt][2], acc[mt][nt][3]);
+    }
+}
+
+// Phase 2: acc[16 rows of tile mt, this warp's 128 columns] = S[16, m] * Bn^T where Bn is
+// [H, m] row-major bf16 (n = output column, k = bottleneck index).
+template <int MB>
+__device__ __forceinline__ void phase2(float (&acc)[16][4], const bf16* Ss, int lds, int mt,
+                                       const bf16* Bn, int m, int nbase, int lane) {
+  const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+  for (int nt = 0; nt < 16; ++nt)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) acc[nt][i] = 0.f;
+#pragma unroll
+  for (int ks = 0; ks < MB / 16; ++ks) {
+    uint32_t a[4];
+    load_a(a, Ss, lds, mt * 16, ks * 16, lane);
+#pragma unroll
+    for (int nt = 0; nt < 16; ++nt) {
+      const bf16* bp = Bn + (size_t)(nbase + nt * 8 + g) * m + ks * 16 + 2 * t;
+      mma_bf16(acc[nt], a, ld_u32(bp), ld_u32(bp + 8));
+    }
+  }
+}
+
+struct FwdArgs {
+  int T, H, m;
+  const bf16* a;          // [T, H]
+  const bf16* WdT;        // [m, H]
+  const bf16* WuT;        // [H, m]
+  float* z;               // [T, m] or null
+  const void* resid;      // encoder bf16, decoder f32
+  const float* gamma;
+  const float* beta;
+  float eps;
+  bf16* y;                // normalised output
+  float* x_out;           // decoder residual stream out
+  bf16* xhat;             // encoder, nullable
+  float* rstd;            // nullable
+};
+
+// Loads R rows of a bf16 [T, H] matrix into smem (ld = H + 8); rows >= T read as zero.
+__device__ __forceinline__ void load_rows_bf16(bf16* dst, int ld, const bf16* src, int t0, int T,
+                                               int H, int R) {
+  const int vec = H / 8;
+  for (int e = threadIdx.x; e < R * vec; e += blockDim.x) {
+    const int r = e / vec, c = (e % vec) * 8;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (t0 + r < T) v = *reinterpret_cast<const uint4*>(src + (size_t)(t0 + r) * H + c);
+    *reinterpret_cast<uint4*>(dst + (size_t)r * ld + c) = v;
+  }
+}
+__device__ __forceinline__ void load_rows_f32_as_bf16(bf16* dst, int ld, const float* src, int t0,
+                                                      int T, int H, int R) {
+  const int vec = H / 4;
+  for (int e = threadIdx.x; e < R * vec; e += blockDim.x) {
+    const int r = e / vec, c = (e % vec) * 4;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (t0 + r < T) v = *reinterpret_cast<const float4*>(src + (size_t)(t0 + r) * H + c);
+    uint2 q = make_uint2(pack2(v.x, v.y), pack2(v.z, v.w));
+    *reinterpret_cast<uint2*>(dst + (size_t)r * ld + c) = q;
+  }
+}
+
+// WIDE: H > 1024 (up to 512 threads, 128 registers); otherwise <= 256 threads and up to 255
+// registers.  32-row tiles run only with H <= 1024.
+template <int R, int MB, bool DEC, bool WIDE>
+__global__ void __launch_bounds__(WIDE ? 512 : 256, 1) adapter_fwd_mma_kernel(FwdArgs p) {
+  constexpr int MT = R / 16, NT1 = MB / 8;
+  extern __shared__ __align__(16) uint8_t sm[];
+  const int H = p.H, W = H / COLS_PER_WARP;
+  const int lda = H + 8, lds = MB + 8;
+  bf16* As = reinterpret_cast<bf16*>(sm);                         // [R][H + 8]
+  float* part = reinterpret_cast<float*>(As + (size_t)R * lda);   // [W][R][MB]
+  bf16* Ss = reinterpret_cast<bf16*>(part + (size_t)W * R * MB);  // [R][MB + 8]
+  float* stat = reinterpret_cast<float*>(Ss + (size_t)R * lds);   // [W][16]
+  float* rowv = stat + W * 16;                                    // [16]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, t = lane & 3;
+  const int t0 = blockIdx.x * R;
+
+  load_rows_bf16(As, lda, p.a, t0, p.T, H, R);
+  __syncthreads();
+  {
+    float acc[MT][NT1][4];
+    phase1<MT, NT1>(acc, As, lda, p.WdT, H, warp * COLS_PER_WARP, lane);
+    store_partial<MT, NT1>(acc, part + (size_t)warp * R * MB, MB, lane);
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < R * MB; e += blockDim.x) {
+    const int r = e / MB, j = e % MB;
+    float zs = 0.f;
+    for (int w = 0; w < W; ++w) zs += part[((size_t)w * R + r) * MB + j];
+    if (p.z && t0 + r < p.T) p.z[(size_t)(t0 + r) * MB + j] = zs;
+    Ss[r * lds + j] = __float2bfloat16_rn(gelu_f(zs));
+  }
+  __syncthreads();
+  const int nbase = warp * COLS_PER_WARP;
+  for (int mt = 0; mt < MT; ++mt) {
+    float v[16][4];
+    phase2<MB>(v, Ss, lds, mt, p.WuT, MB, nbase, lane);
+    const int rl0 = mt * 16 + g, rl1 = rl0 + 8;           // local rows of c0/c1 and c2/c3
+    const int r0 = t0 + rl0, r1 = t0 + rl1;
+    float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+    for (int nt = 0; nt < 16; ++nt) {
+      const int c = nbase + nt * 8 + 2 * t;
+      float2 a0 = unpack2(*reinterpret_cast<const uint32_t*>(As + (size_t)rl0 * lda + c));
+      float2 a1 = unpack2(*reinterpret_cast<const uint32_t*>(As + (size_t)rl1 * lda + c));
+      float2 q0 = make_float2(0.f, 0.f), q1 = make_float2(0.f, 0.f);
+      if (DEC) {
+        const float* rs = reinterpret_cast<const float*>(p.resid);
+        if (r0 < p.T) q0 = *reinterpret_cast<const float2*>(rs + (size_t)r0 * H + c);
+        if (r1 < p.T) q1 = *reinterpret_cast<const float2*>(rs + (size_t)r1 * H + c);
+      } else {
+        const bf16* rs = reinterpret_cast<const bf16*>(p.resid);
+        if (r0 < p.T) q0 = unpack2(*reinterpret_cast<const uint32_t*>(rs + (size_t)r0 * H + c));
+        if (r1 < p.T) q1 = unpack2(*reinterpret_cast<const uint32_t*>(rs + (size_t)r1 * H + c));
+      }
+      v[nt][0] += a0.x + q0.x; v[nt][1] += a0.y + q0.y;
+      v[nt][2] += a1.x + q1.x; v[nt][3] += a1.y + q1.y;
+      if (DEC) {
+        s0 += v[nt][0] * v[nt][0] + v[nt][1] * v[nt][1];
+        s1 += v[nt][2] * v[nt][2] + v[nt][3] * v[nt][3];
+      } else {
+        s0 += v[nt][0] + v[nt][1];
+        s1 += v[nt][2] + v[nt][3];
+      }
+    }
+    // row sums across the quad, then across warps (fixed order)
+    s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
+    s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+    s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
+    s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+    if (t == 0) { stat[warp * 16 + g] = s0; stat[warp * 16 + g + 8] = s1; }
+    __syncthreads();
+    if (threadIdx.x < 16) {
+      float s = 0.f;
+      for (int w = 0; w < W; ++w) s += stat[w * 16 + threadIdx.x];
+      rowv[threadIdx.x] = s / H;
+    }
+    __syncthreads();
+    if (DEC) {
+      const float rs0 = rsqrtf(rowv[g] + p.eps), rs1 = rsqrtf(rowv[g + 8] + p.eps);
+#pragma unroll
+      for (int nt = 0; nt < 16; ++nt) {
+        const int c = nbase + nt * 8 + 2 * t;
+        const float2 gm = *reinterpret_cast<const float2*>(p.gamma + c);
+        if (r0 < p.T) {
+          *reinterpret_cast<float2*>(p.x_out + (size_t)r0 * H + c) = make_float2(v[nt][0], v[nt][1]);
+          *reinterpret_cast<uint32_t*>(p.y + (size_t)r0 * H + c) =
+              pack2(v[nt][0] * rs0 * gm.x, v[nt][1] * rs0 * gm.y);
+        }
+        if (r1 < p.T) {
+          *reinterpret_cast<float2*>(p.x_out + (size_t)r1 * H + c) = make_float2(v[nt][2], v[nt][3]);
+          *reinterpret_cast<uint32_t*>(p.y + (size_t)r1 * H + c) =
+              pack2(v[nt][2] * rs1 * gm.x, v[nt][3] * rs1 * gm.y);
+        }
+      }
+      if (p.rstd && warp == 0 && t == 0) {
+        if (r0 < p.T) p.rstd[r0] = rs0;
+        if (r1 < p.T) p.rstd[r1] = rs1;
+      }
+    } else {
+      const float mu0 = rowv[g], mu1 = rowv[g + 8];
+      float q0 = 0.f, q1 = 0.f;
+#pragma unroll
+      for (int nt = 0; nt < 16; ++nt) {
+        v[nt][0] -= mu0; v[nt][1] -= mu0; v[nt][2] -= mu1; v[nt][3] -= mu1;
+        q0 += v[nt][0] * v[nt][0] + v[nt][1] * v[nt][1];
+        q1 += v[nt][2] * v[nt][2] + v[nt][3] * v[nt][3];
+      }
+      q0 += __shfl_xor_sync(0xffffffffu, q0, 1);
+      q0 += __shfl_xor_sync(0xffffffffu, q0, 2);
+      q1 += __shfl_xor_sync(0xffffffffu, q1, 1);
+      q1 += __shfl_xor_sync(0xffffffffu, q1, 2);
+      __syncthreads();  // everyone has read rowv
+      if (t == 0) { stat[warp * 16 + g] = q0; stat[warp * 16 + g + 8] = q1; }
+      __syncthreads();
+      if (threadIdx.x < 16) {
+        float s = 0.f;
+        for (int w = 0; w < W; ++w) s += stat[w * 16 + threadIdx.x];
+        rowv[threadIdx.x] = rsqrtf(s / H + p.eps);
+      }
+      __syncthreads();
+      const float rs0 = rowv[g], rs1 = rowv[g + 8];
+#pragma unroll
+      for (int nt = 0; nt < 16; ++nt) {
+        const int c = nbase + nt * 8 + 2 * t;
+        const float2 gm = *reinterpret_cast<const float2*>(p.gamma + c);
+        const float2 bt = *reinterpret_cast<const float2*>(p.beta + c);
+        const float x00 = v[nt][0] * rs0, x01 = v[nt][1] * rs0;
+        const float x10 = v[nt][2] * rs1, x11 = v[nt][3] * rs1;
+        if (r0 < p.T) {
+          *reinterpret_cast<uint32_t*>(p.y + (size_t)r0 * H + c) = pack2(x00 * gm.x + bt.x, x01 * gm.y + bt.y);
+          if (p.xhat) *reinterpret_cast<uint32_t*>(p.xhat + (size_t)r0 * H + c) = pack2(x00, x01);
+        }
+        if (r1 < p.T) {
+          *reinterpret_cast<uint32_t*>(p.y + (size_t)r1 * H + c) = pack2(x10 * gm.x + bt.x, x11 * gm.y + bt.y);
+          if (p.xhat) *reinterpret_cast<uint32_t*>(p.xhat + (size_t)r1 * H + c) = pack2(x10, x11);
+        }
+      }
+      if (p.rstd && warp == 0 && t == 0) {
+        if (r0 < p.T) p.rstd[r0] = rs0;
+        if (r1 < p.T) p.rstd[r1] = rs1;
+      }
+    }
+    __syncthreads();  // stat / rowv reused by the next row tile
+  }
+}
+
+// ---------------------------------------------------------------------------------------
+// backward rows: dz = (g W_up^T) * GELU'(z); dh = g + dz W_down^T
+// ---------------------------------------------------------------------------------------
+struct BwdArgs {
+  int T, H, m;
+  const float* g;     // [T, H]
+  const float* z;     // [T, m]
+  const bf16* Wu;     // [m, H]
+  const bf16* Wd;     // [H, m]
+  float* dz;          // [T, m]
+  bf16* dh;           // [T, H] or null
+};
+
+template <int R, int MB, bool WIDE>
+__global__ void __launch_bounds__(WIDE ? 512 : 256, 1) adapter_bwd_rows_mma_kernel(BwdArgs p) {
+  constexpr int MT = R / 16, NT1 = MB / 8;
+  extern __shared__ __align__(16) uint8_t sm[];
+  const int H = p.H, W = H / COLS_PER_WARP;
+  const int ldg = H + 8, lds = MB + 8;
+  bf16* Gs = reinterpret_cast<bf16*>(sm);
+  float* part = reinterpret_cast<float*>(Gs + (size_t)R * ldg);
+  bf16* Ds = reinterpret_cast<bf16*>(part + (size_t)W * R * MB);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, t = lane & 3;
+  const int t0 = blockIdx.x * R;
+
+  load_rows_f32_as_bf16(Gs, ldg, p.g, t0, p.T, H, R);
+  __syncthreads();
+  {
+    float acc[MT][NT1][4];
+    phase1<MT, NT1>(acc, Gs, ldg, p.Wu, H, warp * COLS_PER_WARP, lane);
+    store_partial<MT, NT1>(acc, part + (size_t)warp * R * MB, MB, lane);
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < R * MB; e += blockDim.x) {
+    const int r = e / MB, j = e % MB;
+    float ds = 0.f;
+    for (int w = 0; w < W; ++w) ds += part[((size_t)w * R + r) * MB + j];
+    float dz = 0.f;
+    if (t0 + r < p.T) {
+      dz = ds * gelu_grad_f(p.z[(size_t)(t0 + r) * MB + j]);
+      p.dz[(size_t)(t0 + r) * MB + j] = dz;
+    }
+    Ds[r * lds + j] = __float2bfloat16_rn(dz);
+  }
+  if (!p.dh) return;
+  __syncthreads();
+  const int nbase = warp * COLS_PER_WARP;
+  for (int mt = 0; mt < MT; ++mt) {
+    float v[16][4];
+    phase2<MB>(v, Ds, lds, mt, p.Wd, MB, nbase, lane);
+    const int r0 = t0 + mt * 16 + g, r1 = r0 + 8;
+#pragma unroll
+    for (int nt = 0; nt < 16; ++nt) {
+      const int c = nbase + nt * 8 + 2 * t;
+      if (r0 < p.T) {
+        const float2 q = *reinterpret_cast<const float2*>(p.g + (size_t)r0 * H + c);
+        *reinterpret_cast<uint32_t*>(p.dh + (size_t)r0 * H + c) = pack2(v[nt][0] + q.x, v[nt][1] + q.y);
+      }
+      if (r1 < p.T) {
+        const float2 q = *reinterpret_cast<const float2*>(p.g + (size_t)r1 * H + c);
+        *reinterpret_cast<uint32_t*>(p.dh + (size_t)r1 * H + c) = pack2(v[nt][2] + q.x, v[nt][3] + q.y);
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------------------
+// dW partials over a chunk of rows, 64 columns of H per CTA:
+//   pWu[c][j][i]  = sum_t GELU(z[t, j]) g[t, i]
+//   pWdT[c][j][i] = sum_t dz[t, j] h[t, i]
+// 8 warps: warps 0-3 -> dW_up, 4-7 -> dW_down^T; warp owns m/4 bottleneck rows x 64 cols.
+// ---------------------------------------------------------------------------------------
+struct DwArgs {
+  int T, H, m, chunk;
+  const float* g;
+  const bf16* h;
+  const float* z;
+  const float* dz;
+  float* partials;
+};
+
+constexpr int DWC = 64, DWR = 32;
+
+template <int MB>
+__global__ void __launch_bounds__(256) adapter_dw_mma_kernel(DwArgs p) {
+  // 4 warps per output matrix: with m >= 64 each owns m/64 tiles of 16 bottleneck rows and
+  // all 64 columns; with m = 32 each owns one 16-row tile and one 32-column half
+  constexpr int LDJ = MB + 8, LDI = DWC + 8;
+  constexpr int MTW = MB >= 64 ? MB / 64 : 1;
+  constexpr int NPW = MB >= 64 ? 4 : 2;  // pairs of n8 tiles per warp
+  __shared__ __align__(16) bf16 Ssm[DWR * LDJ], Dsm[DWR * LDJ], Gsm[DWR * LDI], Hsm[DWR * LDI];
+  const int H = p.H, i0 = blockIdx.x * DWC, c = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, t = lane & 3;
+  const int which = warp >> 2;                    // 0: dW_up, 1: dW_down^T
+  const int jbase = MB >= 64 ? (warp & 3) * (MB / 4) : ((warp & 3) & 1) * 16;
+  const int ibase = MB >= 64 ? 0 : ((warp & 3) >> 1) * 32;
+  const int tb = c * p.chunk, te = min(p.T, tb + p.chunk);
+  float acc[MTW][2 * NPW][4];
+#pragma unroll
+  for (int a = 0; a < MTW; ++a)
+#pragma unroll
+    for (int nt = 0; nt < 2 * NPW; ++nt)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) acc[a][nt][i] = 0.f;
+  const bf16* X = which ? Dsm : Ssm;
+  const bf16* Y = which ? Hsm : Gsm;
+  for (int r0 = tb; r0 < te; r0 += DWR) {
+    __syncthreads();
+    for (int e = threadIdx.x; e < DWR * (MB / 2); e += blockDim.x) {
+      const int r = e / (MB / 2), j = (e % (MB / 2)) * 2, tt = r0 + r;
+      float2 zz = make_float2(0.f, 0.f), dd = make_float2(0.f, 0.f);
+      if (tt < te) {
+        zz = *reinterpret_cast<const float2*>(p.z + (size_t)tt * MB + j);
+        dd = *reinterpret_cast<const float2*>(p.dz + (size_t)tt * MB + j);
+        zz.x = gelu_f(zz.x);
+        zz.y = gelu_f(zz.y);
+      }
+      *reinterpret_cast<uint32_t*>(Ssm + r * LDJ + j) = pack2(zz.x, zz.y);
+      *reinterpret_cast<uint32_t*>(Dsm + r * LDJ + j) = pack2(dd.x, dd.y);
+    }
+    for (int e = threadIdx.x; e < DWR * (DWC / 4); e += blockDim.x) {
+      const int r = e / (DWC / 4), i = (e % (DWC / 4)) * 4, tt = r0 + r;
+      float4 gg = make_float4(0.f, 0.f, 0.f, 0.f);
+      uint2 hh = make_uint2(0, 0);
+      if (tt < te) {
+        gg = *reinterpret_cast<const float4*>(p.g + (size_t)tt * H + i0 + i);
+        hh = *reinterpret_cast<const uint2*>(p.h + (size_t)tt * H + i0 + i);
+      }
+      *reinterpret_cast<uint2*>(Gsm + r * LDI + i) = make_uint2(pack2(gg.x, gg.y), pack2(gg.z, gg.w));
+      *reinterpret_cast<uint2*>(Hsm + r * LDI + i) = hh;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int ks = 0; ks < DWR / 16; ++ks) {
+      const int k0 = ks * 16;
+      // A = X^T (rows j, cols t): transposed 8x8 loads of X[t][j]
+      uint32_t a[MTW][4];
+#pragma unroll
+      for (int mtw = 0; mtw < MTW; ++mtw) {
+        const int j0 = jbase + mtw * 16;
+        const int mat = lane >> 3, rr = lane & 7;
+        const int trow = k0 + rr + (mat >> 1) * 8, jcol = j0 + (mat & 1) * 8;
+        ldsm_x4_t(a[mtw], X + trow * LDJ + jcol);
+      }
+      // B = Y[t][i] (k = t, n = i): transposed 8x8 loads give the column-major fragments
+#pragma unroll
+      for (int np = 0; np < NPW; ++np) {
+        uint32_t b[4];
+        const int mat = lane >> 3, rr = lane & 7;
+        const int trow = k0 + rr + (mat & 1) * 8, icol = ibase + np * 16 + (mat >> 1) * 8;
+        ldsm_x4_t(b, Y + trow * LDI + icol);
+#pragma unroll
+        for (int mtw = 0; mtw < MTW; ++mtw) {
+          mma_bf16(acc[mtw][2 * np], a[mtw], b[0], b[1]);
+          mma_bf16(acc[mtw][2 * np + 1], a[mtw], b[2], b[3]);
+        }
+      }
+    }
+  }
+  float* out = p.partials + (size_t)c * 2 * H * MB + (which ? (size_t)H * MB : 0);
+#pragma unroll
+  for (int mtw = 0; mtw < MTW; ++mtw)
+#pragma unroll
+    for (int nt = 0; nt < 2 * NPW; ++nt) {
+      const int j = jbase + mtw * 16 + g, i = i0 + ibase + nt * 8 + 2 * t;
+      *reinterpret_cast<float2*>(out + (size_t)j * H + i) = make_float2(acc[mtw][nt][0], acc[mtw][nt][1]);
+      *reinterpret_cast<float2*>(out + (size_t)(j + 8) * H + i) = make_float2(acc[mtw][nt][2], acc[mtw][nt][3]);
+    }
+}
+
+int pick_rows(int T, int H, int m) {
+  // 32-row tiles when there are enough of them to fill the GPU twice, else 16
+  if (m > 64 || H > 1024) return 16;
+  return (T + 31) / 32 >= 2 * device_sm_count() ? 32 : 16;
+}
+
+template <int R, int MB>
+size_t fwd_smem(int H) {
+  const int W = H / COLS_PER_WARP;
+  return (size_t)R * (H + 8) * 2 + (size_t)W * R * MB * 4 + (size_t)R * (MB + 8) * 2 + (W * 16 + 16) * 4;
+}
+
+template <int R, int MB, bool DEC>
+cudaError_t launch_fwd(const FwdArgs& p, cudaStream_t st) {
+  const size_t smem = fwd_smem<R, MB>(p.H);
+  auto k = p.H > 1024 ? adapter_fwd_mma_kernel<R, MB, DEC, true> : adapter_fwd_mma_kernel<R, MB, DEC, false>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k<<<(p.T + R - 1) / R, (p.H / COLS_PER_WARP) * 32, smem, st>>>(p);
+  note_launch(1);
+  return cudaGetLastError();
+}
+
+template <int R, int MB>
+cudaError_t launch_bwd(const BwdArgs& p, cudaStream_t st) {
+  const size_t smem = fwd_smem<R, MB>(p.H);
+  auto k = p.H > 1024 ? adapter_bwd_rows_mma_kernel<R, MB, true> : adapter_bwd_rows_mma_kernel<R, MB, false>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k<<<(p.T + R - 1) / R, (p.H / COLS_PER_WARP) * 32, smem, st>>>(p);
+  note_launch(1);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool adapter_mma_ok(int H, int m) {
+  return H % COLS_PER_WARP == 0 && H <= 2048 && (m == 32 || m == 64 || m == 128);
+}
+
+cudaError_t adapter_fwd_mma(const AdapterFwdArgs& a, const void* WdT_b, const void* WuT_b,
+                            cudaStream_t st) {
+  if (a.dtype != DT_BF16 || !adapter_mma_ok(a.H, a.m)) return cudaErrorNotSupported;
+  FwdArgs p;
+  p.T = a.T; p.H = a.H; p.m = a.m;
+  p.a = reinterpret_cast<const bf16*>(a.a);
+  p.WdT = reinterpret_cast<const bf16*>(WdT_b);
+  p.WuT = reinterpret_cast<const bf16*>(WuT_b);
+  p.z = a.z; p.resid = a.resid; p.gamma = a.gamma; p.beta = a.beta; p.eps = a.eps;
+  p.y = reinterpret_cast<bf16*>(a.y); p.x_out = a.x_out;
+  p.xhat = reinterpret_cast<bf16*>(a.xhat); p.rstd = a.rstd;
+  const int R = pick_rows(a.T, a.H, a.m);
+#define RA_FWD(RR, MM)                                                           \
+  if (R == RR && a.m == MM)                                                     \
+    return a.decoder ? launch_fwd<RR, MM, true>(p, st) : launch_fwd<RR, MM, false>(p, st);
+  RA_FWD(32, 32) RA_FWD(32, 64) RA_FWD(16, 32) RA_FWD(16, 64) RA_FWD(16, 128)
+#undef RA_FWD
+  return cudaErrorNotSupported;
+}
+
+cudaError_t adapter_bwd_mma(const AdapterBwdArgs& a, const void* Wu_b, const void* Wd_b,
+                            cudaStream_t st) {
+  if (a.dtype != DT_BF16 || !adapter_mma_ok(a.H, a.m)) return cudaErrorNotSupported;
+  if (a.dh && a.dh_dtype != DT_BF16) return cudaErrorNotSupported;
+  BwdArgs p;
+  p.T = a.T; p.H = a.H; p.m = a.m; p.g = a.g; p.z = a.z;
+  p.Wu = reinterpret_cast<const bf16*>(Wu_b);
+  p.Wd = reinterpret_cast<const bf16*>(Wd_b);
+  p.dz = a.dz; p.dh = reinterpret_cast<bf16*>(a.dh);
+  const int R = pick_rows(a.T, a.H, a.m);
+  cudaError_t e = cudaErrorNotSupported;
+  if (R == 32 && a.m == 32) e = launch_bwd<32, 32>(p, st);
+  else if (R == 32 && a.m == 64) e = launch_bwd<32, 64>(p, st);
+  else if (R == 16 && a.m == 32) e = launch_bwd<16, 32>(p, st);
+  else if (R == 16 && a.m == 64) e = launch_bwd<16, 64>(p, st);
+  else if (R == 16 && a.m == 128) e = launch_bwd<16, 128>(p, st);
+  if (e != cudaSuccess) return e;
+  // weight-gradient partials on the tensor cores, then the fixed-order sum
+  DwArgs d;
+  d.T = a.T; d.H = a.H; d.m = a.m; d.g = a.g; d.h = reinterpret_cast<const bf16*>(a.h);
+  d.z = a.z; d.dz = a.dz; d.partials = a.partials;
+  const int nchunk = adapter_dw_chunks(a.T, a.H);
+  d.chunk = (a.T + nchunk - 1) / nchunk;
+  dim3 grid(a.H / DWC, nchunk);
+  if (a.m == 32) adapter_dw_mma_kernel<32><<<grid, 256, 0, st>>>(d);
+  else if (a.m == 64) adapter_dw_mma_kernel<64><<<grid, 256, 0, st>>>(d);
+  else adapter_dw_mma_kernel<128><<<grid, 256, 0, st>>>(d);
+  note_launch(1);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return adapter_dw_reduce(a.partials, nchunk, a.H, a.m, a.dWd, a.dWu, st);
+}
+
+}  // namespace ra

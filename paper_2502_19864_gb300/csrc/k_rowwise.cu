@@ -560,14 +560,17 @@ __global__ void pack_rows_kernel(const float* src, void* dst, int R, int C, int 
 // transposed copies of the adapter matrices of layers [l0, l1): for each layer the four
 // matrices WdA [H,m], WuA [m,H], WdF [H,m], WuF [m,H] (contiguous, 4Hm per layer) go to
 // WdT [m,H], WuT [H,m], ... at the same offsets of PT.
-__global__ void adapter_transpose_kernel(const float* P, float* PT, int H, int m) {
+__global__ void adapter_transpose_kernel(const float* P, float* PT, bf16* PB, bf16* PTB, int H, int m) {
   int layer = blockIdx.z >> 2, mat = blockIdx.z & 3;
   int64_t base = (int64_t)layer * 4 * H * m + (int64_t)mat * H * m;
   int rows = (mat & 1) ? m : H, cols = (mat & 1) ? H : m;
   int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= (int64_t)rows * cols) return;
   int r = (int)(e / cols), c = (int)(e % cols);
-  PT[base + (int64_t)c * rows + r] = P[base + e];
+  const float v = P[base + e];
+  PT[base + (int64_t)c * rows + r] = v;
+  if (PB) PB[base + e] = __float2bfloat16_rn(v);
+  if (PTB) PTB[base + (int64_t)c * rows + r] = __float2bfloat16_rn(v);
 }
 
 __global__ void fill_kernel(float* dst, float v, int64_t n) {
@@ -582,6 +585,8 @@ inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1)
 // =========================================================================================
 cudaError_t adapter_fwd(const AdapterFwdArgs& a, cudaStream_t st) {
   if (a.m > MAXM || a.m <= 0) return cudaErrorInvalidValue;
+  if (a.dtype == DT_BF16 && a.WdT_b && a.WuT_b && adapter_mma_ok(a.H, a.m))
+    return adapter_fwd_mma(a, a.WdT_b, a.WuT_b, st);
   size_t smem = ((size_t)ROWS * a.H + ROWS * MAXM) * sizeof(float);
   unsigned grid = blocks_for(a.T, ROWS);
   if (a.dtype == DT_BF16) {
@@ -599,8 +604,21 @@ size_t adapter_bwd_partials_floats(int T, int H, int m) {
   return (size_t)dw_chunks(T, H) * 2 * H * m;
 }
 
+int adapter_dw_chunks(int T, int H) { return dw_chunks(T, H); }
+
+cudaError_t adapter_dw_reduce(const float* partials, int nchunk, int H, int m, float* dWd,
+                              float* dWu, cudaStream_t st) {
+  int64_t n = 2LL * H * m;
+  adapter_dw_reduce_kernel<<<blocks_for(n, 256), 256, 0, st>>>(partials, nchunk, H, m, dWd, dWu);
+  note_launch(1);
+  return cudaGetLastError();
+}
+
 cudaError_t adapter_bwd(const AdapterBwdArgs& a, cudaStream_t st) {
   if (a.m > MAXM || a.m <= 0) return cudaErrorInvalidValue;
+  if (a.dtype == DT_BF16 && a.Wu_b && a.Wd_b && adapter_mma_ok(a.H, a.m) &&
+      (!a.dh || a.dh_dtype == DT_BF16))
+    return adapter_bwd_mma(a, a.Wu_b, a.Wd_b, st);
   size_t smem = ((size_t)ROWS * a.H + ROWS * MAXM) * sizeof(float);
   unsigned grid = blocks_for(a.T, ROWS);
   if (a.dh_dtype == DT_BF16) {
@@ -737,10 +755,12 @@ cudaError_t pack_rows(const float* src, void* dst, int dst_dtype, int R, int C, 
   return cudaGetLastError();
 }
 
-cudaError_t adapter_transpose(const float* P, float* PT, int n_layers, int H, int m, cudaStream_t st) {
+cudaError_t adapter_transpose(const float* P, float* PT, void* PB, void* PTB, int n_layers,
+                              int H, int m, cudaStream_t st) {
   if (n_layers <= 0) return cudaSuccess;
   dim3 grid(blocks_for((int64_t)H * m, 256), 1, 4 * n_layers);
-  adapter_transpose_kernel<<<grid, 256, 0, st>>>(P, PT, H, m);
+  adapter_transpose_kernel<<<grid, 256, 0, st>>>(P, PT, reinterpret_cast<bf16*>(PB),
+                                                 reinterpret_cast<bf16*>(PTB), H, m);
   note_launch(1);
   return cudaGetLastError();
 }

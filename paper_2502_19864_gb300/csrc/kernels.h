@@ -96,8 +96,15 @@ struct AdapterFwdArgs {
   float* x_out = nullptr;       // decoder: f32 residual stream out
   void* xhat = nullptr;         // encoder: act [T, H] or null
   float* rstd = nullptr;        // [T] or null
+  // bf16 shadows of the adapter weights (bf16 models): W_down^T [m, H], W_up^T [H, m];
+  // when given (and the shape suits), the tensor-core kernel runs
+  const void* WdT_b = nullptr;
+  const void* WuT_b = nullptr;
 };
 cudaError_t adapter_fwd(const AdapterFwdArgs& a, cudaStream_t st);
+cudaError_t adapter_fwd_mma(const AdapterFwdArgs& a, const void* WdT_b, const void* WuT_b,
+                            cudaStream_t st);
+bool adapter_mma_ok(int H, int m);
 
 // Adapter backward, row part: dz = (g Wu^T) * GELU'(z) -> dz (f32 [T, m]);
 // dh = g + dz Wd^T -> dh (act) if non-null.  WuT [H, m] and WdT [m, H] are transposed copies.
@@ -114,9 +121,18 @@ struct AdapterBwdArgs {
   float* dWd = nullptr;         // [H, m]
   float* dWu = nullptr;         // [m, H]
   float* partials = nullptr;    // scratch, adapter_bwd_partials_floats(T, H, m)
+  // bf16 shadows (bf16 models): W_up [m, H], W_down [H, m]
+  const void* Wu_b = nullptr;
+  const void* Wd_b = nullptr;
 };
 size_t adapter_bwd_partials_floats(int T, int H, int m);
 cudaError_t adapter_bwd(const AdapterBwdArgs& a, cudaStream_t st);
+cudaError_t adapter_bwd_mma(const AdapterBwdArgs& a, const void* Wu_b, const void* Wd_b,
+                            cudaStream_t st);
+// chunk count of the dW reduction (a pure function of T and H) and its fixed-order sum
+int adapter_dw_chunks(int T, int H);
+cudaError_t adapter_dw_reduce(const float* partials, int nchunk, int H, int m, float* dWd,
+                              float* dWu, cudaStream_t st);
 
 // LayerNorm backward with frozen gamma: ds = rstd * (gy - mean(gy) - xhat mean(gy xhat)),
 // gy = dy * gamma.  dy f32, xhat act, ds f32.
@@ -171,8 +187,10 @@ cudaError_t transpose_f32(const float* src, void* dst, int dst_dtype, int rows, 
 // [2F, H] matrix in 64-row blocks alternating gate and up (or to its transpose [H, 2F]).
 cudaError_t pack_rows(const float* src, void* dst, int dst_dtype, int R, int C, int part,
                       bool transposed, cudaStream_t st);
-// Transposed f32 copies of the adapter matrices of n_layers consecutive layers.
-cudaError_t adapter_transpose(const float* P, float* PT, int n_layers, int H, int m, cudaStream_t st);
+// Transposed f32 copies of the adapter matrices of n_layers consecutive layers, and (when
+// PB / PTB are given) bf16 copies of both layouts.
+cudaError_t adapter_transpose(const float* P, float* PT, void* PB, void* PTB, int n_layers,
+                              int H, int m, cudaStream_t st);
 cudaError_t fill_f32(float* dst, float v, int64_t n, cudaStream_t st);
 
 }  // namespace ra

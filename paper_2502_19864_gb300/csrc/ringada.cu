@@ -42,6 +42,8 @@ struct Carve {
 struct LayerWOff {  // offsets into the weights region
   size_t Wqkv, WqkvT, bqkv, Wo, WoT, bo, W1, W1T, b1, W2, W2T, b2, g1, be1, g2, be2;
 };
+typedef uint16_t bf16_t;  // storage of the bf16 adapter shadows (host side never reads them)
+
 struct SlotOff {  // offsets of one saved-activation slot, relative to the slot base
   size_t qkv, O, lse, a, zA, xhat1, rstd1, u, f, zF, xhat2, rstd2;  // encoder
   size_t x_in, x1, gu;                                               // decoder extras
@@ -66,6 +68,7 @@ struct ra_ctx {
   size_t n_train = 0;       // floats in P (= G = M = V)
   size_t n_head = 0;        // encoder head floats at the end of P
   size_t t_P = 0, t_G = 0, t_M = 0, t_V = 0, t_PT = 0, t_steps = 0;
+  size_t t_PB = 0, t_PTB = 0;  // bf16 shadows of the adapters (both layouts), bf16 models
   // workspace
   SlotOff so{};
   size_t ws_err = 0, ws_arena = 0;
@@ -120,6 +123,16 @@ struct ra_ctx {
   float* G() const { return reinterpret_cast<float*>(Tr + t_G); }
   float* PT() const { return reinterpret_cast<float*>(Tr + t_PT); }
   int32_t* steps() const { return reinterpret_cast<int32_t*>(Tr + t_steps); }
+  bf16_t* PB() const { return act == DT_BF16 ? reinterpret_cast<bf16_t*>(Tr + t_PB) : nullptr; }
+  // bf16 shadow of adapter matrix `mat` (0 WdA [H,m], 1 WuA [m,H], 2 WdF, 3 WuF) of a layer,
+  // in the master layout (shadow) or transposed (shadowT); null for fp32 models
+  const void* shadow(int layer, int mat) const {
+    return act == DT_BF16 ? PB() + (size_t)layer * 4 * H * m + (size_t)mat * H * m : nullptr;
+  }
+  const void* shadowT(int layer, int mat) const {
+    return act == DT_BF16 ? PTB() + (size_t)layer * 4 * H * m + (size_t)mat * H * m : nullptr;
+  }
+  bf16_t* PTB() const { return act == DT_BF16 ? reinterpret_cast<bf16_t*>(Tr + t_PTB) : nullptr; }
   size_t per_layer_train() const { return (size_t)4 * H * m; }
   char* slot(int layer) const {  // slot base of a saved layer (layer >= L - max_depth)
     int s = layer - (L - max_depth);
@@ -225,6 +238,10 @@ void plan(ra_ctx* c) {
   c->t_V = t.take(c->n_train * 4);
   c->t_PT = t.take(L * 4 * H * m * 4);
   c->t_steps = t.take((L + 1) * 4);
+  if (c->act == DT_BF16) {
+    c->t_PB = t.take(L * 4 * H * m * 2);
+    c->t_PTB = t.take(L * 4 * H * m * 2);
+  }
   c->t_bytes = t.off;
   // ---- workspace ----
   const size_t Bh = (size_t)c->cfg.max_batch * c->nh * c->cfg.max_seq;  // lse rows
@@ -407,6 +424,7 @@ ra_status ra_set_weights(ra_ctx* ctx, const ra_tensor_desc* list, int32_t n, ra_
       return fail(ctx, RA_ERR_ARG, "entry %d: numel %lld, expected %lld", i, (long long)d.numel,
                   (long long)want);
   }
+  bool adapters_changed = false;
   for (int i = 0; i < n; ++i) {
     const ra_tensor_desc& d = list[i];
     const float* src = d.data_dev;
@@ -429,9 +447,7 @@ ra_status ra_set_weights(ra_ctx* ctx, const ra_tensor_desc* list, int32_t n, ra_
         case RA_P_WDA: case RA_P_WUA: case RA_P_WDF: case RA_P_WUF: {
           size_t off = (size_t)(d.param - RA_P_WDA) * H * m;
           CU(cudaMemcpyAsync(Pl + off, src, bytes, cudaMemcpyDeviceToDevice, st));
-          bool down = d.param == RA_P_WDA || d.param == RA_P_WDF;
-          int rows = down ? H : m, cols = down ? m : H;
-          CU(transpose_f32(src, ctx->PT() + (size_t)d.layer * 4 * H * m + off, DT_F32, rows, cols, rows, st));
+          adapters_changed = true;
         } break;
         case RA_P_WQKV:
           CU(convert_f32(src, ctx->w(o.Wqkv), act, d.numel, st));
@@ -472,6 +488,9 @@ ra_status ra_set_weights(ra_ctx* ctx, const ra_tensor_desc* list, int32_t n, ra_
     }
     ctx->set_mask[(size_t)(d.layer + 1) * RA_P_COUNT + d.param] = 1;
   }
+  // transposed and bf16 copies of the adapters the step's kernels read
+  if (adapters_changed)
+    CU(adapter_transpose(ctx->P(), ctx->PT(), ctx->PB(), ctx->PTB(), ctx->L, H, m, st));
   // every parameter of the model present?
   bool all = true;
   for (int l = -1; l < ctx->L && all; ++l)
@@ -612,6 +631,7 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     AdapterFwdArgs ad;
     ad.T = T; ad.H = H; ad.m = m; ad.dtype = act; ad.decoder = false;
     ad.a = a; ad.Wd = Pl; ad.Wu = Pl + (size_t)H * m; ad.z = zA; ad.resid = xin;
+    ad.WdT_b = ctx->shadowT(l, 0); ad.WuT_b = ctx->shadowT(l, 1);
     ad.gamma = ctx->w<float>(o.g1); ad.beta = ctx->w<float>(o.be1); ad.eps = ctx->cfg.norm_eps;
     ad.y = y1; ad.xhat = xhat1; ad.rstd = rstd1;
     CU(P_adapter_fwd(ctx, ad, st));
@@ -623,6 +643,7 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     g.C = f; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.b2);
     CU(P_gemm(ctx, g, st));
     ad.a = f; ad.Wd = Pl + (size_t)2 * H * m; ad.Wu = Pl + (size_t)3 * H * m; ad.z = zF;
+    ad.WdT_b = ctx->shadowT(l, 2); ad.WuT_b = ctx->shadowT(l, 3);
     ad.resid = y1; ad.gamma = ctx->w<float>(o.g2); ad.beta = ctx->w<float>(o.be2);
     ad.y = xout; ad.xhat = xhat2; ad.rstd = rstd2;
     CU(P_adapter_fwd(ctx, ad, st));
@@ -700,6 +721,7 @@ ra_status decoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     AdapterFwdArgs ad;
     ad.T = T; ad.H = H; ad.m = m; ad.dtype = act; ad.decoder = true;
     ad.a = a; ad.Wd = Pl; ad.Wu = Pl + (size_t)H * m; ad.z = zA; ad.resid = xin;
+    ad.WdT_b = ctx->shadowT(l, 0); ad.WuT_b = ctx->shadowT(l, 1);
     ad.gamma = ctx->w<float>(o.g2); ad.eps = ctx->cfg.norm_eps;
     ad.y = nbuf; ad.x_out = x1; ad.rstd = rstd2;
     CU(P_adapter_fwd(ctx, ad, st));
@@ -711,6 +733,7 @@ ra_status decoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     g.C = f; g.ldc = H; g.c_dtype = act;
     CU(P_gemm(ctx, g, st));
     ad.a = f; ad.Wd = Pl + (size_t)2 * H * m; ad.Wu = Pl + (size_t)3 * H * m; ad.z = zF;
+    ad.WdT_b = ctx->shadowT(l, 2); ad.WuT_b = ctx->shadowT(l, 3);
     ad.resid = x1; ad.gamma = gnext;
     ad.y = (l + 1 < L) ? nbuf : ctx->ws<void>(ctx->h_nf);
     ad.x_out = xnext; ad.rstd = rstd_next;
@@ -808,6 +831,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       // FFN-branch adapter: g = ds2, input f, z_F
       ab.g = ds2; ab.h = sb + so.f; ab.z = (float*)(sb + so.zF);
       ab.WuT = PTl + (size_t)3 * H * m; ab.WdT = PTl + (size_t)2 * H * m;
+      ab.Wu_b = ctx->shadow(l, 3); ab.Wd_b = ctx->shadow(l, 2);
       ab.dh = ctx->ws(ctx->b_df); ab.dh_dtype = act;
       ab.dWd = Gl + (size_t)2 * H * m; ab.dWu = Gl + (size_t)3 * H * m;
       CU(P_adapter_bwd(ctx, ab, st));
@@ -828,6 +852,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       // attention-branch adapter
       ab.g = ds1; ab.h = sb + so.a; ab.z = (float*)(sb + so.zA);
       ab.WuT = PTl + (size_t)H * m; ab.WdT = PTl;
+      ab.Wu_b = ctx->shadow(l, 1); ab.Wd_b = ctx->shadow(l, 0);
       ab.dh = lowest ? nullptr : ctx->ws(ctx->b_da);
       ab.dWd = Gl; ab.dWu = Gl + (size_t)H * m;
       CU(P_adapter_bwd(ctx, ab, st));
@@ -849,6 +874,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       // FFN-branch adapter: g = dY (= d x2), input f, z_F
       ab.g = dY; ab.h = sb + so.f; ab.z = (float*)(sb + so.zF);
       ab.WuT = PTl + (size_t)3 * H * m; ab.WdT = PTl + (size_t)2 * H * m;
+      ab.Wu_b = ctx->shadow(l, 3); ab.Wd_b = ctx->shadow(l, 2);
       ab.dh = ctx->ws(ctx->b_df); ab.dh_dtype = act;
       ab.dWd = Gl + (size_t)2 * H * m; ab.dWu = Gl + (size_t)3 * H * m;
       CU(P_adapter_bwd(ctx, ab, st));
@@ -866,6 +892,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
               [&] { return rmsnorm_bwd(dn2, (float*)(sb + so.x1), (float*)(sb + so.rstd2), ctx->w<float>(o.g2), dY, dx1, T, H, st); }));
       ab.g = dx1; ab.h = sb + so.a; ab.z = (float*)(sb + so.zA);
       ab.WuT = PTl + (size_t)H * m; ab.WdT = PTl;
+      ab.Wu_b = ctx->shadow(l, 1); ab.Wd_b = ctx->shadow(l, 0);
       ab.dh = lowest ? nullptr : ctx->ws(ctx->b_da);
       ab.dWd = Gl; ab.dWu = Gl + (size_t)H * m;
       CU(P_adapter_bwd(ctx, ab, st));
@@ -921,7 +948,9 @@ ra_status ra_adapter_update(ra_ctx* ctx, const ra_adam_cfg* adam, ra_stream_t st
   CU(prof(ctx, RA_PROF_UPDATE, 0, (double)a.n * 4 * 6 + (double)(L - k) * 4 * ctx->H * ctx->m * 8, st, [&] {
     cudaError_t e = adam_update(a, st);
     if (e == cudaSuccess) e = adam_bump(ctx->steps() + k, a.n_seg, st);
-    if (e == cudaSuccess) e = adapter_transpose(ctx->P() + off, ctx->PT() + off, L - k, ctx->H, ctx->m, st);
+    if (e == cudaSuccess)
+      e = adapter_transpose(ctx->P() + off, ctx->PT() + off, ctx->PB() ? ctx->PB() + off : nullptr,
+                            ctx->PTB() ? ctx->PTB() + off : nullptr, L - k, ctx->H, ctx->m, st);
     return e;
   }));
   ctx->bwd_since_update = false;
@@ -1008,7 +1037,7 @@ ra_status ra_set_trainable(ra_ctx* ctx, const void* host, size_t n) {
   CU(cudaMemcpy(ctx->Tr + ctx->t_M, p + fb, fb, cudaMemcpyHostToDevice));
   CU(cudaMemcpy(ctx->Tr + ctx->t_V, p + 2 * fb, fb, cudaMemcpyHostToDevice));
   CU(cudaMemcpy(ctx->Tr + ctx->t_steps, p + 3 * fb, (ctx->L + 1) * sizeof(int32_t), cudaMemcpyHostToDevice));
-  CU(adapter_transpose(ctx->P(), ctx->PT(), ctx->L, ctx->H, ctx->m, 0));
+  CU(adapter_transpose(ctx->P(), ctx->PT(), ctx->PB(), ctx->PTB(), ctx->L, ctx->H, ctx->m, 0));
   CU(cudaDeviceSynchronize());
   ctx->depth = (int)hdr[4];
   ctx->n_updates = (int)hdr[5];
