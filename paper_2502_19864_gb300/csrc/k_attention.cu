@@ -335,8 +335,10 @@ cudaError_t bwd_impl(const AttnArgs& a, cudaStream_t st) {
   int T_ = a.B * a.S;
   int64_t warps = (int64_t)T_ * a.n_heads;
   attn_bwd_pre_kernel<T><<<(unsigned)((warps * 32 + 255) / 256), 256, 0, st>>>(a);
+  note_launch(1);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  if (attention_mma_ok(a)) return attention_bwd_mma(a, st);
   int ld = a.head_dim + 1;
   size_t smem1 = (size_t)(2 * 64 * ld + 2 * 64 + 2 * 32 * ld) * sizeof(float);
   cudaFuncSetAttribute(attn_bwd_dkdv_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
@@ -346,7 +348,7 @@ cudaError_t bwd_impl(const AttnArgs& a, cudaStream_t st) {
   size_t smem2 = (size_t)(2 * KB * ld + 2 * 32 * ld) * sizeof(float);
   cudaFuncSetAttribute(attn_bwd_dq_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
   attn_bwd_dq_kernel<T><<<dim3((a.S + 31) / 32, a.B * a.n_heads), 256, smem2, st>>>(a);
-  note_launch(3);
+  note_launch(2);
   return cudaGetLastError();
 }
 
@@ -354,6 +356,7 @@ cudaError_t bwd_impl(const AttnArgs& a, cudaStream_t st) {
 
 cudaError_t attention_fwd(const AttnArgs& a, cudaStream_t st) {
   if (a.head_dim > MAXD || a.head_dim % 32 != 0) return cudaErrorInvalidValue;
+  if (attention_mma_ok(a)) return attention_fwd_mma(a, st);
   return a.dtype == DT_BF16 ? fwd_impl<bf16>(a, st) : fwd_impl<float>(a, st);
 }
 

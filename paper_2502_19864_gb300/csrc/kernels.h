@@ -73,6 +73,10 @@ struct AttnArgs {
 };
 cudaError_t attention_fwd(const AttnArgs& a, cudaStream_t st);
 cudaError_t attention_bwd(const AttnArgs& a, cudaStream_t st);
+// tensor-core versions (bf16, head_dim 64 or 128); the backward expects D in a.Dscratch
+bool attention_mma_ok(const AttnArgs& a);
+cudaError_t attention_fwd_mma(const AttnArgs& a, cudaStream_t st);
+cudaError_t attention_bwd_mma(const AttnArgs& a, cudaStream_t st);
 
 // ---------------------------------------------------------------------------------------
 // Row-wise fused kernels
