@@ -229,6 +229,15 @@ typedef struct {
 ra_status ra_profile_enable(ra_ctx* ctx, int32_t on);
 /* Sums the records; the caller must have synchronised the recorded work first. */
 ra_status ra_profile_read(ra_ctx* ctx, ra_profile* out);
+/* The individual records behind ra_profile_read, in call order: category, device
+ * milliseconds, algorithmic flops and bytes of each recorded kernel call.  Writes up to
+ * `max` records to out (host array) and the total number to *n. */
+typedef struct {
+  int32_t cat;
+  float ms;
+  double flops, bytes;
+} ra_profile_record;
+ra_status ra_profile_records(ra_ctx* ctx, ra_profile_record* out, int32_t max, int32_t* n);
 /* Kernels this library has launched in this process so far (every entry point). */
 int64_t ra_kernel_launches(void);
 

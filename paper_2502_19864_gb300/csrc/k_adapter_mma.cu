@@ -11,17 +11,18 @@
 //   backward  dz = (g W_up^T) * GELU'(z); dh = g + dz W_down^T;
 //   dW        per row-chunk partials of dW_up = GELU(z)^T g and dW_down^T = dz^T h, summed
 //             afterwards in a fixed order (deterministic).
-// CTA = R rows (16 or 32) x H / 128 warps.  Phase 1 (the reduction over H) splits K across
-// warps and sums the per-warp partials of z in a fixed order; phase 2 splits the H output
-// columns across warps; row statistics for the norm are combined across warps in shared
-// memory in a fixed order.
+// CTA = 16 rows x H / 64 warps (64 registers per thread, two CTAs per SM up to H = 1024).
+// Phase 1 (the reduction over H) splits K across warps in slices of 64 (128 when the
+// partial buffer would pass 64 KB) and sums the per-warp partials of z in a fixed order;
+// phase 2 gives each warp 64 of the H output columns; row statistics for the norm are
+// combined across warps in shared memory in a fixed order.
 #include "common.cuh"
 #include "kernels.h"
 
 namespace ra {
 namespace {
 
-constexpr int COLS_PER_WARP = 128;
+constexpr int COLS_PER_WARP = 64, R = 16;
 
 __device__ __forceinline__ void mma_bf16(float* d, const uint32_t* a, uint32_t b0, uint32_t b1) {
   asm volatile(
@@ -61,65 +62,59 @@ __device__ __forceinline__ void load_a(uint32_t* a, const bf16* s, int ld, int r
   ldsm_x4(a, s + (size_t)r * ld + c);
 }
 
-// Phase 1 shared by forward and backward: partial[w] = X[R, kslice] * Bw^T over this warp's
-// 128-wide slice of H, where Bw is [m, H] row-major bf16 in global memory (B fragments
-// read directly; the matrix is small and stays in L1/L2).
-template <int MT, int NT>
-__device__ __forceinline__ void phase1(float (&acc)[MT][NT][4], const bf16* Xs, int ldx,
-                                       const bf16* Bw, int H, int kbase, int lane) {
+// Phase 1 shared by forward and backward: part[w] = X[16, kslice] * Bw^T over this warp's
+// slice [kbase, kbase + ks_len) of H, where Bw is [m, H] row-major bf16 in global memory (B
+// fragments read directly; the matrix is small and stays in L1/L2).  The m output columns
+// are produced in groups of 8 n-tiles to bound the registers.
+template <int MB>
+__device__ __forceinline__ void phase1_store(const bf16* Xs, int ldx, const bf16* Bw, int H,
+                                             int kbase, int ks_len, float* part, int lane) {
   const int g = lane >> 2, t = lane & 3;
+  constexpr int NG = MB >= 64 ? MB / 64 : 1, NTG = MB >= 64 ? 8 : MB / 8;
+#pragma unroll 1
+  for (int ng = 0; ng < NG; ++ng) {
+    float acc[NTG][4];
 #pragma unroll
-  for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-      for (int i = 0; i < 4; ++i) acc[mt][nt][i] = 0.f;
+    for (int nt = 0; nt < NTG; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
 #pragma unroll 2
-  for (int ks = 0; ks < COLS_PER_WARP / 16; ++ks) {
-    const int k0 = kbase + ks * 16;
-    uint32_t a[MT][4];
+    for (int k0 = kbase; k0 < kbase + ks_len; k0 += 16) {
+      uint32_t a[4];
+      load_a(a, Xs, ldx, 0, k0, lane);
 #pragma unroll
-    for (int mt = 0; mt < MT; ++mt) load_a(a[mt], Xs, ldx, mt * 16, k0, lane);
+      for (int nt = 0; nt < NTG; ++nt) {
+        const bf16* bp = Bw + (size_t)(ng * 64 + nt * 8 + g) * H + k0 + 2 * t;
+        mma_bf16(acc[nt], a, ld_u32(bp), ld_u32(bp + 8));
+      }
+    }
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-      const bf16* bp = Bw + (size_t)(nt * 8 + g) * H + k0 + 2 * t;
-      const uint32_t b0 = ld_u32(bp), b1 = ld_u32(bp + 8);
-#pragma unroll
-      for (int mt = 0; mt < MT; ++mt) mma_bf16(acc[mt][nt], a[mt], b0, b1);
+    for (int nt = 0; nt < NTG; ++nt) {
+      const int c = ng * 64 + nt * 8 + 2 * t;
+      *reinterpret_cast<float2*>(part + g * MB + c) = make_float2(acc[nt][0], acc[nt][1]);
+      *reinterpret_cast<float2*>(part + (g + 8) * MB + c) = make_float2(acc[nt][2], acc[nt][3]);
     }
   }
 }
 
-template <int MT, int NT>
-__device__ __forceinline__ void store_partial(const float (&acc)[MT][NT][4], float* part, int m,
-                                              int lane) {
-  const int g = lane >> 2, t = lane & 3;
-#pragma unroll
-  for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-      const int r = mt * 16 + g, c = nt * 8 + 2 * t;
-      *reinterpret_cast<float2*>(part + r * m + c) = make_float2(acc[mt][nt][0], acc[mt][nt][1]);
-      *reinterpret_cast<float2*>(part + (r + 8) * m + c) = make_float2(acc[mt][nt][2], acc[mt][nt][3]);
-    }
+// K-slice of phase 1: 64 columns of H per warp unless the per-warp partials of z would pass
+// 64 KB of shared memory, then 128 (and only the first H / 128 warps take part)
+__host__ __device__ inline int phase1_slice(int H, int m) {
+  return (H / 64) * R * m * 4 > 65536 ? 128 : 64;
 }
 
-// Phase 2: acc[16 rows of tile mt, this warp's 128 columns] = S[16, m] * Bn^T where Bn is
-// [H, m] row-major bf16 (n = output column, k = bottleneck index).
+// Phase 2: acc[16 rows, this warp's 64 columns] = S[16, m] * Bn^T where Bn is [H, m]
+// row-major bf16 (n = output column, k = bottleneck index).
 template <int MB>
-__device__ __forceinline__ void phase2(float (&acc)[16][4], const bf16* Ss, int lds, int mt,
+__device__ __forceinline__ void phase2(float (&acc)[8][4], const bf16* Ss, int lds,
                                        const bf16* Bn, int m, int nbase, int lane) {
   const int g = lane >> 2, t = lane & 3;
 #pragma unroll
-  for (int nt = 0; nt < 16; ++nt)
-#pragma unroll
-    for (int i = 0; i < 4; ++i) acc[nt][i] = 0.f;
+  for (int nt = 0; nt < 8; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
 #pragma unroll
   for (int ks = 0; ks < MB / 16; ++ks) {
     uint32_t a[4];
-    load_a(a, Ss, lds, mt * 16, ks * 16, lane);
+    load_a(a, Ss, lds, 0, ks * 16, lane);
 #pragma unroll
-    for (int nt = 0; nt < 16; ++nt) {
+    for (int nt = 0; nt < 8; ++nt) {
       const bf16* bp = Bn + (size_t)(nbase + nt * 8 + g) * m + ks * 16 + 2 * t;
       mma_bf16(acc[nt], a, ld_u32(bp), ld_u32(bp + 8));
     }
@@ -165,17 +160,17 @@ __device__ __forceinline__ void load_rows_f32_as_bf16(bf16* dst, int ld, const f
   }
 }
 
-// WIDE: H > 1024 (up to 512 threads, 128 registers); otherwise <= 256 threads and up to 255
-// registers.  32-row tiles run only with H <= 1024.
-template <int R, int MB, bool DEC, bool WIDE>
-__global__ void __launch_bounds__(WIDE ? 512 : 256, 1) adapter_fwd_mma_kernel(FwdArgs p) {
-  constexpr int MT = R / 16, NT1 = MB / 8;
+// WIDE: H > 1024 (up to 1024 threads, one CTA per SM); otherwise up to 512 threads and two
+// CTAs per SM.  Both cap the registers at 64 per thread.
+template <int MB, bool DEC, bool WIDE>
+__global__ void __launch_bounds__(WIDE ? 1024 : 512, WIDE ? 1 : 2) adapter_fwd_mma_kernel(FwdArgs p) {
   extern __shared__ __align__(16) uint8_t sm[];
   const int H = p.H, W = H / COLS_PER_WARP;
+  const int KS = phase1_slice(H, MB), W1 = H / KS;
   const int lda = H + 8, lds = MB + 8;
   bf16* As = reinterpret_cast<bf16*>(sm);                         // [R][H + 8]
-  float* part = reinterpret_cast<float*>(As + (size_t)R * lda);   // [W][R][MB]
-  bf16* Ss = reinterpret_cast<bf16*>(part + (size_t)W * R * MB);  // [R][MB + 8]
+  float* part = reinterpret_cast<float*>(As + (size_t)R * lda);   // [W1][R][MB]
+  bf16* Ss = reinterpret_cast<bf16*>(part + (size_t)W1 * R * MB); // [R][MB + 8]
   float* stat = reinterpret_cast<float*>(Ss + (size_t)R * lds);   // [W][16]
   float* rowv = stat + W * 16;                                    // [16]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -184,131 +179,124 @@ __global__ void __launch_bounds__(WIDE ? 512 : 256, 1) adapter_fwd_mma_kernel(Fw
 
   load_rows_bf16(As, lda, p.a, t0, p.T, H, R);
   __syncthreads();
-  {
-    float acc[MT][NT1][4];
-    phase1<MT, NT1>(acc, As, lda, p.WdT, H, warp * COLS_PER_WARP, lane);
-    store_partial<MT, NT1>(acc, part + (size_t)warp * R * MB, MB, lane);
-  }
+  if (warp < W1) phase1_store<MB>(As, lda, p.WdT, H, warp * KS, KS, part + (size_t)warp * R * MB, lane);
   __syncthreads();
   for (int e = threadIdx.x; e < R * MB; e += blockDim.x) {
     const int r = e / MB, j = e % MB;
     float zs = 0.f;
-    for (int w = 0; w < W; ++w) zs += part[((size_t)w * R + r) * MB + j];
+    for (int w = 0; w < W1; ++w) zs += part[((size_t)w * R + r) * MB + j];
     if (p.z && t0 + r < p.T) p.z[(size_t)(t0 + r) * MB + j] = zs;
     Ss[r * lds + j] = __float2bfloat16_rn(gelu_f(zs));
   }
   __syncthreads();
   const int nbase = warp * COLS_PER_WARP;
-  for (int mt = 0; mt < MT; ++mt) {
-    float v[16][4];
-    phase2<MB>(v, Ss, lds, mt, p.WuT, MB, nbase, lane);
-    const int rl0 = mt * 16 + g, rl1 = rl0 + 8;           // local rows of c0/c1 and c2/c3
-    const int r0 = t0 + rl0, r1 = t0 + rl1;
-    float s0 = 0.f, s1 = 0.f;
+  float v[8][4];
+  phase2<MB>(v, Ss, lds, p.WuT, MB, nbase, lane);
+  const int rl0 = g, rl1 = g + 8;  // local rows of c0/c1 and c2/c3
+  const int r0 = t0 + rl0, r1 = t0 + rl1;
+  float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-    for (int nt = 0; nt < 16; ++nt) {
+  for (int nt = 0; nt < 8; ++nt) {
+    const int c = nbase + nt * 8 + 2 * t;
+    float2 a0 = unpack2(*reinterpret_cast<const uint32_t*>(As + (size_t)rl0 * lda + c));
+    float2 a1 = unpack2(*reinterpret_cast<const uint32_t*>(As + (size_t)rl1 * lda + c));
+    float2 q0 = make_float2(0.f, 0.f), q1 = make_float2(0.f, 0.f);
+    if (DEC) {
+      const float* rs = reinterpret_cast<const float*>(p.resid);
+      if (r0 < p.T) q0 = *reinterpret_cast<const float2*>(rs + (size_t)r0 * H + c);
+      if (r1 < p.T) q1 = *reinterpret_cast<const float2*>(rs + (size_t)r1 * H + c);
+    } else {
+      const bf16* rs = reinterpret_cast<const bf16*>(p.resid);
+      if (r0 < p.T) q0 = unpack2(*reinterpret_cast<const uint32_t*>(rs + (size_t)r0 * H + c));
+      if (r1 < p.T) q1 = unpack2(*reinterpret_cast<const uint32_t*>(rs + (size_t)r1 * H + c));
+    }
+    v[nt][0] += a0.x + q0.x; v[nt][1] += a0.y + q0.y;
+    v[nt][2] += a1.x + q1.x; v[nt][3] += a1.y + q1.y;
+    if (DEC) {
+      s0 += v[nt][0] * v[nt][0] + v[nt][1] * v[nt][1];
+      s1 += v[nt][2] * v[nt][2] + v[nt][3] * v[nt][3];
+    } else {
+      s0 += v[nt][0] + v[nt][1];
+      s1 += v[nt][2] + v[nt][3];
+    }
+  }
+  // row sums across the quad, then across warps (fixed order)
+  s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
+  s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+  s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
+  s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+  if (t == 0) { stat[warp * 16 + g] = s0; stat[warp * 16 + g + 8] = s1; }
+  __syncthreads();
+  if (threadIdx.x < 16) {
+    float s = 0.f;
+    for (int w = 0; w < W; ++w) s += stat[w * 16 + threadIdx.x];
+    rowv[threadIdx.x] = s / H;
+  }
+  __syncthreads();
+  if (DEC) {
+    const float rs0 = rsqrtf(rowv[g] + p.eps), rs1 = rsqrtf(rowv[g + 8] + p.eps);
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
       const int c = nbase + nt * 8 + 2 * t;
-      float2 a0 = unpack2(*reinterpret_cast<const uint32_t*>(As + (size_t)rl0 * lda + c));
-      float2 a1 = unpack2(*reinterpret_cast<const uint32_t*>(As + (size_t)rl1 * lda + c));
-      float2 q0 = make_float2(0.f, 0.f), q1 = make_float2(0.f, 0.f);
-      if (DEC) {
-        const float* rs = reinterpret_cast<const float*>(p.resid);
-        if (r0 < p.T) q0 = *reinterpret_cast<const float2*>(rs + (size_t)r0 * H + c);
-        if (r1 < p.T) q1 = *reinterpret_cast<const float2*>(rs + (size_t)r1 * H + c);
-      } else {
-        const bf16* rs = reinterpret_cast<const bf16*>(p.resid);
-        if (r0 < p.T) q0 = unpack2(*reinterpret_cast<const uint32_t*>(rs + (size_t)r0 * H + c));
-        if (r1 < p.T) q1 = unpack2(*reinterpret_cast<const uint32_t*>(rs + (size_t)r1 * H + c));
+      const float2 gm = *reinterpret_cast<const float2*>(p.gamma + c);
+      if (r0 < p.T) {
+        *reinterpret_cast<float2*>(p.x_out + (size_t)r0 * H + c) = make_float2(v[nt][0], v[nt][1]);
+        *reinterpret_cast<uint32_t*>(p.y + (size_t)r0 * H + c) =
+            pack2(v[nt][0] * rs0 * gm.x, v[nt][1] * rs0 * gm.y);
       }
-      v[nt][0] += a0.x + q0.x; v[nt][1] += a0.y + q0.y;
-      v[nt][2] += a1.x + q1.x; v[nt][3] += a1.y + q1.y;
-      if (DEC) {
-        s0 += v[nt][0] * v[nt][0] + v[nt][1] * v[nt][1];
-        s1 += v[nt][2] * v[nt][2] + v[nt][3] * v[nt][3];
-      } else {
-        s0 += v[nt][0] + v[nt][1];
-        s1 += v[nt][2] + v[nt][3];
+      if (r1 < p.T) {
+        *reinterpret_cast<float2*>(p.x_out + (size_t)r1 * H + c) = make_float2(v[nt][2], v[nt][3]);
+        *reinterpret_cast<uint32_t*>(p.y + (size_t)r1 * H + c) =
+            pack2(v[nt][2] * rs1 * gm.x, v[nt][3] * rs1 * gm.y);
       }
     }
-    // row sums across the quad, then across warps (fixed order)
-    s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
-    s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
-    s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
-    s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
-    if (t == 0) { stat[warp * 16 + g] = s0; stat[warp * 16 + g + 8] = s1; }
+    if (p.rstd && warp == 0 && t == 0) {
+      if (r0 < p.T) p.rstd[r0] = rs0;
+      if (r1 < p.T) p.rstd[r1] = rs1;
+    }
+  } else {
+    const float mu0 = rowv[g], mu1 = rowv[g + 8];
+    float q0 = 0.f, q1 = 0.f;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      v[nt][0] -= mu0; v[nt][1] -= mu0; v[nt][2] -= mu1; v[nt][3] -= mu1;
+      q0 += v[nt][0] * v[nt][0] + v[nt][1] * v[nt][1];
+      q1 += v[nt][2] * v[nt][2] + v[nt][3] * v[nt][3];
+    }
+    q0 += __shfl_xor_sync(0xffffffffu, q0, 1);
+    q0 += __shfl_xor_sync(0xffffffffu, q0, 2);
+    q1 += __shfl_xor_sync(0xffffffffu, q1, 1);
+    q1 += __shfl_xor_sync(0xffffffffu, q1, 2);
+    __syncthreads();  // everyone has read rowv
+    if (t == 0) { stat[warp * 16 + g] = q0; stat[warp * 16 + g + 8] = q1; }
     __syncthreads();
     if (threadIdx.x < 16) {
       float s = 0.f;
       for (int w = 0; w < W; ++w) s += stat[w * 16 + threadIdx.x];
-      rowv[threadIdx.x] = s / H;
+      rowv[threadIdx.x] = rsqrtf(s / H + p.eps);
     }
     __syncthreads();
-    if (DEC) {
-      const float rs0 = rsqrtf(rowv[g] + p.eps), rs1 = rsqrtf(rowv[g + 8] + p.eps);
+    const float rs0 = rowv[g], rs1 = rowv[g + 8];
 #pragma unroll
-      for (int nt = 0; nt < 16; ++nt) {
-        const int c = nbase + nt * 8 + 2 * t;
-        const float2 gm = *reinterpret_cast<const float2*>(p.gamma + c);
-        if (r0 < p.T) {
-          *reinterpret_cast<float2*>(p.x_out + (size_t)r0 * H + c) = make_float2(v[nt][0], v[nt][1]);
-          *reinterpret_cast<uint32_t*>(p.y + (size_t)r0 * H + c) =
-              pack2(v[nt][0] * rs0 * gm.x, v[nt][1] * rs0 * gm.y);
-        }
-        if (r1 < p.T) {
-          *reinterpret_cast<float2*>(p.x_out + (size_t)r1 * H + c) = make_float2(v[nt][2], v[nt][3]);
-          *reinterpret_cast<uint32_t*>(p.y + (size_t)r1 * H + c) =
-              pack2(v[nt][2] * rs1 * gm.x, v[nt][3] * rs1 * gm.y);
-        }
+    for (int nt = 0; nt < 8; ++nt) {
+      const int c = nbase + nt * 8 + 2 * t;
+      const float2 gm = *reinterpret_cast<const float2*>(p.gamma + c);
+      const float2 bt = *reinterpret_cast<const float2*>(p.beta + c);
+      const float x00 = v[nt][0] * rs0, x01 = v[nt][1] * rs0;
+      const float x10 = v[nt][2] * rs1, x11 = v[nt][3] * rs1;
+      if (r0 < p.T) {
+        *reinterpret_cast<uint32_t*>(p.y + (size_t)r0 * H + c) = pack2(x00 * gm.x + bt.x, x01 * gm.y + bt.y);
+        if (p.xhat) *reinterpret_cast<uint32_t*>(p.xhat + (size_t)r0 * H + c) = pack2(x00, x01);
       }
-      if (p.rstd && warp == 0 && t == 0) {
-        if (r0 < p.T) p.rstd[r0] = rs0;
-        if (r1 < p.T) p.rstd[r1] = rs1;
-      }
-    } else {
-      const float mu0 = rowv[g], mu1 = rowv[g + 8];
-      float q0 = 0.f, q1 = 0.f;
-#pragma unroll
-      for (int nt = 0; nt < 16; ++nt) {
-        v[nt][0] -= mu0; v[nt][1] -= mu0; v[nt][2] -= mu1; v[nt][3] -= mu1;
-        q0 += v[nt][0] * v[nt][0] + v[nt][1] * v[nt][1];
-        q1 += v[nt][2] * v[nt][2] + v[nt][3] * v[nt][3];
-      }
-      q0 += __shfl_xor_sync(0xffffffffu, q0, 1);
-      q0 += __shfl_xor_sync(0xffffffffu, q0, 2);
-      q1 += __shfl_xor_sync(0xffffffffu, q1, 1);
-      q1 += __shfl_xor_sync(0xffffffffu, q1, 2);
-      __syncthreads();  // everyone has read rowv
-      if (t == 0) { stat[warp * 16 + g] = q0; stat[warp * 16 + g + 8] = q1; }
-      __syncthreads();
-      if (threadIdx.x < 16) {
-        float s = 0.f;
-        for (int w = 0; w < W; ++w) s += stat[w * 16 + threadIdx.x];
-        rowv[threadIdx.x] = rsqrtf(s / H + p.eps);
-      }
-      __syncthreads();
-      const float rs0 = rowv[g], rs1 = rowv[g + 8];
-#pragma unroll
-      for (int nt = 0; nt < 16; ++nt) {
-        const int c = nbase + nt * 8 + 2 * t;
-        const float2 gm = *reinterpret_cast<const float2*>(p.gamma + c);
-        const float2 bt = *reinterpret_cast<const float2*>(p.beta + c);
-        const float x00 = v[nt][0] * rs0, x01 = v[nt][1] * rs0;
-        const float x10 = v[nt][2] * rs1, x11 = v[nt][3] * rs1;
-        if (r0 < p.T) {
-          *reinterpret_cast<uint32_t*>(p.y + (size_t)r0 * H + c) = pack2(x00 * gm.x + bt.x, x01 * gm.y + bt.y);
-          if (p.xhat) *reinterpret_cast<uint32_t*>(p.xhat + (size_t)r0 * H + c) = pack2(x00, x01);
-        }
-        if (r1 < p.T) {
-          *reinterpret_cast<uint32_t*>(p.y + (size_t)r1 * H + c) = pack2(x10 * gm.x + bt.x, x11 * gm.y + bt.y);
-          if (p.xhat) *reinterpret_cast<uint32_t*>(p.xhat + (size_t)r1 * H + c) = pack2(x10, x11);
-        }
-      }
-      if (p.rstd && warp == 0 && t == 0) {
-        if (r0 < p.T) p.rstd[r0] = rs0;
-        if (r1 < p.T) p.rstd[r1] = rs1;
+      if (r1 < p.T) {
+        *reinterpret_cast<uint32_t*>(p.y + (size_t)r1 * H + c) = pack2(x10 * gm.x + bt.x, x11 * gm.y + bt.y);
+        if (p.xhat) *reinterpret_cast<uint32_t*>(p.xhat + (size_t)r1 * H + c) = pack2(x10, x11);
       }
     }
-    __syncthreads();  // stat / rowv reused by the next row tile
+    if (p.rstd && warp == 0 && t == 0) {
+      if (r0 < p.T) p.rstd[r0] = rs0;
+      if (r1 < p.T) p.rstd[r1] = rs1;
+    }
   }
 }
 
@@ -325,31 +313,27 @@ struct BwdArgs {
   bf16* dh;           // [T, H] or null
 };
 
-template <int R, int MB, bool WIDE>
-__global__ void __launch_bounds__(WIDE ? 512 : 256, 1) adapter_bwd_rows_mma_kernel(BwdArgs p) {
-  constexpr int MT = R / 16, NT1 = MB / 8;
+template <int MB, bool WIDE>
+__global__ void __launch_bounds__(WIDE ? 1024 : 512, WIDE ? 1 : 2) adapter_bwd_rows_mma_kernel(BwdArgs p) {
   extern __shared__ __align__(16) uint8_t sm[];
-  const int H = p.H, W = H / COLS_PER_WARP;
+  const int H = p.H;
+  const int KS = phase1_slice(H, MB), W1 = H / KS;
   const int ldg = H + 8, lds = MB + 8;
   bf16* Gs = reinterpret_cast<bf16*>(sm);
   float* part = reinterpret_cast<float*>(Gs + (size_t)R * ldg);
-  bf16* Ds = reinterpret_cast<bf16*>(part + (size_t)W * R * MB);
+  bf16* Ds = reinterpret_cast<bf16*>(part + (size_t)W1 * R * MB);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, t = lane & 3;
   const int t0 = blockIdx.x * R;
 
   load_rows_f32_as_bf16(Gs, ldg, p.g, t0, p.T, H, R);
   __syncthreads();
-  {
-    float acc[MT][NT1][4];
-    phase1<MT, NT1>(acc, Gs, ldg, p.Wu, H, warp * COLS_PER_WARP, lane);
-    store_partial<MT, NT1>(acc, part + (size_t)warp * R * MB, MB, lane);
-  }
+  if (warp < W1) phase1_store<MB>(Gs, ldg, p.Wu, H, warp * KS, KS, part + (size_t)warp * R * MB, lane);
   __syncthreads();
   for (int e = threadIdx.x; e < R * MB; e += blockDim.x) {
     const int r = e / MB, j = e % MB;
     float ds = 0.f;
-    for (int w = 0; w < W; ++w) ds += part[((size_t)w * R + r) * MB + j];
+    for (int w = 0; w < W1; ++w) ds += part[((size_t)w * R + r) * MB + j];
     float dz = 0.f;
     if (t0 + r < p.T) {
       dz = ds * gelu_grad_f(p.z[(size_t)(t0 + r) * MB + j]);
@@ -360,21 +344,19 @@ __global__ void __launch_bounds__(WIDE ? 512 : 256, 1) adapter_bwd_rows_mma_kern
   if (!p.dh) return;
   __syncthreads();
   const int nbase = warp * COLS_PER_WARP;
-  for (int mt = 0; mt < MT; ++mt) {
-    float v[16][4];
-    phase2<MB>(v, Ds, lds, mt, p.Wd, MB, nbase, lane);
-    const int r0 = t0 + mt * 16 + g, r1 = r0 + 8;
+  float v[8][4];
+  phase2<MB>(v, Ds, lds, p.Wd, MB, nbase, lane);
+  const int r0 = t0 + g, r1 = r0 + 8;
 #pragma unroll
-    for (int nt = 0; nt < 16; ++nt) {
-      const int c = nbase + nt * 8 + 2 * t;
-      if (r0 < p.T) {
-        const float2 q = *reinterpret_cast<const float2*>(p.g + (size_t)r0 * H + c);
-        *reinterpret_cast<uint32_t*>(p.dh + (size_t)r0 * H + c) = pack2(v[nt][0] + q.x, v[nt][1] + q.y);
-      }
-      if (r1 < p.T) {
-        const float2 q = *reinterpret_cast<const float2*>(p.g + (size_t)r1 * H + c);
-        *reinterpret_cast<uint32_t*>(p.dh + (size_t)r1 * H + c) = pack2(v[nt][2] + q.x, v[nt][3] + q.y);
-      }
+  for (int nt = 0; nt < 8; ++nt) {
+    const int c = nbase + nt * 8 + 2 * t;
+    if (r0 < p.T) {
+      const float2 q = *reinterpret_cast<const float2*>(p.g + (size_t)r0 * H + c);
+      *reinterpret_cast<uint32_t*>(p.dh + (size_t)r0 * H + c) = pack2(v[nt][0] + q.x, v[nt][1] + q.y);
+    }
+    if (r1 < p.T) {
+      const float2 q = *reinterpret_cast<const float2*>(p.g + (size_t)r1 * H + c);
+      *reinterpret_cast<uint32_t*>(p.dh + (size_t)r1 * H + c) = pack2(v[nt][2] + q.x, v[nt][3] + q.y);
     }
   }
 }
@@ -420,32 +402,49 @@ __global__ void __launch_bounds__(256) adapter_dw_mma_kernel(DwArgs p) {
       for (int i = 0; i < 4; ++i) acc[a][nt][i] = 0.f;
   const bf16* X = which ? Dsm : Ssm;
   const bf16* Y = which ? Hsm : Gsm;
+  // each thread's share of one 32-row tile: (z, dz) pairs and (g, h) quads
+  constexpr int NZ = DWR * (MB / 2) / 256, NG = DWR * (DWC / 4) / 256;
+  float2 zr[NZ], dr[NZ];
+  float4 gr[NG];
+  uint2 hr[NG];
+  auto fetch = [&](int r0) {
+#pragma unroll
+    for (int q = 0; q < NZ; ++q) {
+      const int e = threadIdx.x + q * 256, r = e / (MB / 2), j = (e % (MB / 2)) * 2, tt = r0 + r;
+      zr[q] = dr[q] = make_float2(0.f, 0.f);
+      if (tt < te) {
+        zr[q] = *reinterpret_cast<const float2*>(p.z + (size_t)tt * MB + j);
+        dr[q] = *reinterpret_cast<const float2*>(p.dz + (size_t)tt * MB + j);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < NG; ++q) {
+      const int e = threadIdx.x + q * 256, r = e / (DWC / 4), i = (e % (DWC / 4)) * 4, tt = r0 + r;
+      gr[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+      hr[q] = make_uint2(0, 0);
+      if (tt < te) {
+        gr[q] = *reinterpret_cast<const float4*>(p.g + (size_t)tt * H + i0 + i);
+        hr[q] = *reinterpret_cast<const uint2*>(p.h + (size_t)tt * H + i0 + i);
+      }
+    }
+  };
+  if (tb < te) fetch(tb);
   for (int r0 = tb; r0 < te; r0 += DWR) {
     __syncthreads();
-    for (int e = threadIdx.x; e < DWR * (MB / 2); e += blockDim.x) {
-      const int r = e / (MB / 2), j = (e % (MB / 2)) * 2, tt = r0 + r;
-      float2 zz = make_float2(0.f, 0.f), dd = make_float2(0.f, 0.f);
-      if (tt < te) {
-        zz = *reinterpret_cast<const float2*>(p.z + (size_t)tt * MB + j);
-        dd = *reinterpret_cast<const float2*>(p.dz + (size_t)tt * MB + j);
-        zz.x = gelu_f(zz.x);
-        zz.y = gelu_f(zz.y);
-      }
-      *reinterpret_cast<uint32_t*>(Ssm + r * LDJ + j) = pack2(zz.x, zz.y);
-      *reinterpret_cast<uint32_t*>(Dsm + r * LDJ + j) = pack2(dd.x, dd.y);
+#pragma unroll
+    for (int q = 0; q < NZ; ++q) {
+      const int e = threadIdx.x + q * 256, r = e / (MB / 2), j = (e % (MB / 2)) * 2;
+      *reinterpret_cast<uint32_t*>(Ssm + r * LDJ + j) = pack2(gelu_f(zr[q].x), gelu_f(zr[q].y));
+      *reinterpret_cast<uint32_t*>(Dsm + r * LDJ + j) = pack2(dr[q].x, dr[q].y);
     }
-    for (int e = threadIdx.x; e < DWR * (DWC / 4); e += blockDim.x) {
-      const int r = e / (DWC / 4), i = (e % (DWC / 4)) * 4, tt = r0 + r;
-      float4 gg = make_float4(0.f, 0.f, 0.f, 0.f);
-      uint2 hh = make_uint2(0, 0);
-      if (tt < te) {
-        gg = *reinterpret_cast<const float4*>(p.g + (size_t)tt * H + i0 + i);
-        hh = *reinterpret_cast<const uint2*>(p.h + (size_t)tt * H + i0 + i);
-      }
-      *reinterpret_cast<uint2*>(Gsm + r * LDI + i) = make_uint2(pack2(gg.x, gg.y), pack2(gg.z, gg.w));
-      *reinterpret_cast<uint2*>(Hsm + r * LDI + i) = hh;
+#pragma unroll
+    for (int q = 0; q < NG; ++q) {
+      const int e = threadIdx.x + q * 256, r = e / (DWC / 4), i = (e % (DWC / 4)) * 4;
+      *reinterpret_cast<uint2*>(Gsm + r * LDI + i) = make_uint2(pack2(gr[q].x, gr[q].y), pack2(gr[q].z, gr[q].w));
+      *reinterpret_cast<uint2*>(Hsm + r * LDI + i) = hr[q];
     }
     __syncthreads();
+    if (r0 + DWR < te) fetch(r0 + DWR);  // next tile's loads overlap this tile's products
 #pragma unroll
     for (int ks = 0; ks < DWR / 16; ++ks) {
       const int k0 = ks * 16;
@@ -484,22 +483,15 @@ __global__ void __launch_bounds__(256) adapter_dw_mma_kernel(DwArgs p) {
     }
 }
 
-int pick_rows(int T, int H, int m) {
-  // 32-row tiles when there are enough of them to fill the GPU twice, else 16
-  if (m > 64 || H > 1024) return 16;
-  return (T + 31) / 32 >= 2 * device_sm_count() ? 32 : 16;
+size_t rows_smem(int H, int m) {
+  const int W = H / COLS_PER_WARP, W1 = H / phase1_slice(H, m);
+  return (size_t)R * (H + 8) * 2 + (size_t)W1 * R * m * 4 + (size_t)R * (m + 8) * 2 + (W * 16 + 16) * 4;
 }
 
-template <int R, int MB>
-size_t fwd_smem(int H) {
-  const int W = H / COLS_PER_WARP;
-  return (size_t)R * (H + 8) * 2 + (size_t)W * R * MB * 4 + (size_t)R * (MB + 8) * 2 + (W * 16 + 16) * 4;
-}
-
-template <int R, int MB, bool DEC>
+template <int MB, bool DEC>
 cudaError_t launch_fwd(const FwdArgs& p, cudaStream_t st) {
-  const size_t smem = fwd_smem<R, MB>(p.H);
-  auto k = p.H > 1024 ? adapter_fwd_mma_kernel<R, MB, DEC, true> : adapter_fwd_mma_kernel<R, MB, DEC, false>;
+  const size_t smem = rows_smem(p.H, MB);
+  auto k = p.H > 1024 ? adapter_fwd_mma_kernel<MB, DEC, true> : adapter_fwd_mma_kernel<MB, DEC, false>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k<<<(p.T + R - 1) / R, (p.H / COLS_PER_WARP) * 32, smem, st>>>(p);
@@ -507,10 +499,10 @@ cudaError_t launch_fwd(const FwdArgs& p, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-template <int R, int MB>
+template <int MB>
 cudaError_t launch_bwd(const BwdArgs& p, cudaStream_t st) {
-  const size_t smem = fwd_smem<R, MB>(p.H);
-  auto k = p.H > 1024 ? adapter_bwd_rows_mma_kernel<R, MB, true> : adapter_bwd_rows_mma_kernel<R, MB, false>;
+  const size_t smem = rows_smem(p.H, MB);
+  auto k = p.H > 1024 ? adapter_bwd_rows_mma_kernel<MB, true> : adapter_bwd_rows_mma_kernel<MB, false>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k<<<(p.T + R - 1) / R, (p.H / COLS_PER_WARP) * 32, smem, st>>>(p);
@@ -521,7 +513,8 @@ cudaError_t launch_bwd(const BwdArgs& p, cudaStream_t st) {
 }  // namespace
 
 bool adapter_mma_ok(int H, int m) {
-  return H % COLS_PER_WARP == 0 && H <= 2048 && (m == 32 || m == 64 || m == 128);
+  return H % 128 == 0 && H <= 2048 && (m == 32 || m == 64 || m == 128) &&
+         rows_smem(H, m) <= 220 * 1024;
 }
 
 cudaError_t adapter_fwd_mma(const AdapterFwdArgs& a, const void* WdT_b, const void* WuT_b,
@@ -535,12 +528,11 @@ cudaError_t adapter_fwd_mma(const AdapterFwdArgs& a, const void* WdT_b, const vo
   p.z = a.z; p.resid = a.resid; p.gamma = a.gamma; p.beta = a.beta; p.eps = a.eps;
   p.y = reinterpret_cast<bf16*>(a.y); p.x_out = a.x_out;
   p.xhat = reinterpret_cast<bf16*>(a.xhat); p.rstd = a.rstd;
-  const int R = pick_rows(a.T, a.H, a.m);
-#define RA_FWD(RR, MM)                                                           \
-  if (R == RR && a.m == MM)                                                     \
-    return a.decoder ? launch_fwd<RR, MM, true>(p, st) : launch_fwd<RR, MM, false>(p, st);
-  RA_FWD(32, 32) RA_FWD(32, 64) RA_FWD(16, 32) RA_FWD(16, 64) RA_FWD(16, 128)
-#undef RA_FWD
+  switch (a.m) {
+    case 32: return a.decoder ? launch_fwd<32, true>(p, st) : launch_fwd<32, false>(p, st);
+    case 64: return a.decoder ? launch_fwd<64, true>(p, st) : launch_fwd<64, false>(p, st);
+    case 128: return a.decoder ? launch_fwd<128, true>(p, st) : launch_fwd<128, false>(p, st);
+  }
   return cudaErrorNotSupported;
 }
 
@@ -553,13 +545,10 @@ cudaError_t adapter_bwd_mma(const AdapterBwdArgs& a, const void* Wu_b, const voi
   p.Wu = reinterpret_cast<const bf16*>(Wu_b);
   p.Wd = reinterpret_cast<const bf16*>(Wd_b);
   p.dz = a.dz; p.dh = reinterpret_cast<bf16*>(a.dh);
-  const int R = pick_rows(a.T, a.H, a.m);
   cudaError_t e = cudaErrorNotSupported;
-  if (R == 32 && a.m == 32) e = launch_bwd<32, 32>(p, st);
-  else if (R == 32 && a.m == 64) e = launch_bwd<32, 64>(p, st);
-  else if (R == 16 && a.m == 32) e = launch_bwd<16, 32>(p, st);
-  else if (R == 16 && a.m == 64) e = launch_bwd<16, 64>(p, st);
-  else if (R == 16 && a.m == 128) e = launch_bwd<16, 128>(p, st);
+  if (a.m == 32) e = launch_bwd<32>(p, st);
+  else if (a.m == 64) e = launch_bwd<64>(p, st);
+  else if (a.m == 128) e = launch_bwd<128>(p, st);
   if (e != cudaSuccess) return e;
   // weight-gradient partials on the tensor cores, then the fixed-order sum
   DwArgs d;

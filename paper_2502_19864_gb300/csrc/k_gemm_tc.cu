@@ -6,14 +6,16 @@
 // backward (fused GELU' / SwiGLU' / residual epilogues) -- the dense contractions of the
 // step.
 //
-// Structure (one persistent CTA per SM, 192 threads):
+// Structure (one persistent CTA per SM, 320 threads):
 //   warp 0      TMA producer: 128 x 64 A tiles and BN x 64 B tiles (128-byte swizzle) into
 //               a STAGES-deep shared-memory ring, completion tracked by mbarrier tx counts;
 //   warp 1      allocates 2*BN TMEM columns (two accumulators); one thread issues
 //               tcgen05.mma (M = 128, N = BN, K = 16) and tcgen05.commit to free each stage
 //               and to publish each finished accumulator;
-//   warps 2..5  epilogue: tcgen05.ld of their 32 TMEM lanes, fused math, vector stores;
-//               the second accumulator lets the next tile's main loop overlap this.
+//   warps 2..9  epilogue: two warps per TMEM lane quadrant (warp w may only read lanes
+//               32 * (w % 4) .. + 31), each taking half of the tile's columns: tcgen05.ld,
+//               fused math, vector stores; the second accumulator lets the next tile's
+//               main loop overlap this.
 // Every mbarrier wait is bounded (global timer); on expiry the kernel records
 // RA_DEVERR_TIMEOUT, drains its own copies and MMAs, frees TMEM and returns.
 #include <cuda.h>
@@ -28,7 +30,7 @@
 namespace ra {
 namespace {
 
-constexpr int BM = 128, BK = 64, NTHREADS = 192;
+constexpr int BM = 128, BK = 64, NTHREADS = 320, EPI_WARPS = 8;
 
 template <int BN>
 struct TileCfg {
@@ -276,7 +278,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull_bar[a], 1);
-      mbar_init(&tempty_bar[a], 4);
+      mbar_init(&tempty_bar[a], EPI_WARPS);
     }
     mbar_init(&drain_bar, 1);
     abort_sh = 0;
@@ -360,8 +362,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       mbar_wait(&drain_bar, 0, &no_abort, nullptr);
     }
   } else {
-    // ------------------------------------------------------------------ epilogue (warps 2..5)
-    const int quad = warp & 3;  // TMEM lanes 32*quad .. 32*quad + 31
+    // ------------------------------------------------------------------ epilogue (warps 2..9)
+    const int quad = warp & 3;             // TMEM lanes 32*quad .. 32*quad + 31
+    const int half = (warp - 2) >> 2;      // which half of the tile's columns
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x) {
@@ -371,11 +374,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const int row = m0 + quad * 32 + lane;
       const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
       if (EPI == EPI_SWIGLU) {
-        // per 128-column block: gate columns [0, 64), up columns [64, 128)
+        // per 128-column block: gate columns [0, 64), up columns [64, 128); the two warps of
+        // a quadrant split each block's 64 gate columns
 #pragma unroll 1
         for (int blk = 0; blk < BN; blk += 128) {
 #pragma unroll 1
-          for (int c0 = 0; c0 < 64; c0 += 32) {
+          for (int c0 = half * 32; c0 < half * 32 + 32; c0 += 32) {
             float g[32], u[32];
             tmem_ld32(tbase + blk + c0, g);
             tmem_ld32(tbase + blk + 64 + c0, u);
@@ -399,7 +403,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         }
       } else {
 #pragma unroll 1
-        for (int c0 = 0; c0 < BN; c0 += 32) {
+        for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
           float v[32];
           tmem_ld32(tbase + c0, v);
           if (row < p.M && n0 + c0 < p.N) epi_chunk<EPI>(p, row, n0 + c0, v);

@@ -1115,6 +1115,22 @@ ra_status ra_profile_read(ra_ctx* ctx, ra_profile* out) {
   return RA_OK;
 }
 
+ra_status ra_profile_records(ra_ctx* ctx, ra_profile_record* out, int32_t max, int32_t* n) {
+  if (!ctx || !n || (max > 0 && !out)) return RA_ERR_ARG;
+  int32_t i = 0;
+  for (const auto& r : ctx->recs) {
+    if (i < max) {
+      float ms = 0.f;
+      cudaError_t e = cudaEventElapsedTime(&ms, r.a, r.b);
+      if (e != cudaSuccess) return fail(ctx, RA_ERR_CUDA, "cudaEventElapsedTime: %s", cudaGetErrorString(e));
+      out[i] = ra_profile_record{r.cat, ms, r.flops, r.bytes};
+    }
+    ++i;
+  }
+  *n = i;
+  return RA_OK;
+}
+
 int64_t ra_kernel_launches(void) { return (int64_t)launches_so_far(); }
 
 // ---- stand-alone kernels -----------------------------------------------------------------

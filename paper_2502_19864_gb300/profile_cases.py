@@ -1,7 +1,8 @@
 """Small, self-contained launch cases for profiler captures (ncu) of single kernels.
 
-  python -m paper_2502_19864_gb300.profile_cases gemm M N K [--reps R]
-      R launches of the tensor-core GEMM C[M,N] = A[M,K] B[N,K]^T (bf16, via ra_gemm_bf16)
+  python -m paper_2502_19864_gb300.profile_cases gemm M N K [--reps R] [--gelu]
+      R launches of the tensor-core GEMM C[M,N] = A[M,K] B[N,K]^T (bf16, via ra_gemm_bf16);
+      --gelu adds the bias + GELU epilogue (writes C and GELU(C))
   python -m paper_2502_19864_gb300.profile_cases step CONFIG D [--reps R]
       R eager steps (forward, early-stopped backward, update) of a synthetic workload
 
@@ -16,15 +17,18 @@ import sys
 sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
 
 
-def gemm_case(M, N, K, reps):
+def gemm_case(M, N, K, reps, gelu=False):
     import torch
     from paper_2502_19864_gb300 import ringada as R
     g = torch.Generator().manual_seed(0)
     A = torch.randn(M, K, generator=g).to(torch.bfloat16).cuda()
     B = (torch.randn(N, K, generator=g) * 0.05).to(torch.bfloat16).cuda()
     C = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    bias = torch.randn(N, generator=g).float().cuda() if gelu else None
+    G = torch.empty(M, N, dtype=torch.bfloat16, device="cuda") if gelu else None
     for _ in range(reps):
-        R.ra_gemm_bf16(A.data_ptr(), B.data_ptr(), C.data_ptr(), M, N, K)
+        R.ra_gemm_bf16(A.data_ptr(), B.data_ptr(), C.data_ptr(), M, N, K,
+                       bias.data_ptr() if gelu else None, G.data_ptr() if gelu else None)
     torch.cuda.synchronize()
     print("gemm %dx%dx%d x%d done" % (M, N, K, reps))
 
@@ -60,12 +64,13 @@ def main():
     ap.add_argument("case", choices=["gemm", "step"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--gelu", action="store_true")
     a = ap.parse_args()
     import __graft_entry__
     __graft_entry__.build()
     if a.case == "gemm":
         M, N, K = (int(v) for v in a.args[:3])
-        gemm_case(M, N, K, a.reps)
+        gemm_case(M, N, K, a.reps, a.gelu)
     else:
         step_case(a.args[0], int(a.args[1]), a.reps)
 

@@ -76,6 +76,10 @@ class ra_profile(C.Structure):
                 ("calls", C.c_int32 * 8)]
 
 
+class ra_profile_record(C.Structure):
+    _fields_ = [("cat", C.c_int32), ("ms", C.c_float), ("flops", C.c_double), ("bytes", C.c_double)]
+
+
 class RingAdaError(RuntimeError):
     def __init__(self, status, msg):
         super().__init__("%s: %s" % (STATUS_NAMES.get(status, status), msg))
@@ -120,6 +124,7 @@ _SIGS = {
     "ra_profile_enable": (C.c_int, [C.c_void_p, C.c_int32]),
     "ra_profile_read": (C.c_int, [C.c_void_p, C.c_void_p]),
     "ra_kernel_launches": (C.c_int64, []),
+    "ra_profile_records": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_int32)]),
 }
 
 
@@ -279,6 +284,14 @@ def ra_profile_read(ctx):
     _check(lib().ra_profile_read(ctx, C.byref(p)), ctx)
     return {cat: dict(ms=p.ms[i], flops=p.flops[i], bytes=p.bytes[i], calls=p.calls[i])
             for i, cat in enumerate(PROF_CATS)}
+
+
+def ra_profile_records(ctx, max_records=4096):
+    """[(category, ms, flops, bytes)] of every recorded kernel call, in call order."""
+    arr = (ra_profile_record * max_records)()
+    n = C.c_int32()
+    _check(lib().ra_profile_records(ctx, arr, max_records, C.byref(n)), ctx)
+    return [(PROF_CATS[r.cat], r.ms, r.flops, r.bytes) for r in arr[:min(n.value, max_records)]]
 
 
 def ra_kernel_launches() -> int:
