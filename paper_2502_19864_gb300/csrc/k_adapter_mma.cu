@@ -46,6 +46,11 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t* r, const void* p) {
 __device__ __forceinline__ uint32_t ld_u32(const bf16* p) {
   return __ldg(reinterpret_cast<const unsigned int*>(p));
 }
+// B fragments of two k16 steps from a fragment-major weight row (see frag_pos): .x/.y are
+// b0/b1 of the first step, .z/.w of the second
+__device__ __forceinline__ uint4 ld_frag2(const bf16* row, int k0, int t) {
+  return __ldg(reinterpret_cast<const uint4*>(row + k0 + t * 8));
+}
 __device__ __forceinline__ uint32_t pack2(float a, float b) {
   __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<uint32_t*>(&h);
@@ -63,8 +68,9 @@ __device__ __forceinline__ void load_a(uint32_t* a, const bf16* s, int ld, int r
 }
 
 // Phase 1 shared by forward and backward: part[w] = X[16, kslice] * Bw^T over this warp's
-// slice [kbase, kbase + ks_len) of H, where Bw is [m, H] row-major bf16 in global memory (B
-// fragments read directly; the matrix is small and stays in L1/L2).  The m output columns
+// slice [kbase, kbase + ks_len) of H, where Bw is [m, H] bf16 in fragment-major order (B
+// fragments read directly, 16 bytes per thread per two k16 steps; the matrix is small and
+// stays in L1/L2).  The m output columns
 // are produced in groups of 8 n-tiles to bound the registers.
 template <int MB>
 __device__ __forceinline__ void phase1_store(const bf16* Xs, int ldx, const bf16* Bw, int H,
@@ -76,14 +82,16 @@ __device__ __forceinline__ void phase1_store(const bf16* Xs, int ldx, const bf16
     float acc[NTG][4];
 #pragma unroll
     for (int nt = 0; nt < NTG; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
-#pragma unroll 2
-    for (int k0 = kbase; k0 < kbase + ks_len; k0 += 16) {
-      uint32_t a[4];
-      load_a(a, Xs, ldx, 0, k0, lane);
+#pragma unroll 1
+    for (int k0 = kbase; k0 < kbase + ks_len; k0 += 32) {
+      uint32_t a0[4], a1[4];
+      load_a(a0, Xs, ldx, 0, k0, lane);
+      load_a(a1, Xs, ldx, 0, k0 + 16, lane);
 #pragma unroll
       for (int nt = 0; nt < NTG; ++nt) {
-        const bf16* bp = Bw + (size_t)(ng * 64 + nt * 8 + g) * H + k0 + 2 * t;
-        mma_bf16(acc[nt], a, ld_u32(bp), ld_u32(bp + 8));
+        const uint4 b = ld_frag2(Bw + (size_t)(ng * 64 + nt * 8 + g) * H, k0, t);
+        mma_bf16(acc[nt], a0, b.x, b.y);
+        mma_bf16(acc[nt], a1, b.z, b.w);
       }
     }
 #pragma unroll
@@ -101,8 +109,8 @@ __host__ __device__ inline int phase1_slice(int H, int m) {
   return (H / 64) * R * m * 4 > 65536 ? 128 : 64;
 }
 
-// Phase 2: acc[16 rows, this warp's 64 columns] = S[16, m] * Bn^T where Bn is [H, m]
-// row-major bf16 (n = output column, k = bottleneck index).
+// Phase 2: acc[16 rows, this warp's 64 columns] = S[16, m] * Bn^T where Bn is [H, m] bf16
+// in fragment-major order (n = output column, k = bottleneck index).
 template <int MB>
 __device__ __forceinline__ void phase2(float (&acc)[8][4], const bf16* Ss, int lds,
                                        const bf16* Bn, int m, int nbase, int lane) {
@@ -110,13 +118,15 @@ __device__ __forceinline__ void phase2(float (&acc)[8][4], const bf16* Ss, int l
 #pragma unroll
   for (int nt = 0; nt < 8; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
 #pragma unroll
-  for (int ks = 0; ks < MB / 16; ++ks) {
-    uint32_t a[4];
-    load_a(a, Ss, lds, 0, ks * 16, lane);
+  for (int k0 = 0; k0 < MB; k0 += 32) {
+    uint32_t a0[4], a1[4];
+    load_a(a0, Ss, lds, 0, k0, lane);
+    load_a(a1, Ss, lds, 0, k0 + 16, lane);
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
-      const bf16* bp = Bn + (size_t)(nbase + nt * 8 + g) * m + ks * 16 + 2 * t;
-      mma_bf16(acc[nt], a, ld_u32(bp), ld_u32(bp + 8));
+      const uint4 b = ld_frag2(Bn + (size_t)(nbase + nt * 8 + g) * m, k0, t);
+      mma_bf16(acc[nt], a0, b.x, b.y);
+      mma_bf16(acc[nt], a1, b.z, b.w);
     }
   }
 }

@@ -44,7 +44,7 @@ struct TileCfg {
 
 struct TcParams {
   int M, N, K;
-  int n_tiles_n, num_tiles, k_blocks;
+  int n_tiles_n, m_tiles, num_tiles, k_blocks;
   int epi;
   void* C; int ldc; int c_dtype;
   const float* bias;
@@ -125,6 +125,33 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
           smem_u32(bar))
       : "memory");
 }
+// 32 lanes x 32 consecutive fp32 columns, issue only; tmem_wait32 completes it.  The wait
+// takes the destination registers as in/out operands so no use can be scheduled above it.
+__device__ __forceinline__ void tmem_ld32_issue(uint32_t taddr, uint32_t* r) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait32(uint32_t* r) {
+  asm volatile(
+      "tcgen05.wait::ld.sync.aligned;"
+      : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+        "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]),
+        "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]),
+        "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]),
+        "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]),
+        "+r"(r[31])
+      :
+      : "memory");
+}
 // 32 lanes x 32 consecutive fp32 columns: thread i gets lane (base + i), columns c..c+31
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   uint32_t r[32];
@@ -201,47 +228,75 @@ __device__ __forceinline__ void load8(const void* base, int dt, int64_t off, flo
   }
 }
 
+// Operands of one row's 32-column chunk [n, n + 32) that do not come from TMEM (bias,
+// saved pre-activations, residual), fetched before the TMEM load completes.
+template <int EPI>
+struct EpiIn {
+  float bias[EPI == EPI_STORE || EPI == EPI_BIAS_GELU ? 32 : 1];
+  float aux[EPI == EPI_DGELU || EPI == EPI_RESID ? 32 : (EPI == EPI_DSWIGLU ? 64 : 1)];
+};
+
+template <int EPI>
+__device__ __forceinline__ void epi_fetch(const TcParams& p, int row, int n, EpiIn<EPI>& in) {
+#pragma unroll
+  for (int g = 0; g < 4; ++g) {
+    const int c = n + 8 * g;
+    if (c >= p.N) break;
+    if (EPI == EPI_STORE || EPI == EPI_BIAS_GELU) {
+      if (p.bias) {
+        const float4 b0 = *reinterpret_cast<const float4*>(p.bias + c);
+        const float4 b1 = *reinterpret_cast<const float4*>(p.bias + c + 4);
+        float* b = in.bias + 8 * g;
+        b[0] = b0.x; b[1] = b0.y; b[2] = b0.z; b[3] = b0.w;
+        b[4] = b1.x; b[5] = b1.y; b[6] = b1.z; b[7] = b1.w;
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) in.bias[8 * g + i] = 0.f;
+      }
+    } else if (EPI == EPI_DGELU || EPI == EPI_RESID) {
+      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + c, in.aux + 8 * g);
+    } else if (EPI == EPI_DSWIGLU) {
+      const int64_t gc = (int64_t)(c >> 6) * 128 + (c & 63);
+      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + gc, in.aux + 8 * g);
+      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + gc + 64, in.aux + 32 + 8 * g);
+    }
+  }
+}
+
 // One row's 32 accumulator columns [n, n + 32) of output C (non-SwiGLU epilogues).
 template <int EPI>
-__device__ __forceinline__ void epi_chunk(const TcParams& p, int row, int n, float* v) {
+__device__ __forceinline__ void epi_chunk(const TcParams& p, int row, int n, float* v,
+                                          const EpiIn<EPI>& in) {
 #pragma unroll
   for (int g = 0; g < 4; ++g) {
     const int c = n + 8 * g;
     if (c >= p.N) break;
     float* x = v + 8 * g;
     if (EPI == EPI_STORE) {
-      if (p.bias) {
 #pragma unroll
-        for (int i = 0; i < 8; ++i) x[i] += p.bias[c + i];
-      }
+      for (int i = 0; i < 8; ++i) x[i] += in.bias[8 * g + i];
       store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
     } else if (EPI == EPI_BIAS_GELU) {
-      if (p.bias) {
 #pragma unroll
-        for (int i = 0; i < 8; ++i) x[i] += p.bias[c + i];
-      }
+      for (int i = 0; i < 8; ++i) x[i] += in.bias[8 * g + i];
       if (p.C) store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
 #pragma unroll
       for (int i = 0; i < 8; ++i) x[i] = gelu_f(x[i]);
       store8(p.C2, p.c2_dtype, (int64_t)row * p.ldc2 + c, x);
     } else if (EPI == EPI_DGELU) {
-      float u[8];
-      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + c, u);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) x[i] *= gelu_grad_f(u[i]);
+      for (int i = 0; i < 8; ++i) x[i] *= gelu_grad_f(in.aux[8 * g + i]);
       store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
     } else if (EPI == EPI_RESID) {
-      float r[8];
-      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + c, r);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) x[i] += r[i];
+      for (int i = 0; i < 8; ++i) x[i] += in.aux[8 * g + i];
       store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
     } else if (EPI == EPI_DSWIGLU) {
       // column c of d(h) -> packed gate column gc and up column gc + 64
       const int64_t gc = (int64_t)(c >> 6) * 128 + (c & 63);
-      float gt[8], up[8], dg[8], du[8];
-      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + gc, gt);
-      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + gc + 64, up);
+      const float* gt = in.aux + 8 * g;
+      const float* up = in.aux + 32 + 8 * g;
+      float dg[8], du[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         dg[i] = x[i] * up[i] * silu_grad_f(gt[i]);
@@ -251,6 +306,17 @@ __device__ __forceinline__ void epi_chunk(const TcParams& p, int row, int n, flo
       store8(p.C, p.c_dtype, (int64_t)row * p.ldc + gc + 64, du);
     }
   }
+}
+
+// Tile order: groups of 8 M-tiles swept across N, so that CTAs running at the same time
+// share A rows and B columns in L2.
+__device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mt, int& nt) {
+  constexpr int GM = 8;
+  const int per_group = GM * n_tiles;
+  const int grp = tile / per_group, in = tile % per_group;
+  const int gsz = min(GM, m_tiles - grp * GM);
+  mt = grp * GM + in % gsz;
+  nt = in / gsz;
 }
 
 // ---- the kernel -------------------------------------------------------------------------------
@@ -310,7 +376,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       for (int s = 0; s < STAGES; ++s) pending_phase[s] = -1;
       bool ok = true;
       for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
-        const int m0 = (tile / p.n_tiles_n) * BM, n0 = (tile % p.n_tiles_n) * BN;
+        int mt, nt;
+        tile_coords(tile, p.m_tiles, p.n_tiles_n, mt, nt);
+        const int m0 = mt * BM, n0 = nt * BN;
         for (int kb = 0; kb < p.k_blocks; ++kb) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, &abort_sh, p.err)) { ok = false; break; }
           mbar_expect_tx(&full_bar[stage], Cfg::STAGE_BYTES);
@@ -368,7 +436,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x) {
-      const int m0 = (tile / p.n_tiles_n) * BM, n0 = (tile % p.n_tiles_n) * BN;
+      int mt, nt;
+      tile_coords(tile, p.m_tiles, p.n_tiles_n, mt, nt);
+      const int m0 = mt * BM, n0 = nt * BN;
       if (!mbar_wait(&tfull_bar[acc], acc_phase, &abort_sh, p.err)) break;
       tc_fence_after();
       const int row = m0 + quad * 32 + lane;
@@ -404,9 +474,14 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       } else {
 #pragma unroll 1
         for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
-          float v[32];
-          tmem_ld32(tbase + c0, v);
-          if (row < p.M && n0 + c0 < p.N) epi_chunk<EPI>(p, row, n0 + c0, v);
+          uint32_t r[32];
+          tmem_ld32_issue(tbase + c0, r);
+          const bool live = row < p.M && n0 + c0 < p.N;
+          EpiIn<EPI> in;
+          if (live) epi_fetch<EPI>(p, row, n0 + c0, in);
+          tmem_wait32(r);
+          float* v = reinterpret_cast<float*>(r);
+          if (live) epi_chunk<EPI>(p, row, n0 + c0, v, in);
         }
       }
       tc_fence_before();
@@ -566,6 +641,7 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   TcParams p;
   p.M = g.M; p.N = g.N; p.K = g.K;
   p.n_tiles_n = (g.N + BNsel - 1) / BNsel;
+  p.m_tiles = m_tiles;
   p.num_tiles = m_tiles * p.n_tiles_n;
   p.k_blocks = (g.K + BK - 1) / BK;
   p.epi = g.epi;

@@ -560,6 +560,14 @@ __global__ void pack_rows_kernel(const float* src, void* dst, int R, int C, int 
 // transposed copies of the adapter matrices of layers [l0, l1): for each layer the four
 // matrices WdA [H,m], WuA [m,H], WdF [H,m], WuF [m,H] (contiguous, 4Hm per layer) go to
 // WdT [m,H], WuT [H,m], ... at the same offsets of PT.
+// Position of element k of a row inside the fragment-major order of the bf16 adapter shadows:
+// within each 32-wide block, the values k = 8q + 2t + b (q, b in {0..3}, {0, 1}) that thread
+// t of an mma.sync needs for two k16 steps are stored together at 8t + 2q + b.
+__device__ __forceinline__ int frag_pos(int k) {
+  const int w = k & 31;
+  return (k & ~31) + ((w & 7) >> 1) * 8 + (w >> 3) * 2 + (w & 1);
+}
+
 __global__ void adapter_transpose_kernel(const float* P, float* PT, bf16* PB, bf16* PTB, int H, int m) {
   int layer = blockIdx.z >> 2, mat = blockIdx.z & 3;
   int64_t base = (int64_t)layer * 4 * H * m + (int64_t)mat * H * m;
@@ -569,8 +577,8 @@ __global__ void adapter_transpose_kernel(const float* P, float* PT, bf16* PB, bf
   int r = (int)(e / cols), c = (int)(e % cols);
   const float v = P[base + e];
   PT[base + (int64_t)c * rows + r] = v;
-  if (PB) PB[base + e] = __float2bfloat16_rn(v);
-  if (PTB) PTB[base + (int64_t)c * rows + r] = __float2bfloat16_rn(v);
+  if (PB) PB[base + (int64_t)r * cols + frag_pos(c)] = __float2bfloat16_rn(v);
+  if (PTB) PTB[base + (int64_t)c * rows + frag_pos(r)] = __float2bfloat16_rn(v);
 }
 
 __global__ void fill_kernel(float* dst, float v, int64_t n) {
