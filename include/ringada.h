@@ -191,6 +191,13 @@ ra_status ra_get_stats(const ra_ctx* ctx, ra_stats* out);
  * call (RA_ERR_TIMEOUT), or a CUDA error occurred (RA_ERR_CUDA).  Clears the flag. */
 ra_status ra_sync_status(ra_ctx* ctx, ra_stream_t stream);
 
+/* Failure-detection hook: enqueues one kernel whose single thread waits, bounded by
+ * limit_us microseconds (1 .. 1000000), on a device barrier that nothing ever signals --
+ * the same bounded wait every pipelined kernel of the step uses.  The wait expires, the
+ * kernel records the timeout and returns; the next ra_sync_status on the stream reports
+ * RA_ERR_TIMEOUT and clears it.  Nothing faults or hangs, and the context stays usable. */
+ra_status ra_selftest_wait_timeout(ra_ctx* ctx, int32_t limit_us, ra_stream_t stream);
+
 /* Message of the last failing call on ctx (never null; "" if none). */
 const char* ra_last_error(const ra_ctx* ctx);
 

@@ -81,7 +81,7 @@ __device__ __forceinline__ bool mbar_try(uint32_t addr, uint32_t parity) {
 // Bounded wait for the phase of `parity` to complete.  Returns false if the CTA was told to
 // abort or the global-timer limit passed (then the error word gets RA_DEVERR_TIMEOUT).
 __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                       unsigned* err) {
+                                       unsigned* err, uint64_t limit_ns = kWaitLimitNs) {
   const uint32_t addr = smem_u32(bar);
   if (mbar_try(addr, parity)) return true;
   const uint64_t t0 = global_ns();
@@ -89,7 +89,7 @@ __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile 
     if (mbar_try(addr, parity)) return true;
     if ((it & 63) == 0) {
       if (*abort_flag) return false;
-      if (global_ns() - t0 > kWaitLimitNs) {
+      if (global_ns() - t0 > limit_ns) {
         *abort_flag = 1;
         set_dev_error(err, RA_DEVERR_TIMEOUT);
         return false;
@@ -501,6 +501,21 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   }
 }
 
+// Failure-detection self-test: one thread waits, with the same bounded wait as the GEMM,
+// on an mbarrier that nothing ever arrives on; the wait expires after limit_ns, records
+// RA_DEVERR_TIMEOUT and the kernel returns normally.
+__global__ void selftest_wait_kernel(unsigned* err, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ volatile int abort_sh;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_sh = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_wait(&bar, 0, &abort_sh, err, limit_ns);
+}
+
 // ---- host side --------------------------------------------------------------------------------
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
@@ -597,6 +612,12 @@ cudaError_t dispatch(const CUtensorMap& a, const CUtensorMap& b, const TcParams&
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 }  // namespace
+
+cudaError_t selftest_wait(unsigned* err, uint64_t limit_ns, cudaStream_t st) {
+  selftest_wait_kernel<<<1, 32, 0, st>>>(err, limit_ns);
+  note_launch(1);
+  return cudaGetLastError();
+}
 
 bool tc_available() {
   static int v = -1;

@@ -48,6 +48,9 @@ cudaError_t gemm(const GemmArgs& a, cudaStream_t st);
 // tcgen05 path; returns cudaErrorNotSupported if the shape/dtype is not handled.
 cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st);
 cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st);
+// Bounded-wait self-test (failure detection): a wait that nothing satisfies runs out after
+// limit_ns and sets RA_DEVERR_TIMEOUT in *err.
+cudaError_t selftest_wait(unsigned* err, uint64_t limit_ns, cudaStream_t st);
 // Whether the tcgen05 path is usable on the current device (sm_103).
 bool tc_available();
 int device_sm_count();

@@ -1084,6 +1084,15 @@ ra_status ra_sync_status(ra_ctx* ctx, ra_stream_t stream) {
   return RA_OK;
 }
 
+ra_status ra_selftest_wait_timeout(ra_ctx* ctx, int32_t limit_us, ra_stream_t stream) {
+  if (!ctx) return RA_ERR_ARG;
+  if (!ctx->WS) return fail(ctx, RA_ERR_STATE, "ra_bind_memory first");
+  if (limit_us < 1 || limit_us > 1000000) return fail(ctx, RA_ERR_ARG, "limit_us outside 1..1000000");
+  CU(cudaSetDevice(ctx->device));
+  CU(selftest_wait(ctx->ws<unsigned>(ctx->ws_err), (uint64_t)limit_us * 1000ull, (cudaStream_t)stream));
+  return RA_OK;
+}
+
 const char* ra_last_error(const ra_ctx* ctx) { return ctx ? ctx->err.c_str() : "null context"; }
 
 void ra_destroy(ra_ctx* ctx) { delete ctx; }

@@ -110,6 +110,7 @@ _SIGS = {
     "ra_get_stats": (C.c_int, [C.c_void_p, C.POINTER(ra_stats)]),
     "ra_sync_status": (C.c_int, [C.c_void_p, C.c_void_p]),
     "ra_last_error": (C.c_char_p, [C.c_void_p]),
+    "ra_selftest_wait_timeout": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p]),
     "ra_destroy": (None, [C.c_void_p]),
     "ra_gemm_bf16": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32,
                                C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p]),
@@ -241,6 +242,10 @@ def ra_get_stats(ctx):
 
 def ra_sync_status(ctx, stream=None):
     _check(lib().ra_sync_status(ctx, _stream_ptr(stream)), ctx)
+
+
+def ra_selftest_wait_timeout(ctx, limit_us: int, stream=None):
+    _check(lib().ra_selftest_wait_timeout(ctx, limit_us, _stream_ptr(stream)), ctx)
 
 
 def ra_last_error(ctx) -> str:

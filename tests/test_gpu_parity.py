@@ -268,3 +268,24 @@ def test_schedule_first_five_steps_base():
             assert err < 1e-1, (key, err)
     finally:
         run.close()
+
+
+def test_bounded_wait_expiry_is_reported_and_the_context_survives():
+    """Failure detection without a GPU fault: a device wait that nothing satisfies runs out
+    after 20 ms, the kernel returns, ra_sync_status reports RA_ERR_TIMEOUT, and the next
+    step on the same context is correct."""
+    cfg = synth.CONFIGS["tiny"]
+    w = synth.make_workload(cfg, 0)
+    run = GpuRun(cfg, w)
+    try:
+        R.ra_selftest_wait_timeout(run.ctx, 20000)
+        with pytest.raises(R.RingAdaError) as e:
+            R.ra_sync_status(run.ctx)
+        assert e.value.status == R.RA_ERR_TIMEOUT
+        R.ra_sync_status(run.ctx)                   # the flag was cleared
+        layers, head = O.to_f64_params(w["layers"], w["head"])
+        ref = O.step(cfg, layers, head, w["x"], w["labels"], 1)
+        loss = run.step(1)
+        assert abs(loss - ref["loss"]) <= 1e-4 * abs(ref["loss"])
+    finally:
+        run.close()
