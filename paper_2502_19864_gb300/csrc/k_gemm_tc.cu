@@ -14,13 +14,16 @@
 //               and to publish each finished accumulator;
 //   warps 2..9  epilogue: two warps per TMEM lane quadrant (warp w may only read lanes
 //               32 * (w % 4) .. + 31), each taking half of the tile's columns: tcgen05.ld,
-//               fused math, vector stores; the second accumulator lets the next tile's
-//               main loop overlap this.
+//               fused math, then each 32 x 32 output chunk is staged in shared memory
+//               (TMA swizzle layout, conflict-free) and written by a TMA tensor store, which
+//               coalesces the rows and clips ragged edges; the second accumulator lets the
+//               next tile's main loop overlap this.
 // Every mbarrier wait is bounded (global timer); on expiry the kernel records
 // RA_DEVERR_TIMEOUT, drains its own copies and MMAs, frees TMEM and returns.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <cstring>
 #include <mutex>
 #include <unordered_map>
 
@@ -32,14 +35,31 @@ namespace {
 
 constexpr int BM = 128, BK = 64, NTHREADS = 320, EPI_WARPS = 8;
 
-template <int BN>
+// epilogue staging: 4 KB per warp, one 32 x 32 f32 chunk or two 32 x 32 bf16 chunks (then
+// a second store can be staged while the first is still being read); this keeps the full
+// operand ring (224 KB in all)
+constexpr int SLOT_BYTES = 4096, NSLOT = 1;
+
+// epilogues that read a saved operand per output element (GELU', residual, SwiGLU')
+template <int EPI>
+struct EpiTraits {
+  static constexpr bool AUX = EPI == EPI_DGELU || EPI == EPI_RESID || EPI == EPI_DSWIGLU;
+};
+
+// Every epilogue stages through 4 KB per warp, which keeps the full operand ring.  AUX
+// epilogues TMA-load their operand chunk into that area: bf16 GELU' operands use two 2 KB
+// regions (the next chunk loads while this one computes); 4 KB operands (fp32 residual,
+// packed gate|up) use one region, whose first chunk per tile loads during the main loop.
+template <int BN, bool AUX>
 struct TileCfg {
   static constexpr int STAGES = BN == 256 ? 4 : 6;
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024;  // + alignment slack
+  static constexpr int WARP_STAGING = NSLOT * SLOT_BYTES;
+  static constexpr int STAGING = EPI_WARPS * WARP_STAGING;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + STAGING + 1024;  // + alignment slack
 };
 
 struct TcParams {
@@ -105,6 +125,19 @@ __device__ __forceinline__ void tma_load_2d(const CUtensorMap* tm, uint32_t dst,
       "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
       : "memory");
 }
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, uint32_t src, int c0, int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(tm)),
+               "r"(c0), "r"(c1), "r"(src)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// at most N bulk stores of this thread may still be reading shared memory
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -195,21 +228,83 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<uint32_t*>(&h);
 }
-// store 8 consecutive values (16 bytes for bf16, 32 bytes for f32)
-__device__ __forceinline__ void store8(void* base, int dt, int64_t off, const float* v) {
+// Writes this thread's row (lane) of a 32 x 32 chunk into a staging slot in the TMA swizzle
+// layout the store map uses: bf16 rows are 64 B under the 64-byte swizzle (16-byte chunk q
+// of row r at q ^ ((r >> 1) & 3)), f32 rows 128 B under the 128-byte swizzle (q ^ (r & 7)).
+// Lanes 0..7 then hit eight different bank groups for every q: no bank conflicts.
+__device__ __forceinline__ void stage_row(uint8_t* slot, int dt, int lane, const float* x) {
   if (dt == DT_BF16) {
-    uint4 q;
-    q.x = pack_bf16x2(v[0], v[1]);
-    q.y = pack_bf16x2(v[2], v[3]);
-    q.z = pack_bf16x2(v[4], v[5]);
-    q.w = pack_bf16x2(v[6], v[7]);
-    *reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(base) + off) = q;
+    uint8_t* row = slot + lane * 64;
+    const int sw = (lane >> 1) & 3;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint4 v;
+      v.x = pack_bf16x2(x[8 * q + 0], x[8 * q + 1]);
+      v.y = pack_bf16x2(x[8 * q + 2], x[8 * q + 3]);
+      v.z = pack_bf16x2(x[8 * q + 4], x[8 * q + 5]);
+      v.w = pack_bf16x2(x[8 * q + 6], x[8 * q + 7]);
+      *reinterpret_cast<uint4*>(row + ((q ^ sw) << 4)) = v;
+    }
   } else {
-    float4* p = reinterpret_cast<float4*>(reinterpret_cast<float*>(base) + off);
-    p[0] = make_float4(v[0], v[1], v[2], v[3]);
-    p[1] = make_float4(v[4], v[5], v[6], v[7]);
+    uint8_t* row = slot + lane * 128;
+    const int sw = lane & 7;
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      *reinterpret_cast<float4*>(row + ((q ^ sw) << 4)) =
+          make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3]);
   }
 }
+
+// Reads this thread's row (lane) of a 32 x 32 chunk from the TMA swizzle layout (inverse of
+// stage_row).
+__device__ __forceinline__ void unstage_row(const uint8_t* slot, int dt, int lane, float* x) {
+  if (dt == DT_BF16) {
+    const uint8_t* row = slot + lane * 64;
+    const int sw = (lane >> 1) & 3;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint4 v = *reinterpret_cast<const uint4*>(row + ((q ^ sw) << 4));
+      const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(h[i]);
+        x[8 * q + 2 * i] = f.x;
+        x[8 * q + 2 * i + 1] = f.y;
+      }
+    }
+  } else {
+    const uint8_t* row = slot + lane * 128;
+    const int sw = lane & 7;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float4 v = *reinterpret_cast<const float4*>(row + ((q ^ sw) << 4));
+      x[4 * q] = v.x; x[4 * q + 1] = v.y; x[4 * q + 2] = v.z; x[4 * q + 3] = v.w;
+    }
+  }
+}
+
+// Stores one 32-row x 32-column chunk (rows row0.., columns col..) of this warp through the
+// staging area and a TMA tensor store.  `slot_i` counts the warp's stores; two_slots: every
+// output of the kernel is bf16, so the area holds two chunks.
+__device__ __forceinline__ void store_chunk(const CUtensorMap* tm, uint8_t* staging, int& slot_i,
+                                           int dt, int lane, const float* x, int col, int row0,
+                                           bool two_slots) {
+  uint8_t* slot = staging + (two_slots ? (slot_i & 1) * (SLOT_BYTES / 2) : 0);
+  if (lane == 0) {  // the store that last used this slot has read it
+    if (two_slots) bulk_wait_read<1>();
+    else bulk_wait_read<0>();
+  }
+  __syncwarp();
+  stage_row(slot, dt, lane, x);
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  __syncwarp();
+  if (lane == 0) {
+    tma_store_2d(tm, (uint32_t)__cvta_generic_to_shared(slot), col, row0);
+    bulk_commit();
+  }
+  ++slot_i;
+}
+
 __device__ __forceinline__ void load8(const void* base, int dt, int64_t off, float* v) {
   if (dt == DT_BF16) {
     uint4 q = *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(base) + off);
@@ -263,48 +358,44 @@ __device__ __forceinline__ void epi_fetch(const TcParams& p, int row, int n, Epi
   }
 }
 
-// One row's 32 accumulator columns [n, n + 32) of output C (non-SwiGLU epilogues).
+// One warp's 32 x 32 chunk of output C (non-SwiGLU epilogues): rows row0.., columns n..
+// (this thread holds row row0 + lane in v).
 template <int EPI>
-__device__ __forceinline__ void epi_chunk(const TcParams& p, int row, int n, float* v,
-                                          const EpiIn<EPI>& in) {
+__device__ __forceinline__ void epi_chunk(const TcParams& p, const CUtensorMap* tmC,
+                                          const CUtensorMap* tmC2, uint8_t* staging, int& slot_i,
+                                          int lane, int row0, int n, float* v, const EpiIn<EPI>& in,
+                                          bool ts) {
+  if (EPI == EPI_STORE) {
 #pragma unroll
-  for (int g = 0; g < 4; ++g) {
-    const int c = n + 8 * g;
-    if (c >= p.N) break;
-    float* x = v + 8 * g;
-    if (EPI == EPI_STORE) {
+    for (int i = 0; i < 32; ++i) v[i] += in.bias[i];
+    store_chunk(tmC, staging, slot_i, p.c_dtype, lane, v, n, row0, ts);
+  } else if (EPI == EPI_BIAS_GELU) {
 #pragma unroll
-      for (int i = 0; i < 8; ++i) x[i] += in.bias[8 * g + i];
-      store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
-    } else if (EPI == EPI_BIAS_GELU) {
+    for (int i = 0; i < 32; ++i) v[i] += in.bias[i];
+    if (p.C) store_chunk(tmC, staging, slot_i, p.c_dtype, lane, v, n, row0, ts);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) x[i] += in.bias[8 * g + i];
-      if (p.C) store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
+    for (int i = 0; i < 32; ++i) v[i] = gelu_f(v[i]);
+    store_chunk(tmC2, staging, slot_i, p.c2_dtype, lane, v, n, row0, ts);
+  } else if (EPI == EPI_DGELU) {
 #pragma unroll
-      for (int i = 0; i < 8; ++i) x[i] = gelu_f(x[i]);
-      store8(p.C2, p.c2_dtype, (int64_t)row * p.ldc2 + c, x);
-    } else if (EPI == EPI_DGELU) {
+    for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(in.aux[i]);
+    store_chunk(tmC, staging, slot_i, p.c_dtype, lane, v, n, row0, ts);
+  } else if (EPI == EPI_RESID) {
 #pragma unroll
-      for (int i = 0; i < 8; ++i) x[i] *= gelu_grad_f(in.aux[8 * g + i]);
-      store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
-    } else if (EPI == EPI_RESID) {
+    for (int i = 0; i < 32; ++i) v[i] += in.aux[i];
+    store_chunk(tmC, staging, slot_i, p.c_dtype, lane, v, n, row0, ts);
+  } else if (EPI == EPI_DSWIGLU) {
+    // columns n.. of d(h) -> packed gate columns gc.. and up columns gc + 64..
+    const int gc = (n >> 6) * 128 + (n & 63);
+    float du[32];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) x[i] += in.aux[8 * g + i];
-      store8(p.C, p.c_dtype, (int64_t)row * p.ldc + c, x);
-    } else if (EPI == EPI_DSWIGLU) {
-      // column c of d(h) -> packed gate column gc and up column gc + 64
-      const int64_t gc = (int64_t)(c >> 6) * 128 + (c & 63);
-      const float* gt = in.aux + 8 * g;
-      const float* up = in.aux + 32 + 8 * g;
-      float dg[8], du[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        dg[i] = x[i] * up[i] * silu_grad_f(gt[i]);
-        du[i] = x[i] * silu_f(gt[i]);
-      }
-      store8(p.C, p.c_dtype, (int64_t)row * p.ldc + gc, dg);
-      store8(p.C, p.c_dtype, (int64_t)row * p.ldc + gc + 64, du);
+    for (int i = 0; i < 32; ++i) {
+      const float gt = in.aux[i], up = in.aux[32 + i];
+      du[i] = v[i] * silu_f(gt);
+      v[i] = v[i] * up * silu_grad_f(gt);
     }
+    store_chunk(tmC, staging, slot_i, p.c_dtype, lane, v, gc, row0, ts);
+    store_chunk(tmC, staging, slot_i, p.c_dtype, lane, du, gc + 64, row0, ts);
   }
 }
 
@@ -323,12 +414,14 @@ __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, 
 template <int BN, int EPI>
 __global__ void __launch_bounds__(NTHREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const TcParams p) {
-  using Cfg = TileCfg<BN>;
+                   const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmC2,
+                   const __grid_constant__ CUtensorMap tmX, const TcParams p) {
+  using Cfg = TileCfg<BN, EpiTraits<EPI>::AUX>;
   constexpr int STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES];
   __shared__ __align__(8) uint64_t tfull_bar[2], tempty_bar[2], drain_bar;
+  __shared__ __align__(8) uint64_t aux_bar[EPI_WARPS][2];  // TMA loads of AUX operands
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_sh;
 
@@ -347,6 +440,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       mbar_init(&tempty_bar[a], EPI_WARPS);
     }
     mbar_init(&drain_bar, 1);
+    for (int w = 0; w < EPI_WARPS; ++w) {
+      mbar_init(&aux_bar[w][0], 1);
+      mbar_init(&aux_bar[w][1], 1);
+    }
     abort_sh = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -433,55 +530,126 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     // ------------------------------------------------------------------ epilogue (warps 2..9)
     const int quad = warp & 3;             // TMEM lanes 32*quad .. 32*quad + 31
     const int half = (warp - 2) >> 2;      // which half of the tile's columns
+    uint8_t* staging = smem + STAGES * Cfg::STAGE_BYTES + (warp - 2) * Cfg::WARP_STAGING;
+    const bool two_slots = (!p.C || p.c_dtype == DT_BF16) && (!p.C2 || p.c2_dtype == DT_BF16);
+    int slot_i = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x) {
+    int aux_i = 0;                         // AUX chunks issued by this warp (region = aux_i & 1)
+    uint32_t aux_phase[2] = {0u, 0u};
+    int aux_waited = 0;                    // AUX chunks whose load this warp has waited for
+    uint64_t* abar = aux_bar[warp - 2];
+    // AUX: TMA load of the operand chunk (rows row0.., output columns n..) into a region
+    const int rbytes = (EPI == EPI_DGELU && p.aux_dtype == DT_BF16) ? SLOT_BYTES / 2 : SLOT_BYTES;
+    const int nreg = SLOT_BYTES / rbytes;
+    auto aux_issue = [&](int row0_, int n_) {
+      const int reg = aux_i % nreg;
+      uint8_t* region = staging + reg * rbytes;
+      if (lane == 0) {
+        bulk_wait_read<0>();  // no tensor store still reads this region
+        uint64_t* bar = &abar[reg];
+        if (EPI == EPI_DSWIGLU) {
+          const int gc = (n_ >> 6) * 128 + (n_ & 63);
+          mbar_expect_tx(bar, 4096);
+          tma_load_2d(&tmX, smem_u32(region), bar, gc, row0_);
+          tma_load_2d(&tmX, smem_u32(region + 2048), bar, gc + 64, row0_);
+        } else {
+          mbar_expect_tx(bar, p.aux_dtype == DT_BF16 ? 2048 : 4096);
+          tma_load_2d(&tmX, smem_u32(region), bar, n_, row0_);
+        }
+      }
+      ++aux_i;
+    };
+    bool ok = true;
+    for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
       int mt, nt;
       tile_coords(tile, p.m_tiles, p.n_tiles_n, mt, nt);
       const int m0 = mt * BM, n0 = nt * BN;
+      const int row0 = m0 + quad * 32, row = row0 + lane;
+      const int cbeg = half * (BN / 2), cend = cbeg + BN / 2;
+      // the first operand chunk is fetched while the main loop of this tile still runs
+      if (EpiTraits<EPI>::AUX && n0 + cbeg < p.N && row0 < p.M) aux_issue(row0, n0 + cbeg);
       if (!mbar_wait(&tfull_bar[acc], acc_phase, &abort_sh, p.err)) break;
       tc_fence_after();
-      const int row = m0 + quad * 32 + lane;
       const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
       if (EPI == EPI_SWIGLU) {
         // per 128-column block: gate columns [0, 64), up columns [64, 128); the two warps of
         // a quadrant split each block's 64 gate columns
 #pragma unroll 1
         for (int blk = 0; blk < BN; blk += 128) {
-#pragma unroll 1
-          for (int c0 = half * 32; c0 < half * 32 + 32; c0 += 32) {
-            float g[32], u[32];
-            tmem_ld32(tbase + blk + c0, g);
-            tmem_ld32(tbase + blk + 64 + c0, u);
-            const int ng = n0 + blk + c0;           // packed gate column
-            if (row < p.M && ng < p.N) {
-              if (p.C) {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                  store8(p.C, p.c_dtype, (int64_t)row * p.ldc + ng + 8 * q, g + 8 * q);
-                  store8(p.C, p.c_dtype, (int64_t)row * p.ldc + ng + 64 + 8 * q, u + 8 * q);
-                }
-              }
-              const int hc = (n0 + blk) / 2 + c0;   // column of h = silu(gate) * up
-#pragma unroll
-              for (int i = 0; i < 32; ++i) g[i] = silu_f(g[i]) * u[i];
-#pragma unroll
-              for (int q = 0; q < 4; ++q)
-                store8(p.C2, p.c2_dtype, (int64_t)row * p.ldc2 + hc + 8 * q, g + 8 * q);
+          const int c0 = half * 32;
+          float g[32], u[32];
+          tmem_ld32(tbase + blk + c0, g);
+          tmem_ld32(tbase + blk + 64 + c0, u);
+          const int ng = n0 + blk + c0;           // packed gate column
+          if (ng < p.N && row0 < p.M) {
+            if (p.C) {
+              store_chunk(&tmC, staging, slot_i, p.c_dtype, lane, g, ng, row0, two_slots);
+              store_chunk(&tmC, staging, slot_i, p.c_dtype, lane, u, ng + 64, row0, two_slots);
             }
+#pragma unroll
+            for (int i = 0; i < 32; ++i) g[i] = silu_f(g[i]) * u[i];
+            store_chunk(&tmC2, staging, slot_i, p.c2_dtype, lane, g, (n0 + blk) / 2 + c0, row0, two_slots);
           }
+        }
+      } else if (EpiTraits<EPI>::AUX) {
+#pragma unroll 1
+        for (int c0 = cbeg; c0 < cend; c0 += 32) {
+          if (!(n0 + c0 < p.N && row0 < p.M)) break;  // live chunks form a prefix
+          uint32_t r[32];
+          tmem_ld32_issue(tbase + c0, r);
+          const int reg = (aux_i - 1) % nreg;        // region of this chunk's operand
+          uint8_t* region = staging + reg * rbytes;
+          if (!mbar_wait(&abar[reg], aux_phase[reg], &abort_sh, p.err)) { ok = false; tmem_wait32(r); break; }
+          aux_phase[reg] ^= 1u;
+          ++aux_waited;
+          float x1[32], x2[32];
+          if (EPI == EPI_DSWIGLU) {
+            unstage_row(region, DT_BF16, lane, x1);          // gate
+            unstage_row(region + 2048, DT_BF16, lane, x2);   // up
+          } else {
+            unstage_row(region, p.aux_dtype, lane, x1);
+          }
+          __syncwarp();  // every lane has its operand row before the region is reused
+          const bool more = c0 + 32 < cend && n0 + c0 + 32 < p.N;
+          if (more && nreg == 2) aux_issue(row0, n0 + c0 + 32);
+          tmem_wait32(r);
+          float* v = reinterpret_cast<float*>(r);
+          if (EPI == EPI_DGELU) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(x1[i]);
+            store_chunk(&tmC, region, slot_i, p.c_dtype, lane, v, n0 + c0, row0, false);
+          } else if (EPI == EPI_RESID) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] += x1[i];
+            store_chunk(&tmC, region, slot_i, p.c_dtype, lane, v, n0 + c0, row0, false);
+          } else {
+            // d(h) -> d(gate), d(up) in the packed layout
+            const int n = n0 + c0, gc = (n >> 6) * 128 + (n & 63);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float gt = x1[i], up = x2[i];
+              x2[i] = v[i] * silu_f(gt);                 // d(up)
+              v[i] = v[i] * up * silu_grad_f(gt);         // d(gate)
+            }
+            store_chunk(&tmC, region, slot_i, p.c_dtype, lane, v, gc, row0, false);
+            store_chunk(&tmC, region + 2048, slot_i, p.c_dtype, lane, x2, gc + 64, row0, false);
+          }
+          if (more && nreg == 1) aux_issue(row0, n0 + c0 + 32);  // after the store has read it
         }
       } else {
 #pragma unroll 1
-        for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
+        for (int c0 = cbeg; c0 < cend; c0 += 32) {
           uint32_t r[32];
           tmem_ld32_issue(tbase + c0, r);
-          const bool live = row < p.M && n0 + c0 < p.N;
+          // chunks entirely right of N or below M are skipped (warp-uniform); partial ones
+          // are clipped by the tensor store
+          const bool live_cols = n0 + c0 < p.N && row0 < p.M;
           EpiIn<EPI> in;
-          if (live) epi_fetch<EPI>(p, row, n0 + c0, in);
+          if (live_cols && row < p.M) epi_fetch<EPI>(p, row, n0 + c0, in);
           tmem_wait32(r);
           float* v = reinterpret_cast<float*>(r);
-          if (live) epi_chunk<EPI>(p, row, n0 + c0, v, in);
+          if (live_cols) epi_chunk<EPI>(p, &tmC, &tmC2, staging, slot_i, lane, row0, n0 + c0, v, in, two_slots);
         }
       }
       tc_fence_before();
@@ -489,6 +657,14 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       if (lane == 0) mbar_arrive(&tempty_bar[acc]);
       if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
     }
+    // an operand load issued but not consumed (only after an abort) lands before exit
+    for (; aux_waited < aux_i; ++aux_waited) {
+      const int reg = aux_waited % nreg;
+      volatile int no_abort = 0;
+      mbar_wait(&abar[reg], aux_phase[reg], &no_abort, nullptr);
+      aux_phase[reg] ^= 1u;
+    }
+    if (lane == 0) bulk_wait_all();  // this warp's tensor stores are complete
   }
 
   tc_fence_before();
@@ -540,25 +716,31 @@ EncodeTiledFn encode_fn() {
 struct MapKey {
   const void* ptr;
   int64_t rows, cols, ld;
-  int box_rows;
+  int box_cols, box_rows, dtype;
   bool operator==(const MapKey& o) const {
-    return ptr == o.ptr && rows == o.rows && cols == o.cols && ld == o.ld && box_rows == o.box_rows;
+    return ptr == o.ptr && rows == o.rows && cols == o.cols && ld == o.ld &&
+           box_cols == o.box_cols && box_rows == o.box_rows && dtype == o.dtype;
   }
 };
 struct MapKeyHash {
   size_t operator()(const MapKey& k) const {
     size_t h = std::hash<const void*>()(k.ptr);
     h ^= std::hash<int64_t>()(k.rows * 1000003 + k.cols) + 0x9e3779b9 + (h << 6) + (h >> 2);
-    h ^= std::hash<int64_t>()(k.ld * 31 + k.box_rows) + 0x9e3779b9 + (h << 6) + (h >> 2);
+    h ^= std::hash<int64_t>()(k.ld * 31 + k.box_rows * 7 + k.box_cols * 131 + k.dtype) + 0x9e3779b9 +
+         (h << 6) + (h >> 2);
     return h;
   }
 };
 
-// bf16 row-major [rows, cols] with leading dimension ld; box = 64 columns x box_rows rows
-bool make_map(CUtensorMap* out, const void* ptr, int64_t rows, int64_t cols, int64_t ld, int box_rows) {
+// Row-major [rows, cols] matrix with leading dimension ld (elements of dtype); box of
+// box_cols x box_rows.  Operand loads (box 64 bf16 columns) use the 128-byte swizzle the
+// MMA descriptors expect; output stores (box 32 columns) use the swizzle whose span is one
+// box row (64 B for bf16, 128 B for f32), matching stage_row.
+bool make_map(CUtensorMap* out, const void* ptr, int64_t rows, int64_t cols, int64_t ld,
+              int box_cols, int box_rows, int dtype) {
   static std::mutex mu;
   static std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
-  MapKey key{ptr, rows, cols, ld, box_rows};
+  MapKey key{ptr, rows, cols, ld, box_cols, box_rows, dtype};
   std::lock_guard<std::mutex> lock(mu);
   auto it = cache.find(key);
   if (it != cache.end()) {
@@ -567,13 +749,19 @@ bool make_map(CUtensorMap* out, const void* ptr, int64_t rows, int64_t cols, int
   }
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
+  const int es = dtype == DT_BF16 ? 2 : 4;
+  const int row_bytes = box_cols * es;
+  CUtensorMapSwizzle sw = row_bytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                        : row_bytes == 64  ? CU_TENSOR_MAP_SWIZZLE_64B
+                                           : CU_TENSOR_MAP_SWIZZLE_NONE;
   cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-  cuuint64_t gstride[1] = {(cuuint64_t)ld * 2};
-  cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+  cuuint64_t gstride[1] = {(cuuint64_t)ld * es};
+  cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
   cuuint32_t estride[2] = {1, 1};
-  CUresult r = fn(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), gdim, gstride,
-                  box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(out, dtype == DT_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+                  2, const_cast<void*>(ptr), gdim, gstride, box, estride,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return false;
   if (cache.size() > 4096) cache.clear();
   cache.emplace(key, *out);
@@ -581,30 +769,33 @@ bool make_map(CUtensorMap* out, const void* ptr, int64_t rows, int64_t cols, int
 }
 
 template <int BN, int EPI>
-cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int grid,
+cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
+                   const CUtensorMap& c2, const CUtensorMap& x, const TcParams& p, int grid,
                    cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, TileCfg<BN>::SMEM);
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         TileCfg<BN, EpiTraits<EPI>::AUX>::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  gemm_tc_kernel<BN, EPI><<<grid, NTHREADS, TileCfg<BN>::SMEM, st>>>(a, b, p);
+  gemm_tc_kernel<BN, EPI><<<grid, NTHREADS, TileCfg<BN, EpiTraits<EPI>::AUX>::SMEM, st>>>(a, b, c, c2, x, p);
   note_launch(1);
   return cudaGetLastError();
 }
 
 template <int BN>
-cudaError_t dispatch(const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int grid,
+cudaError_t dispatch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
+                     const CUtensorMap& c2, const CUtensorMap& x, const TcParams& p, int grid,
                      cudaStream_t st) {
   switch (p.epi) {
-    case EPI_STORE: return launch<BN, EPI_STORE>(a, b, p, grid, st);
-    case EPI_BIAS_GELU: return launch<BN, EPI_BIAS_GELU>(a, b, p, grid, st);
-    case EPI_DGELU: return launch<BN, EPI_DGELU>(a, b, p, grid, st);
-    case EPI_RESID: return launch<BN, EPI_RESID>(a, b, p, grid, st);
-    case EPI_SWIGLU: return launch<BN, EPI_SWIGLU>(a, b, p, grid, st);
-    case EPI_DSWIGLU: return launch<BN, EPI_DSWIGLU>(a, b, p, grid, st);
+    case EPI_STORE: return launch<BN, EPI_STORE>(a, b, c, c2, x, p, grid, st);
+    case EPI_BIAS_GELU: return launch<BN, EPI_BIAS_GELU>(a, b, c, c2, x, p, grid, st);
+    case EPI_DGELU: return launch<BN, EPI_DGELU>(a, b, c, c2, x, p, grid, st);
+    case EPI_RESID: return launch<BN, EPI_RESID>(a, b, c, c2, x, p, grid, st);
+    case EPI_SWIGLU: return launch<BN, EPI_SWIGLU>(a, b, c, c2, x, p, grid, st);
+    case EPI_DSWIGLU: return launch<BN, EPI_DSWIGLU>(a, b, c, c2, x, p, grid, st);
   }
   return cudaErrorNotSupported;
 }
@@ -656,9 +847,30 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   };
   const int BNsel = (g.N <= 128 || cost(128) < cost(256)) ? 128 : 256;
 
-  CUtensorMap ma, mb;
-  if (!make_map(&ma, g.A, g.M, g.K, g.lda, BM)) return cudaErrorNotSupported;
-  if (!make_map(&mb, g.B, g.N, g.K, g.ldb, BNsel)) return cudaErrorNotSupported;
+  CUtensorMap ma, mb, mc, mc2, mx;
+  memset(&mc, 0, sizeof mc);
+  memset(&mc2, 0, sizeof mc2);
+  memset(&mx, 0, sizeof mx);
+  if (!make_map(&ma, g.A, g.M, g.K, g.lda, 64, BM, DT_BF16)) return cudaErrorNotSupported;
+  if (!make_map(&mb, g.B, g.N, g.K, g.ldb, 64, BNsel, DT_BF16)) return cudaErrorNotSupported;
+  // output maps: C is [M, N] except the packed d(gate|up) output of the SwiGLU' epilogue,
+  // [M, 2N]; C2 is [M, N] (bias+GELU) or [M, N / 2] (h of the SwiGLU epilogue)
+  if (has_c) {
+    const int64_t cw = g.epi == EPI_DSWIGLU ? 2LL * g.N : g.N;
+    if (!make_map(&mc, g.C, g.M, cw, g.ldc, 32, 32, g.c_dtype)) return cudaErrorNotSupported;
+  }
+  if (g.C2) {
+    const int64_t cw2 = g.epi == EPI_SWIGLU ? g.N / 2 : g.N;
+    if (!make_map(&mc2, g.C2, g.M, cw2, g.ldc2, 32, 32, g.c2_dtype)) return cudaErrorNotSupported;
+  }
+  // operand map of the GELU' / residual / SwiGLU' epilogues: [M, N], or the packed
+  // [M, 2N] gate|up of SwiGLU' (always bf16)
+  if (g.epi == EPI_DGELU || g.epi == EPI_RESID || g.epi == EPI_DSWIGLU) {
+    if (!g.aux) return cudaErrorNotSupported;
+    if (g.epi == EPI_DSWIGLU && g.aux_dtype != DT_BF16) return cudaErrorNotSupported;
+    const int64_t xw = g.epi == EPI_DSWIGLU ? 2LL * g.N : g.N;
+    if (!make_map(&mx, g.aux, g.M, xw, g.ldaux, 32, 32, g.aux_dtype)) return cudaErrorNotSupported;
+  }
   TcParams p;
   p.M = g.M; p.N = g.N; p.K = g.K;
   p.n_tiles_n = (g.N + BNsel - 1) / BNsel;
@@ -672,7 +884,8 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   p.aux = g.aux; p.ldaux = g.ldaux; p.aux_dtype = g.aux_dtype;
   p.err = g.err;
   const int grid = p.num_tiles < sms ? p.num_tiles : sms;
-  return BNsel == 256 ? dispatch<256>(ma, mb, p, grid, st) : dispatch<128>(ma, mb, p, grid, st);
+  return BNsel == 256 ? dispatch<256>(ma, mb, mc, mc2, mx, p, grid, st)
+                      : dispatch<128>(ma, mb, mc, mc2, mx, p, grid, st);
 }
 
 }  // namespace ra
