@@ -32,18 +32,23 @@ METRIC = "fine-tune samples/sec vs unfrozen depth k"
 UNIT = "samples/s"
 HEADLINE_D = 6
 SWEEP = [1, 3, 6, 12]
+# other workloads (--config): depth sweep and headline depth of each
+SWEEPS = {"base": ([1, 3, 6, 12], 6), "large": ([1, 6, 12, 24], 12), "llama": ([4], 4),
+          "tiny": ([1, 2], 1)}
 CPU_SAMPLE_BATCH = 2      # sequences of 128 tokens per oracle step (bounded CPU sample)
 
 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="base")
     ap.add_argument("--no-large", action="store_true", help="skip the BERT-large GEMM check")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--schedule", action="store_true",
+                    help="run the 600-step top-down unfreezing schedule on the BERT-base workload")
     ap.add_argument("--cpu-worker", default=None, help=argparse.SUPPRESS)
     return ap.parse_args()
 
@@ -134,7 +139,7 @@ def start_clock_sampler(index):
     try:
         f = open(path, "w")
         p = subprocess.Popen(["nvidia-smi", "-i", str(index), "--query-gpu=" + q,
-                              "--format=csv,noheader,nounits", "-lms", "200"], stdout=f,
+                              "--format=csv,noheader,nounits", "-lms", "50"], stdout=f,
                              stderr=subprocess.DEVNULL)
         return p, f, path
     except Exception:
@@ -215,6 +220,7 @@ class Runner:
         self.loss_host = torch.zeros(1, dtype=torch.float32).pin_memory()
         self.graphs = {}
         self.launches = {}
+        self.saved = {}
 
     def step(self, d, stream=None):
         R, c = self.R, self.model.ctx
@@ -230,6 +236,7 @@ class Runner:
         self.step(d)                      # eager warm-up (also counts the launches of a step)
         torch.cuda.synchronize()
         self.launches[d] = R.ra_kernel_launches() - n0
+        self.saved[d] = self.model.stats()["saved_bytes_in_use"]
         g = torch.cuda.CUDAGraph()
         s = torch.cuda.Stream()
         s.wait_stream(torch.cuda.current_stream())
@@ -296,13 +303,15 @@ def gpu_main(args):
     from paper_2502_19864_gb300 import ringada as R
 
     cfg = synth.CONFIGS[args.config]
+    global SWEEP, HEADLINE_D
+    SWEEP, HEADLINE_D = SWEEPS[args.config]
     peaks, peak_kind = measured_peaks()
     steps, warmup = args.steps, max(3, args.warmup)
 
     # CPU baseline first (its own process, before the GPU work starts)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = run_cpu_baseline(args.config, HEADLINE_D, CPU_SAMPLE_BATCH, 12.0)
+        cpu = run_cpu_baseline(args.config, HEADLINE_D, 1 if cfg.batch < CPU_SAMPLE_BATCH else CPU_SAMPLE_BATCH, 12.0)
 
     run = Runner(cfg, max(SWEEP), device)
     sweep = {}
@@ -322,8 +331,8 @@ def gpu_main(args):
     sweep[HEADLINE_D] = ms
     prof = R.ra_profile_read(run.model.ctx)   # the last replay's per-kernel device times
     e2e_ms, h2d, d2h = run.time_e2e(HEADLINE_D, steps)
-    stats = run.model.stats()
     launches_headline = run.launches[HEADLINE_D]
+    saved_by_d = dict(run.saved)
     R.ra_set_unfrozen_depth(run.model.ctx, HEADLINE_D)
 
     # max over ranks
@@ -368,18 +377,21 @@ def gpu_main(args):
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
         "warmup": warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": "bert-base-shaped adapter step (12 post-LN layers, H 768, 12 "
-                               "heads, FFN 3072, adapters m 64, batch 32 x 128), d=%d" % HEADLINE_D,
+        "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
+        "config": {"workload": "%s-shaped adapter step (%d layers, H %d, %d heads, FFN %d, adapters "
+                               "m %d, batch %d x %d), d=%d" % (args.config, cfg.n_layers, cfg.hidden,
+                                                                cfg.n_heads, cfg.ffn, cfg.adapter_dim,
+                                                                cfg.batch, cfg.seq, HEADLINE_D),
                    "global_batch": B * world, "seq_len": cfg.seq, "depth": HEADLINE_D,
                    "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2 (>1 GB streamed per step)",
                    "cuda_graph": True},
         "sweep": {"d=%d" % d: {"samples_per_s": world * B / (sweep[d] / 1000.0),
-                               "ms_per_step": sweep[d], "k": cfg.n_layers - d}
+                               "ms_per_step": sweep[d], "k": cfg.n_layers - d,
+                               "saved_activation_bytes": saved_by_d[d]}
                   for d in sorted(sweep)},
         "monotone_in_k": all(sweep[a] > sweep[b] for a, b in zip(sorted(sweep)[1:], sorted(sweep))),
-        "saved_bytes_at_headline": stats["saved_bytes_in_use"],
+        "saved_bytes_at_headline": saved_by_d[HEADLINE_D],
         "roofline": roof,
         "phases_ms": phases,
         "clocks": clocks,
@@ -416,8 +428,71 @@ def large_gemm_check(torch, R, synth, device, peaks):
     return out
 
 
+def schedule_main(args):
+    """The schedule workload: 600 steps of BERT-base with d(s) = min(1 + s // 50, 12), Adam
+    lr 1e-4, one fresh synthetic batch per step (host pinned buffer -> device each step).
+    Reports per-depth step time and phase breakdown, saved-activation bytes per depth, and
+    the loss trajectory (the first five losses are checked against the oracle in the tests)."""
+    import torch
+    import synth
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2502_19864_gb300 import ringada as R
+    torch.cuda.set_device(0)
+    cfg = synth.CONFIGS["base"]
+    run = Runner(cfg, 12, "cuda:0")
+    n_steps, interval = 600, 50
+    batches = [synth.make_batch(cfg, 1000 + i) for i in range(4)]
+    xs = [torch.tensor(x, dtype=torch.float32).to(torch.bfloat16).pin_memory() for x, _ in batches]
+    ys = [torch.tensor(y, dtype=torch.int32).pin_memory() for _, y in batches]
+    per_d = {}
+    losses = []
+    for d in range(1, 13):
+        run.capture(d, profile=True)
+    torch.cuda.synchronize()
+    t_all = time.perf_counter()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_steps)]
+    loss_host = torch.zeros(n_steps, dtype=torch.float32).pin_memory()
+    for s in range(n_steps):
+        d = R.schedule_depth(s, interval=interval, d0=1, d_max=12)
+        run.x.copy_(xs[s % 4], non_blocking=True)
+        run.labels.copy_(ys[s % 4], non_blocking=True)
+        ev[s][0].record()
+        run.graphs[d].replay()
+        ev[s][1].record()
+        loss_host[s:s + 1].copy_(run.loss, non_blocking=True)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t_all
+    for s in range(n_steps):
+        d = R.schedule_depth(s, interval=interval, d0=1, d_max=12)
+        per_d.setdefault(d, []).append(ev[s][0].elapsed_time(ev[s][1]))
+    losses = loss_host.tolist()
+    # per-phase breakdown and saved bytes per depth (one profiled replay each)
+    phases, saved = {}, {}
+    for d in range(1, 13):
+        run.capture(d, profile=True)
+        run.graphs[d].replay()
+        torch.cuda.synchronize()
+        prof = R.ra_profile_read(run.model.ctx)
+        phases["d=%d" % d] = {k: round(v["ms"], 4) for k, v in prof.items()}
+        saved["d=%d" % d] = run.saved[d]
+    out = {
+        "workload": "schedule: bert-base 600 steps, d = min(1 + s // 50, 12), Adam lr 1e-4",
+        "steps": n_steps, "wall_s": wall,
+        "ms_per_step_by_depth": {"d=%d" % d: statistics.median(v) for d, v in sorted(per_d.items())},
+        "samples_per_s_overall": n_steps * cfg.batch / (sum(sum(v) for v in per_d.values()) / 1000.0),
+        "phases_ms_by_depth": phases,
+        "saved_activation_bytes_by_depth": saved,
+        "loss_first5": losses[:5], "loss_every50": losses[::50], "loss_last": losses[-1],
+    }
+    print(json.dumps(out))
+    return 0
+
+
 def main():
     args = parse()
+    if args.schedule:
+        return schedule_main(args)
     if args.cpu_worker:
         cpu_worker(args.cpu_worker)
         return 0
