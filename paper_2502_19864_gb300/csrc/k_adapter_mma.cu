@@ -43,6 +43,15 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t* r, const void* p) {
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
                : "r"(a));
 }
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem, bool valid) {
+  const uint32_t s = (uint32_t)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(s), "l"(gmem),
+               "r"(valid ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
 __device__ __forceinline__ uint32_t ld_u32(const bf16* p) {
   return __ldg(reinterpret_cast<const unsigned int*>(p));
 }
@@ -145,6 +154,7 @@ struct FwdArgs {
   float* x_out;           // decoder residual stream out
   bf16* xhat;             // encoder, nullable
   float* rstd;            // nullable
+  bool stage_resid;       // encoder: residual rows staged in shared memory (when they fit)
 };
 
 // Loads R rows of a bf16 [T, H] matrix into smem (ld = H + 8); rows >= T read as zero.
@@ -156,6 +166,17 @@ __device__ __forceinline__ void load_rows_bf16(bf16* dst, int ld, const bf16* sr
     uint4 v = make_uint4(0, 0, 0, 0);
     if (t0 + r < T) v = *reinterpret_cast<const uint4*>(src + (size_t)(t0 + r) * H + c);
     *reinterpret_cast<uint4*>(dst + (size_t)r * ld + c) = v;
+  }
+}
+// Issues cp.async copies of R rows of a bf16 [T, H] matrix into smem (ld = H + 8); rows >= T
+// are zero-filled.  The caller waits (cp_async_wait_all) and synchronises.
+__device__ __forceinline__ void load_rows_bf16_async(bf16* dst, int ld, const bf16* src, int t0, int T,
+                                                     int H, int R) {
+  const int vec = H / 8;
+  for (int e = threadIdx.x; e < R * vec; e += blockDim.x) {
+    const int r = e / vec, c = (e % vec) * 8;
+    const bool ok = t0 + r < T;
+    cp_async16(dst + (size_t)r * ld + c, src + (size_t)(ok ? t0 + r : 0) * H + c, ok);
   }
 }
 __device__ __forceinline__ void load_rows_f32_as_bf16(bf16* dst, int ld, const float* src, int t0,
@@ -170,10 +191,13 @@ __device__ __forceinline__ void load_rows_f32_as_bf16(bf16* dst, int ld, const f
   }
 }
 
-// WIDE: H > 1024 (up to 1024 threads, one CTA per SM); otherwise up to 512 threads and two
-// CTAs per SM.  Both cap the registers at 64 per thread.
-template <int MB, bool DEC, bool WIDE>
-__global__ void __launch_bounds__(WIDE ? 1024 : 512, WIDE ? 1 : 2) adapter_fwd_mma_kernel(FwdArgs p) {
+// Thread-count classes (H / 64 warps): SZ 0 for H <= 768 (two CTAs per SM at 85 registers),
+// SZ 1 for H <= 1024 (two CTAs per SM at 64), SZ 2 above (one CTA per SM, 64 registers).
+#define RA_ROWS_BOUNDS(SZ) __launch_bounds__((SZ) == 0 ? 384 : (SZ) == 1 ? 512 : 1024, (SZ) == 2 ? 1 : 2)
+__host__ __device__ constexpr int size_class(int H) { return H <= 768 ? 0 : H <= 1024 ? 1 : 2; }
+
+template <int MB, bool DEC, int SZ>
+__global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
   extern __shared__ __align__(16) uint8_t sm[];
   const int H = p.H, W = H / COLS_PER_WARP;
   const int KS = phase1_slice(H, MB), W1 = H / KS;
@@ -183,11 +207,16 @@ __global__ void __launch_bounds__(WIDE ? 1024 : 512, WIDE ? 1 : 2) adapter_fwd_m
   bf16* Ss = reinterpret_cast<bf16*>(part + (size_t)W1 * R * MB); // [R][MB + 8]
   float* stat = reinterpret_cast<float*>(Ss + (size_t)R * lds);   // [W][16]
   float* rowv = stat + W * 16;                                    // [16]
+  bf16* Rs = reinterpret_cast<bf16*>(rowv + 16);                  // encoder: [R][H + 8] residual
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, t = lane & 3;
   const int t0 = blockIdx.x * R;
 
-  load_rows_bf16(As, lda, p.a, t0, p.T, H, R);
+  // the row tile and (encoder) the residual rows are all in flight at once
+  load_rows_bf16_async(As, lda, p.a, t0, p.T, H, R);
+  if (!DEC && p.stage_resid)
+    load_rows_bf16_async(Rs, lda, reinterpret_cast<const bf16*>(p.resid), t0, p.T, H, R);
+  cp_async_wait_all();
   __syncthreads();
   if (warp < W1) phase1_store<MB>(As, lda, p.WdT, H, warp * KS, KS, part + (size_t)warp * R * MB, lane);
   __syncthreads();
@@ -215,6 +244,9 @@ __global__ void __launch_bounds__(WIDE ? 1024 : 512, WIDE ? 1 : 2) adapter_fwd_m
       const float* rs = reinterpret_cast<const float*>(p.resid);
       if (r0 < p.T) q0 = *reinterpret_cast<const float2*>(rs + (size_t)r0 * H + c);
       if (r1 < p.T) q1 = *reinterpret_cast<const float2*>(rs + (size_t)r1 * H + c);
+    } else if (p.stage_resid) {
+      q0 = unpack2(*reinterpret_cast<const uint32_t*>(Rs + (size_t)rl0 * lda + c));
+      q1 = unpack2(*reinterpret_cast<const uint32_t*>(Rs + (size_t)rl1 * lda + c));
     } else {
       const bf16* rs = reinterpret_cast<const bf16*>(p.resid);
       if (r0 < p.T) q0 = unpack2(*reinterpret_cast<const uint32_t*>(rs + (size_t)r0 * H + c));
@@ -323,8 +355,8 @@ struct BwdArgs {
   bf16* dh;           // [T, H] or null
 };
 
-template <int MB, bool WIDE>
-__global__ void __launch_bounds__(WIDE ? 1024 : 512, WIDE ? 1 : 2) adapter_bwd_rows_mma_kernel(BwdArgs p) {
+template <int MB, int SZ>
+__global__ void RA_ROWS_BOUNDS(SZ) adapter_bwd_rows_mma_kernel(BwdArgs p) {
   extern __shared__ __align__(16) uint8_t sm[];
   const int H = p.H;
   const int KS = phase1_slice(H, MB), W1 = H / KS;
@@ -493,15 +525,20 @@ __global__ void __launch_bounds__(256) adapter_dw_mma_kernel(DwArgs p) {
     }
 }
 
-size_t rows_smem(int H, int m) {
+// shared memory of the row kernels; the encoder forward also stages the residual rows
+size_t rows_smem(int H, int m, bool resid_rows = false) {
   const int W = H / COLS_PER_WARP, W1 = H / phase1_slice(H, m);
-  return (size_t)R * (H + 8) * 2 + (size_t)W1 * R * m * 4 + (size_t)R * (m + 8) * 2 + (W * 16 + 16) * 4;
+  return (size_t)R * (H + 8) * 2 + (size_t)W1 * R * m * 4 + (size_t)R * (m + 8) * 2 + (W * 16 + 16) * 4 +
+         (resid_rows ? (size_t)R * (H + 8) * 2 : 0);
 }
 
 template <int MB, bool DEC>
-cudaError_t launch_fwd(const FwdArgs& p, cudaStream_t st) {
-  const size_t smem = rows_smem(p.H, MB);
-  auto k = p.H > 1024 ? adapter_fwd_mma_kernel<MB, DEC, true> : adapter_fwd_mma_kernel<MB, DEC, false>;
+cudaError_t launch_fwd(FwdArgs p, cudaStream_t st) {
+  p.stage_resid = !DEC && rows_smem(p.H, MB, true) <= 220 * 1024;
+  const size_t smem = rows_smem(p.H, MB, p.stage_resid);
+  const int sz = size_class(p.H);
+  auto k = sz == 0 ? adapter_fwd_mma_kernel<MB, DEC, 0>
+         : sz == 1 ? adapter_fwd_mma_kernel<MB, DEC, 1> : adapter_fwd_mma_kernel<MB, DEC, 2>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k<<<(p.T + R - 1) / R, (p.H / COLS_PER_WARP) * 32, smem, st>>>(p);
@@ -512,7 +549,9 @@ cudaError_t launch_fwd(const FwdArgs& p, cudaStream_t st) {
 template <int MB>
 cudaError_t launch_bwd(const BwdArgs& p, cudaStream_t st) {
   const size_t smem = rows_smem(p.H, MB);
-  auto k = p.H > 1024 ? adapter_bwd_rows_mma_kernel<MB, true> : adapter_bwd_rows_mma_kernel<MB, false>;
+  const int sz = size_class(p.H);
+  auto k = sz == 0 ? adapter_bwd_rows_mma_kernel<MB, 0>
+         : sz == 1 ? adapter_bwd_rows_mma_kernel<MB, 1> : adapter_bwd_rows_mma_kernel<MB, 2>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k<<<(p.T + R - 1) / R, (p.H / COLS_PER_WARP) * 32, smem, st>>>(p);
