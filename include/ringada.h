@@ -198,6 +198,14 @@ ra_status ra_sync_status(ra_ctx* ctx, ra_stream_t stream);
  * RA_ERR_TIMEOUT and clears it.  Nothing faults or hangs, and the context stays usable. */
 ra_status ra_selftest_wait_timeout(ra_ctx* ctx, int32_t limit_us, ra_stream_t stream);
 
+/* Diagnostic: y = f(x) for n float32 values with the activation code the step's kernels
+ * use (the sigma of Eq. 1 and its derivative; SiLU of the decoder's SwiGLU FFN).
+ * which: 0 GELU(x) = x Phi(x), 1 GELU'(x) = Phi(x) + x phi(x), 2 SiLU, 3 SiLU'.
+ * x_dev, y_dev: device arrays of n floats owned by the caller (may alias).  Enqueued on
+ * `stream`; RA_ERR_ARG for another `which` or n < 0, RA_ERR_CUDA on a launch error. */
+ra_status ra_eval_activation(int32_t which, const float* x_dev, float* y_dev, int64_t n,
+                             ra_stream_t stream);
+
 /* Message of the last failing call on ctx (never null; "" if none). */
 const char* ra_last_error(const ra_ctx* ctx);
 

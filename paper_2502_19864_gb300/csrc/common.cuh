@@ -29,12 +29,32 @@ __device__ __forceinline__ float warp_max(float v) {
 }
 
 // ---- GELU (sigma of Eq. 1, exact erf form) --------------------------------------------
-__device__ __forceinline__ float gelu_f(float x) {
-  return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
+// erf by Abramowitz & Stegun, Handbook of Mathematical Functions, formula 7.1.28:
+//   erf(x) = 1 - (1 + a1 x + ... + a6 x^6)^-16 for x >= 0, odd extension, |error| <= 3e-7.
+// Evaluated without cancellation: with e = p - 1 carried exactly through the four squarings
+// (p^2k - 1 = e (2 + e)), erf = e16 / (1 + e16); x is clamped at 5, where erf is 1 in fp32.
+// Branch-free with one reciprocal; the epilogues that evaluate GELU or GELU' for every
+// element of a large tile run it instead of a general-purpose erf.
+__device__ __forceinline__ float erf_as7128(float x) {
+  const float t = fminf(fabsf(x), 5.0f);
+  float p = fmaf(t, 4.30638e-5f, 2.765672e-4f);
+  p = fmaf(t, p, 1.520143e-4f);
+  p = fmaf(t, p, 9.2705272e-3f);
+  p = fmaf(t, p, 4.22820123e-2f);
+  float e = t * fmaf(t, p, 7.05230784e-2f);  // p - 1
+  e *= 2.0f + e;  // p^2 - 1
+  e *= 2.0f + e;  // p^4 - 1
+  e *= 2.0f + e;  // p^8 - 1
+  e *= 2.0f + e;  // p^16 - 1
+  return copysignf(__fdividef(e, 1.0f + e), x);
 }
+__device__ __forceinline__ float gelu_f(float x) {
+  return 0.5f * x * (1.0f + erf_as7128(x * 0.70710678118654752f));
+}
+// d/dx GELU = Phi(x) + x phi(x)
 __device__ __forceinline__ float gelu_grad_f(float x) {
-  return 0.5f * (1.0f + erff(x * 0.70710678118654752f)) +
-         x * expf(-0.5f * x * x) * 0.39894228040143268f;
+  return 0.5f * (1.0f + erf_as7128(x * 0.70710678118654752f)) +
+         x * __expf(-0.5f * x * x) * 0.39894228040143268f;
 }
 __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
 __device__ __forceinline__ float silu_grad_f(float x) {

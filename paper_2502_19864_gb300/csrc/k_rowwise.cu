@@ -581,6 +581,13 @@ __global__ void adapter_transpose_kernel(const float* P, float* PT, bf16* PB, bf
   if (PTB) PTB[base + (int64_t)c * rows + frag_pos(r)] = __float2bfloat16_rn(v);
 }
 
+__global__ void activation_kernel(int which, const float* x, float* y, int64_t n) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const float v = x[i];
+  y[i] = which == 0 ? gelu_f(v) : which == 1 ? gelu_grad_f(v) : which == 2 ? silu_f(v) : silu_grad_f(v);
+}
+
 __global__ void fill_kernel(float* dst, float v, int64_t n) {
   int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) dst[i] = v;
@@ -769,6 +776,13 @@ cudaError_t adapter_transpose(const float* P, float* PT, void* PB, void* PTB, in
   dim3 grid(blocks_for((int64_t)H * m, 256), 1, 4 * n_layers);
   adapter_transpose_kernel<<<grid, 256, 0, st>>>(P, PT, reinterpret_cast<bf16*>(PB),
                                                  reinterpret_cast<bf16*>(PTB), H, m);
+  note_launch(1);
+  return cudaGetLastError();
+}
+
+cudaError_t eval_activation(int which, const float* x, float* y, int64_t n, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  activation_kernel<<<blocks_for(n, 256), 256, 0, st>>>(which, x, y, n);
   note_launch(1);
   return cudaGetLastError();
 }

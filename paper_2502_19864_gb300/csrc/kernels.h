@@ -199,5 +199,8 @@ cudaError_t pack_rows(const float* src, void* dst, int dst_dtype, int R, int C, 
 cudaError_t adapter_transpose(const float* P, float* PT, void* PB, void* PTB, int n_layers,
                               int H, int m, cudaStream_t st);
 cudaError_t fill_f32(float* dst, float v, int64_t n, cudaStream_t st);
+// y = f(x) elementwise with the step kernels' own activation code: which 0 GELU, 1 GELU',
+// 2 SiLU, 3 SiLU'
+cudaError_t eval_activation(int which, const float* x, float* y, int64_t n, cudaStream_t st);
 
 }  // namespace ra

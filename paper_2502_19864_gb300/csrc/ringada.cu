@@ -1093,6 +1093,12 @@ ra_status ra_selftest_wait_timeout(ra_ctx* ctx, int32_t limit_us, ra_stream_t st
   return RA_OK;
 }
 
+ra_status ra_eval_activation(int32_t which, const float* x_dev, float* y_dev, int64_t n,
+                             ra_stream_t stream) {
+  if (which < 0 || which > 3 || n < 0 || (n > 0 && (!x_dev || !y_dev))) return RA_ERR_ARG;
+  return eval_activation(which, x_dev, y_dev, n, (cudaStream_t)stream) == cudaSuccess ? RA_OK : RA_ERR_CUDA;
+}
+
 const char* ra_last_error(const ra_ctx* ctx) { return ctx ? ctx->err.c_str() : "null context"; }
 
 void ra_destroy(ra_ctx* ctx) { delete ctx; }

@@ -111,6 +111,7 @@ _SIGS = {
     "ra_sync_status": (C.c_int, [C.c_void_p, C.c_void_p]),
     "ra_last_error": (C.c_char_p, [C.c_void_p]),
     "ra_selftest_wait_timeout": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p]),
+    "ra_eval_activation": (C.c_int, [C.c_int32, C.c_void_p, C.c_void_p, C.c_int64, C.c_void_p]),
     "ra_destroy": (None, [C.c_void_p]),
     "ra_gemm_bf16": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32,
                                C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p]),
@@ -246,6 +247,10 @@ def ra_sync_status(ctx, stream=None):
 
 def ra_selftest_wait_timeout(ctx, limit_us: int, stream=None):
     _check(lib().ra_selftest_wait_timeout(ctx, limit_us, _stream_ptr(stream)), ctx)
+
+
+def ra_eval_activation(which: int, x_ptr, y_ptr, n: int, stream=None):
+    _check(lib().ra_eval_activation(which, x_ptr, y_ptr, n, _stream_ptr(stream)))
 
 
 def ra_last_error(ctx) -> str:
