@@ -55,10 +55,13 @@ __device__ __forceinline__ void cp_async_wait_all() {
 __device__ __forceinline__ uint32_t ld_u32(const bf16* p) {
   return __ldg(reinterpret_cast<const unsigned int*>(p));
 }
-// B fragments of two k16 steps from a fragment-major weight row (see frag_pos): .x/.y are
-// b0/b1 of the first step, .z/.w of the second
-__device__ __forceinline__ uint4 ld_frag2(const bf16* row, int k0, int t) {
-  return __ldg(reinterpret_cast<const uint4*>(row + k0 + t * 8));
+// B fragments of n8 tile `ntile` (rows 8 ntile .. + 7) for the two k16 steps at k0 (a
+// multiple of 32) of a [R, C] bf16 weight in the tiled fragment layout (8 x 32 blocks of 256
+// contiguous elements, each row of a block in fragment order): lane l reads elements
+// [8 l, 8 l + 8) of the block, 512 contiguous bytes per warp.  .x/.y are b0/b1 of the first
+// step, .z/.w of the second.
+__device__ __forceinline__ uint4 ld_frag2(const bf16* W, int C, int ntile, int k0, int lane) {
+  return __ldg(reinterpret_cast<const uint4*>(W + ((size_t)ntile * (C >> 5) + (k0 >> 5)) * 256 + lane * 8));
 }
 __device__ __forceinline__ uint32_t pack2(float a, float b) {
   __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
@@ -77,7 +80,7 @@ __device__ __forceinline__ void load_a(uint32_t* a, const bf16* s, int ld, int r
 }
 
 // Phase 1 shared by forward and backward: part[w] = X[16, kslice] * Bw^T over this warp's
-// slice [kbase, kbase + ks_len) of H, where Bw is [m, H] bf16 in fragment-major order (B
+// slice [kbase, kbase + ks_len) of H, where Bw is [m, H] bf16 in the tiled fragment layout (B
 // fragments read directly, 16 bytes per thread per two k16 steps; the matrix is small and
 // stays in L1/L2).  The m output columns
 // are produced in groups of 8 n-tiles to bound the registers.
@@ -98,7 +101,7 @@ __device__ __forceinline__ void phase1_store(const bf16* Xs, int ldx, const bf16
       load_a(a1, Xs, ldx, 0, k0 + 16, lane);
 #pragma unroll
       for (int nt = 0; nt < NTG; ++nt) {
-        const uint4 b = ld_frag2(Bw + (size_t)(ng * 64 + nt * 8 + g) * H, k0, t);
+        const uint4 b = ld_frag2(Bw, H, ng * 8 + nt, k0, lane);
         mma_bf16(acc[nt], a0, b.x, b.y);
         mma_bf16(acc[nt], a1, b.z, b.w);
       }
@@ -119,7 +122,7 @@ __host__ __device__ inline int phase1_slice(int H, int m) {
 }
 
 // Phase 2: acc[16 rows, this warp's 64 columns] = S[16, m] * Bn^T where Bn is [H, m] bf16
-// in fragment-major order (n = output column, k = bottleneck index).
+// in the tiled fragment layout (n = output column, k = bottleneck index).
 template <int MB>
 __device__ __forceinline__ void phase2(float (&acc)[8][4], const bf16* Ss, int lds,
                                        const bf16* Bn, int m, int nbase, int lane) {
@@ -133,7 +136,7 @@ __device__ __forceinline__ void phase2(float (&acc)[8][4], const bf16* Ss, int l
     load_a(a1, Ss, lds, 0, k0 + 16, lane);
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
-      const uint4 b = ld_frag2(Bn + (size_t)(nbase + nt * 8 + g) * m, k0, t);
+      const uint4 b = ld_frag2(Bn, m, (nbase >> 3) + nt, k0, lane);
       mma_bf16(acc[nt], a0, b.x, b.y);
       mma_bf16(acc[nt], a1, b.z, b.w);
     }

@@ -567,7 +567,19 @@ __device__ __forceinline__ int frag_pos(int k) {
   const int w = k & 31;
   return (k & ~31) + ((w & 7) >> 1) * 8 + (w >> 3) * 2 + (w & 1);
 }
+// Offset of element (n, k) of a bf16 [R, C] matrix in the tiled fragment layout the
+// tensor-core adapter kernels read: 8-row x 32-column blocks of 256 contiguous elements,
+// ordered by row block then column block; inside a block, row n & 7 holds its 32 columns in
+// the m16n8k16 B-fragment order (frag_pos), so the 32 lanes of a warp load the fragments of
+// one n8 tile and two k16 steps as 512 contiguous bytes.
+__device__ __forceinline__ int64_t tfrag_off(int n, int k, int C) {
+  return ((int64_t)(n >> 3) * (C >> 5) + (k >> 5)) * 256 + (n & 7) * 32 + frag_pos(k & 31);
+}
 
+// P (f32 masters) -> PT (f32, transposed) and, for bf16 models, the shadows PB (the master's
+// layout [rows, cols]) and PTB (transposed [cols, rows]) in the tiled fragment layout; when
+// H or m is not a multiple of 32 (no tensor-core kernel reads them then) they are plain
+// row-major copies.
 __global__ void adapter_transpose_kernel(const float* P, float* PT, bf16* PB, bf16* PTB, int H, int m) {
   int layer = blockIdx.z >> 2, mat = blockIdx.z & 3;
   int64_t base = (int64_t)layer * 4 * H * m + (int64_t)mat * H * m;
@@ -577,8 +589,9 @@ __global__ void adapter_transpose_kernel(const float* P, float* PT, bf16* PB, bf
   int r = (int)(e / cols), c = (int)(e % cols);
   const float v = P[base + e];
   PT[base + (int64_t)c * rows + r] = v;
-  if (PB) PB[base + (int64_t)r * cols + frag_pos(c)] = __float2bfloat16_rn(v);
-  if (PTB) PTB[base + (int64_t)c * rows + frag_pos(r)] = __float2bfloat16_rn(v);
+  const bool tiled = (H % 32 == 0) && (m % 32 == 0);
+  if (PB) PB[base + (tiled ? tfrag_off(r, c, cols) : e)] = __float2bfloat16_rn(v);
+  if (PTB) PTB[base + (tiled ? tfrag_off(c, r, rows) : (int64_t)c * rows + r)] = __float2bfloat16_rn(v);
 }
 
 __global__ void activation_kernel(int which, const float* x, float* y, int64_t n) {
