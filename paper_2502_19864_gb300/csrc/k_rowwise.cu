@@ -370,6 +370,128 @@ __global__ void rmsnorm_bwd_kernel(const float* dy, const float* x, const float*
 }
 
 // ---------------------------------------------------------------------------------------
+// Row-resident norm kernels for H = 128 V: one warp per row, the row held in registers
+// (V float4 per lane, lane-contiguous so a warp access is 512 contiguous bytes), one pass
+// over memory.  Same arithmetic as the kernels above, with vector accesses.
+// ---------------------------------------------------------------------------------------
+template <typename T> __device__ __forceinline__ float4 ld4(const void* p, int64_t i);
+template <> __device__ __forceinline__ float4 ld4<float>(const void* p, int64_t i) {
+  return *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(p) + i);
+}
+template <> __device__ __forceinline__ float4 ld4<bf16>(const void* p, int64_t i) {
+  const uint2 u = *reinterpret_cast<const uint2*>(reinterpret_cast<const bf16*>(p) + i);
+  const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+  const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+  return make_float4(a.x, a.y, b.x, b.y);
+}
+template <typename T> __device__ __forceinline__ void st4(void* p, int64_t i, float4 v);
+template <> __device__ __forceinline__ void st4<float>(void* p, int64_t i, float4 v) {
+  *reinterpret_cast<float4*>(reinterpret_cast<float*>(p) + i) = v;
+}
+template <> __device__ __forceinline__ void st4<bf16>(void* p, int64_t i, float4 v) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+  uint2 u;
+  u.x = *reinterpret_cast<uint32_t*>(&a);
+  u.y = *reinterpret_cast<uint32_t*>(&b);
+  *reinterpret_cast<uint2*>(reinterpret_cast<bf16*>(p) + i) = u;
+}
+
+template <typename TX, int V>
+__global__ void __launch_bounds__(256) layernorm_bwd_vec_kernel(const float* dy, const void* xhat,
+    const float* rstd, const float* gamma, float* ds, int Tn, int H) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= Tn) return;
+  const int64_t base = (int64_t)row * H;
+  float4 g[V], x[V];
+  float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    const int c = (v * 32 + lane) * 4;
+    const float4 d = ld4<float>(dy, base + c), gm = ld4<float>(gamma, c);
+    g[v] = make_float4(d.x * gm.x, d.y * gm.y, d.z * gm.z, d.w * gm.w);
+    x[v] = ld4<TX>(xhat, base + c);
+    s1 += g[v].x + g[v].y + g[v].z + g[v].w;
+    s2 += g[v].x * x[v].x + g[v].y * x[v].y + g[v].z * x[v].z + g[v].w * x[v].w;
+  }
+  s1 = warp_sum(s1) / H;
+  s2 = warp_sum(s2) / H;
+  const float r = rstd[row];
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    const int c = (v * 32 + lane) * 4;
+    st4<float>(ds, base + c, make_float4(r * (g[v].x - s1 - x[v].x * s2), r * (g[v].y - s1 - x[v].y * s2),
+                                         r * (g[v].z - s1 - x[v].z * s2), r * (g[v].w - s1 - x[v].w * s2)));
+  }
+}
+
+template <typename TX, typename TN, int V>
+__global__ void __launch_bounds__(256) rmsnorm_fwd_vec_kernel(const void* x, const float* gamma, float eps,
+    void* n, float* rstd, float* xf, int Tn, int H) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= Tn) return;
+  const int64_t base = (int64_t)row * H;
+  float4 a[V];
+  float q = 0.f;
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    a[v] = ld4<TX>(x, base + (v * 32 + lane) * 4);
+    q += a[v].x * a[v].x + a[v].y * a[v].y + a[v].z * a[v].z + a[v].w * a[v].w;
+  }
+  const float r = rsqrtf(warp_sum(q) / H + eps);
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    const int c = (v * 32 + lane) * 4;
+    const float4 gm = ld4<float>(gamma, c);
+    st4<TN>(n, base + c, make_float4(a[v].x * r * gm.x, a[v].y * r * gm.y, a[v].z * r * gm.z, a[v].w * r * gm.w));
+    if (xf) st4<float>(xf, base + c, a[v]);
+  }
+  if (rstd && lane == 0) rstd[row] = r;
+}
+
+template <int V>
+__global__ void __launch_bounds__(256) rmsnorm_bwd_vec_kernel(const float* dy, const float* x, const float* rstd,
+    const float* gamma, const float* resid, float* dx, int Tn, int H) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= Tn) return;
+  const int64_t base = (int64_t)row * H;
+  float4 g[V], a[V];
+  float s = 0.f;
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    const int c = (v * 32 + lane) * 4;
+    const float4 d = ld4<float>(dy, base + c), gm = ld4<float>(gamma, c);
+    g[v] = make_float4(d.x * gm.x, d.y * gm.y, d.z * gm.z, d.w * gm.w);
+    a[v] = ld4<float>(x, base + c);
+    s += g[v].x * a[v].x + g[v].y * a[v].y + g[v].z * a[v].z + g[v].w * a[v].w;
+  }
+  s = warp_sum(s) / H;
+  const float r = rstd[row], k = r * r * r * s;
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    const int c = (v * 32 + lane) * 4;
+    const float4 q = resid ? ld4<float>(resid, base + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+    st4<float>(dx, base + c, make_float4(q.x + r * g[v].x - a[v].x * k, q.y + r * g[v].y - a[v].y * k,
+                                         q.z + r * g[v].z - a[v].z * k, q.w + r * g[v].w - a[v].w * k));
+  }
+}
+
+// V for the row-resident kernels (0: use the scalar kernels)
+inline int row_vec(int H) {
+  if (H % 128) return 0;
+  const int v = H / 128;
+  return (v == 1 || v == 2 || v == 4 || v == 6 || v == 8 || v == 16) ? v : 0;
+}
+#define RA_VEC_SWITCH(V, CALL)                 \
+  switch (V) {                                 \
+    case 1: { constexpr int VV = 1; CALL; } break;  \
+    case 2: { constexpr int VV = 2; CALL; } break;  \
+    case 4: { constexpr int VV = 4; CALL; } break;  \
+    case 6: { constexpr int VV = 6; CALL; } break;  \
+    case 8: { constexpr int VV = 8; CALL; } break;  \
+    case 16: { constexpr int VV = 16; CALL; } break; \
+  }
+
+// ---------------------------------------------------------------------------------------
 // Heads
 // ---------------------------------------------------------------------------------------
 constexpr int MAXC = 32, MAXB = 256;
@@ -675,8 +797,14 @@ cudaError_t layernorm_bwd(const float* dy, const void* xhat, const float* rstd,
                           const float* gamma, float* ds, int T, int H, int dtype,
                           cudaStream_t st) {
   unsigned grid = blocks_for((int64_t)T * 32, 256);
-  if (dtype == DT_BF16) layernorm_bwd_kernel<bf16><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H);
-  else layernorm_bwd_kernel<float><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H);
+  if (const int V = row_vec(H)) {
+    if (dtype == DT_BF16) RA_VEC_SWITCH(V, (layernorm_bwd_vec_kernel<bf16, VV><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H)))
+    else RA_VEC_SWITCH(V, (layernorm_bwd_vec_kernel<float, VV><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H)))
+  } else if (dtype == DT_BF16) {
+    layernorm_bwd_kernel<bf16><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H);
+  } else {
+    layernorm_bwd_kernel<float><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H);
+  }
   note_launch(1);
   return cudaGetLastError();
 }
@@ -685,6 +813,18 @@ cudaError_t rmsnorm_fwd(const void* x, int x_dtype, const float* gamma, float ep
                         int n_dtype, float* rstd, float* x_f32_out, int T, int H,
                         cudaStream_t st) {
   unsigned grid = blocks_for((int64_t)T * 32, 256);
+  if (const int V = row_vec(H)) {
+    if (x_dtype == DT_BF16 && n_dtype == DT_BF16)
+      RA_VEC_SWITCH(V, (rmsnorm_fwd_vec_kernel<bf16, bf16, VV><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H)))
+    else if (x_dtype == DT_F32 && n_dtype == DT_BF16)
+      RA_VEC_SWITCH(V, (rmsnorm_fwd_vec_kernel<float, bf16, VV><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H)))
+    else if (x_dtype == DT_BF16)
+      RA_VEC_SWITCH(V, (rmsnorm_fwd_vec_kernel<bf16, float, VV><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H)))
+    else
+      RA_VEC_SWITCH(V, (rmsnorm_fwd_vec_kernel<float, float, VV><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H)))
+    note_launch(1);
+    return cudaGetLastError();
+  }
   if (x_dtype == DT_BF16 && n_dtype == DT_BF16)
     rmsnorm_fwd_kernel<bf16, bf16><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H);
   else if (x_dtype == DT_F32 && n_dtype == DT_BF16)
@@ -699,7 +839,10 @@ cudaError_t rmsnorm_fwd(const void* x, int x_dtype, const float* gamma, float ep
 
 cudaError_t rmsnorm_bwd(const float* dy, const float* x, const float* rstd, const float* gamma,
                         const float* resid, float* dx, int T, int H, cudaStream_t st) {
-  rmsnorm_bwd_kernel<<<blocks_for((int64_t)T * 32, 256), 256, 0, st>>>(dy, x, rstd, gamma, resid, dx, T, H);
+  if (const int V = row_vec(H))
+    RA_VEC_SWITCH(V, (rmsnorm_bwd_vec_kernel<VV><<<blocks_for((int64_t)T * 32, 256), 256, 0, st>>>(dy, x, rstd, gamma, resid, dx, T, H)))
+  else
+    rmsnorm_bwd_kernel<<<blocks_for((int64_t)T * 32, 256), 256, 0, st>>>(dy, x, rstd, gamma, resid, dx, T, H);
   note_launch(1);
   return cudaGetLastError();
 }
