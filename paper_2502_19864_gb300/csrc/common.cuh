@@ -41,20 +41,52 @@ __device__ __forceinline__ float erf_as7128(float x) {
   p = fmaf(t, p, 1.520143e-4f);
   p = fmaf(t, p, 9.2705272e-3f);
   p = fmaf(t, p, 4.22820123e-2f);
-  float e = t * fmaf(t, p, 7.05230784e-2f);  // p - 1
-  e *= 2.0f + e;  // p^2 - 1
-  e *= 2.0f + e;  // p^4 - 1
-  e *= 2.0f + e;  // p^8 - 1
-  e *= 2.0f + e;  // p^16 - 1
-  return copysignf(__fdividef(e, 1.0f + e), x);
+  float e = __fmul_rn(t, fmaf(t, p, 7.05230784e-2f));  // p - 1
+  e = __fmul_rn(e, __fadd_rn(e, 2.0f));  // p^2 - 1
+  e = __fmul_rn(e, __fadd_rn(e, 2.0f));  // p^4 - 1
+  e = __fmul_rn(e, __fadd_rn(e, 2.0f));  // p^8 - 1
+  e = __fmul_rn(e, __fadd_rn(e, 2.0f));  // p^16 - 1
+  return copysignf(__fdividef(e, __fadd_rn(e, 1.0f)), x);
 }
+// GELU(x) = x Phi(x) = h + h erf(x / sqrt 2) with h = x / 2.  The operation sequence (no
+// contraction) is the one the packed form below applies to each component, so both give
+// bitwise the same result.
 __device__ __forceinline__ float gelu_f(float x) {
-  return 0.5f * x * (1.0f + erf_as7128(x * 0.70710678118654752f));
+  const float h = __fmul_rn(x, 0.5f);
+  return __fmaf_rn(h, erf_as7128(__fmul_rn(x, 0.70710678118654752f)), h);
 }
 // d/dx GELU = Phi(x) + x phi(x)
 __device__ __forceinline__ float gelu_grad_f(float x) {
-  return 0.5f * (1.0f + erf_as7128(x * 0.70710678118654752f)) +
-         x * __expf(-0.5f * x * x) * 0.39894228040143268f;
+  const float Phi = __fmaf_rn(erf_as7128(__fmul_rn(x, 0.70710678118654752f)), 0.5f, 0.5f);
+  const float q = __fmul_rn(__fmul_rn(x, -0.5f), x);
+  return __fadd_rn(Phi, __fmul_rn(__fmul_rn(x, __expf(q)), 0.39894228040143268f));
+}
+
+// ---- packed forms: two values per instruction with the sm_100 fp32x2 arithmetic --------
+__device__ __forceinline__ float2 f2(float v) { return make_float2(v, v); }
+__device__ __forceinline__ float2 erf2_as7128(float2 x) {
+  const float2 t = make_float2(fminf(fabsf(x.x), 5.0f), fminf(fabsf(x.y), 5.0f));
+  float2 p = __ffma2_rn(t, f2(4.30638e-5f), f2(2.765672e-4f));
+  p = __ffma2_rn(t, p, f2(1.520143e-4f));
+  p = __ffma2_rn(t, p, f2(9.2705272e-3f));
+  p = __ffma2_rn(t, p, f2(4.22820123e-2f));
+  float2 e = __fmul2_rn(t, __ffma2_rn(t, p, f2(7.05230784e-2f)));  // p - 1
+  e = __fmul2_rn(e, __fadd2_rn(e, f2(2.0f)));  // p^2 - 1
+  e = __fmul2_rn(e, __fadd2_rn(e, f2(2.0f)));  // p^4 - 1
+  e = __fmul2_rn(e, __fadd2_rn(e, f2(2.0f)));  // p^8 - 1
+  e = __fmul2_rn(e, __fadd2_rn(e, f2(2.0f)));  // p^16 - 1
+  const float2 d = __fadd2_rn(e, f2(1.0f));
+  return make_float2(copysignf(__fdividef(e.x, d.x), x.x), copysignf(__fdividef(e.y, d.y), x.y));
+}
+__device__ __forceinline__ float2 gelu2(float2 x) {
+  const float2 h = __fmul2_rn(x, f2(0.5f));
+  return __ffma2_rn(h, erf2_as7128(__fmul2_rn(x, f2(0.70710678118654752f))), h);
+}
+__device__ __forceinline__ float2 gelu_grad2(float2 x) {
+  const float2 Phi = __ffma2_rn(erf2_as7128(__fmul2_rn(x, f2(0.70710678118654752f))), f2(0.5f), f2(0.5f));
+  const float2 q = __fmul2_rn(__fmul2_rn(x, f2(-0.5f)), x);
+  const float2 ex = make_float2(__expf(q.x), __expf(q.y));
+  return __fadd2_rn(Phi, __fmul2_rn(__fmul2_rn(x, ex), f2(0.39894228040143268f)));
 }
 __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
 __device__ __forceinline__ float silu_grad_f(float x) {

@@ -305,97 +305,64 @@ __device__ __forceinline__ void store_chunk(const CUtensorMap* tm, uint8_t* stag
   ++slot_i;
 }
 
-__device__ __forceinline__ void load8(const void* base, int dt, int64_t off, float* v) {
-  if (dt == DT_BF16) {
-    uint4 q = *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(base) + off);
-    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&q);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float2 f = __bfloat1622float2(h[i]);
-      v[2 * i] = f.x;
-      v[2 * i + 1] = f.y;
-    }
-  } else {
-    const float4* p = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(base) + off);
-    float4 a = p[0], b = p[1];
-    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-  }
-}
-
-// Operands of one row's 32-column chunk [n, n + 32) that do not come from TMEM (bias,
-// saved pre-activations, residual), fetched before the TMEM load completes.
+// Bias of one row's 32-column chunk [n, n + 32) (read from registers of the warp).
 template <int EPI>
 struct EpiIn {
-  float bias[EPI == EPI_STORE || EPI == EPI_BIAS_GELU ? 32 : 1];
-  float aux[EPI == EPI_DGELU || EPI == EPI_RESID ? 32 : (EPI == EPI_DSWIGLU ? 64 : 1)];
+  float bias[32];
 };
 
-template <int EPI>
-__device__ __forceinline__ void epi_fetch(const TcParams& p, int row, int n, EpiIn<EPI>& in) {
+// GELU of 8 values, kept out of line: the epilogue then carries one copy of its code instead
+// of one per element, which keeps the hot loop inside the instruction cache.
+struct F8 {
+  float v[8];
+};
+__device__ __noinline__ F8 gelu8(F8 x) {
 #pragma unroll
-  for (int g = 0; g < 4; ++g) {
-    const int c = n + 8 * g;
-    if (c >= p.N) break;
-    if (EPI == EPI_STORE || EPI == EPI_BIAS_GELU) {
-      if (p.bias) {
-        const float4 b0 = *reinterpret_cast<const float4*>(p.bias + c);
-        const float4 b1 = *reinterpret_cast<const float4*>(p.bias + c + 4);
-        float* b = in.bias + 8 * g;
-        b[0] = b0.x; b[1] = b0.y; b[2] = b0.z; b[3] = b0.w;
-        b[4] = b1.x; b[5] = b1.y; b[6] = b1.z; b[7] = b1.w;
-      } else {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) in.bias[8 * g + i] = 0.f;
-      }
-    } else if (EPI == EPI_DGELU || EPI == EPI_RESID) {
-      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + c, in.aux + 8 * g);
-    } else if (EPI == EPI_DSWIGLU) {
-      const int64_t gc = (int64_t)(c >> 6) * 128 + (c & 63);
-      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + gc, in.aux + 8 * g);
-      load8(p.aux, p.aux_dtype, (int64_t)row * p.ldaux + gc + 64, in.aux + 32 + 8 * g);
-    }
+  for (int i = 0; i < 8; i += 2) {
+    const float2 y = gelu2(make_float2(x.v[i], x.v[i + 1]));
+    x.v[i] = y.x;
+    x.v[i + 1] = y.y;
   }
+  return x;
+}
+// g * GELU'(u) for 8 values, out of line for the same reason
+__device__ __noinline__ F8 dgelu8(F8 g, F8 u) {
+#pragma unroll
+  for (int i = 0; i < 8; i += 2) {
+    const float2 y = __fmul2_rn(make_float2(g.v[i], g.v[i + 1]), gelu_grad2(make_float2(u.v[i], u.v[i + 1])));
+    g.v[i] = y.x;
+    g.v[i + 1] = y.y;
+  }
+  return g;
 }
 
-// One warp's 32 x 32 chunk of output C (non-SwiGLU epilogues): rows row0.., columns n..
-// (this thread holds row row0 + lane in v).
+// One warp's 32 x 32 chunk of output C of the STORE and BIAS_GELU epilogues: rows row0..,
+// columns n.. (this thread holds row row0 + lane in v).
 template <int EPI>
 __device__ __forceinline__ void epi_chunk(const TcParams& p, const CUtensorMap* tmC,
                                           const CUtensorMap* tmC2, uint8_t* staging, int& slot_i,
                                           int lane, int row0, int n, float* v, const EpiIn<EPI>& in,
                                           bool ts) {
-  if (EPI == EPI_STORE) {
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] += in.bias[i];
+  for (int i = 0; i < 32; i += 2) {
+    const float2 y = __fadd2_rn(make_float2(v[i], v[i + 1]), make_float2(in.bias[i], in.bias[i + 1]));
+    v[i] = y.x;
+    v[i + 1] = y.y;
+  }
+  if (EPI == EPI_STORE) {
     store_chunk(tmC, staging, slot_i, p.c_dtype, lane, v, n, row0, ts);
   } else if (EPI == EPI_BIAS_GELU) {
-#pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] += in.bias[i];
     if (p.C) store_chunk(tmC, staging, slot_i, p.c_dtype, lane, v, n, row0, ts);
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = gelu_f(v[i]);
-    store_chunk(tmC2, staging, slot_i, p.c2_dtype, lane, v, n, row0, ts);
-  } else if (EPI == EPI_DGELU) {
+    for (int j = 0; j < 32; j += 8) {
+      F8 x;
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(in.aux[i]);
-    store_chunk(tmC, staging, slot_i, p.c_dtype, lane, v, n, row0, ts);
-  } else if (EPI == EPI_RESID) {
+      for (int i = 0; i < 8; ++i) x.v[i] = v[j + i];
+      x = gelu8(x);
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] += in.aux[i];
-    store_chunk(tmC, staging, slot_i, p.c_dtype, lane, v, n, row0, ts);
-  } else if (EPI == EPI_DSWIGLU) {
-    // columns n.. of d(h) -> packed gate columns gc.. and up columns gc + 64..
-    const int gc = (n >> 6) * 128 + (n & 63);
-    float du[32];
-#pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      const float gt = in.aux[i], up = in.aux[32 + i];
-      du[i] = v[i] * silu_f(gt);
-      v[i] = v[i] * up * silu_grad_f(gt);
+      for (int i = 0; i < 8; ++i) v[j + i] = x.v[i];
     }
-    store_chunk(tmC, staging, slot_i, p.c_dtype, lane, v, gc, row0, ts);
-    store_chunk(tmC, staging, slot_i, p.c_dtype, lane, du, gc + 64, row0, ts);
+    store_chunk(tmC2, staging, slot_i, p.c2_dtype, lane, v, n, row0, ts);
   }
 }
 
@@ -569,6 +536,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const int cbeg = half * (BN / 2), cend = cbeg + BN / 2;
       // the first operand chunk is fetched while the main loop of this tile still runs
       if (EpiTraits<EPI>::AUX && n0 + cbeg < p.N && row0 < p.M) aux_issue(row0, n0 + cbeg);
+      // bias of this warp's columns (BN / 2 floats, one 128-byte line per 32) brought into L1
+      // while the accumulator is still being produced; the chunks then read it with
+      // broadcast vector loads
+      if ((EPI == EPI_STORE || EPI == EPI_BIAS_GELU) && p.bias && lane < BN / 64 &&
+          n0 + cbeg + 32 * lane < p.N)
+        asm volatile("prefetch.global.L1 [%0];" ::"l"(p.bias + n0 + cbeg + 32 * lane));
       if (!mbar_wait(&tfull_bar[acc], acc_phase, &abort_sh, p.err)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
@@ -617,7 +590,14 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           float* v = reinterpret_cast<float*>(r);
           if (EPI == EPI_DGELU) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(x1[i]);
+            for (int j = 0; j < 32; j += 8) {
+              F8 g8, u8;
+#pragma unroll
+              for (int i = 0; i < 8; ++i) { g8.v[i] = v[j + i]; u8.v[i] = x1[j + i]; }
+              g8 = dgelu8(g8, u8);
+#pragma unroll
+              for (int i = 0; i < 8; ++i) v[j + i] = g8.v[i];
+            }
             store_chunk(&tmC, region, slot_i, p.c_dtype, lane, v, n0 + c0, row0, false);
           } else if (EPI == EPI_RESID) {
 #pragma unroll
@@ -638,19 +618,54 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           if (more && nreg == 1) aux_issue(row0, n0 + c0 + 32);  // after the store has read it
         }
       } else {
-#pragma unroll 1
-        for (int c0 = cbeg; c0 < cend; c0 += 32) {
-          uint32_t r[32];
-          tmem_ld32_issue(tbase + c0, r);
+        // STORE / BIAS_GELU: the TMEM load of chunk i + 1 is in flight while chunk i is
+        // computed and stored; the accumulator is released as soon as its last chunk is in
+        // registers, so the next tile's MMAs need not wait for these stores
+        constexpr int NCH = BN / 64;  // 2 or 4 chunks of 32 columns per warp
+        uint32_t ra[32], rb[32];
+        auto chunk = [&](int ci, uint32_t* r) {
+          const int c0 = cbeg + 32 * ci;
           // chunks entirely right of N or below M are skipped (warp-uniform); partial ones
           // are clipped by the tensor store
-          const bool live_cols = n0 + c0 < p.N && row0 < p.M;
-          EpiIn<EPI> in;
-          if (live_cols && row < p.M) epi_fetch<EPI>(p, row, n0 + c0, in);
-          tmem_wait32(r);
-          float* v = reinterpret_cast<float*>(r);
-          if (live_cols) epi_chunk<EPI>(p, &tmC, &tmC2, staging, slot_i, lane, row0, n0 + c0, v, in, two_slots);
+          if (n0 + c0 < p.N && row0 < p.M) {
+            EpiIn<EPI> in;
+            // (N is a multiple of 8: a group of 8 that starts below N ends below it)
+#pragma unroll
+            for (int g8 = 0; g8 < 4; ++g8) {
+              const int c = n0 + c0 + 8 * g8;
+              float4 b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
+              if (p.bias && c < p.N) {
+                b0 = __ldg(reinterpret_cast<const float4*>(p.bias + c));
+                b1 = __ldg(reinterpret_cast<const float4*>(p.bias + c + 4));
+              }
+              float* b = in.bias + 8 * g8;
+              b[0] = b0.x; b[1] = b0.y; b[2] = b0.z; b[3] = b0.w;
+              b[4] = b1.x; b[5] = b1.y; b[6] = b1.z; b[7] = b1.w;
+            }
+            epi_chunk<EPI>(p, &tmC, &tmC2, staging, slot_i, lane, row0, n0 + c0,
+                           reinterpret_cast<float*>(r), in, two_slots);
+          }
+        };
+        tmem_ld32_issue(tbase + cbeg, ra);
+#pragma unroll 1
+        for (int ci = 0; ci < NCH; ci += 2) {
+          tmem_wait32(ra);
+          tmem_ld32_issue(tbase + cbeg + 32 * (ci + 1), rb);
+          chunk(ci, ra);
+          tmem_wait32(rb);
+          if (ci + 2 < NCH) {
+            tmem_ld32_issue(tbase + cbeg + 32 * (ci + 2), ra);
+          } else {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+          }
+          chunk(ci + 1, rb);
         }
+      }
+      if (EPI == EPI_STORE || EPI == EPI_BIAS_GELU) {  // released above
+        if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+        continue;
       }
       tc_fence_before();
       __syncwarp();
