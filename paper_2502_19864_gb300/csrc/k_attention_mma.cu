@@ -92,6 +92,38 @@ __device__ __forceinline__ void load_tile(bf16* dst, const bf16* qkv, int ld_qkv
   }
 }
 
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(gmem), "r"(valid ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* smem, const void* gmem, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(d), "l"(gmem), "r"(valid ? 4 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Stages rows [r0, r0 + n) of a bf16 [T, ld] matrix at column col0 (DH columns) into a
+// [n][DH + 8] smem tile: with RoPE synchronously through load_tile, otherwise as cp.async
+// copies (rows >= S zero-filled) that the caller commits and waits for.
+template <int DH>
+__device__ __forceinline__ void stage_tile(bf16* dst, const bf16* src, int ld, int b, int S, int r0,
+                                           int n, int col0, bool rope, float theta) {
+  if (rope) {
+    load_tile<DH>(dst, src, ld, b, S, r0, n, col0, true, theta);
+    return;
+  }
+  constexpr int LD = DH + 8;
+  for (int e = threadIdx.x; e < n * (DH / 8); e += blockDim.x) {
+    const int r = e / (DH / 8), c = (e % (DH / 8)) * 8, s = r0 + r;
+    const bool ok = s < S;
+    cp_async16(dst + r * LD + c, src + (size_t)(b * S + (ok ? s : 0)) * ld + col0 + c, ok);
+  }
+}
+
 // transpose of the RoPE rotation on accumulator registers: acc[nt][.] holds columns
 // nt*8 + 2t (+1) of rows g (c0, c1) and g + 8 (c2, c3); the pair partner of column d < DH/2
 // is d + DH/2, i.e. n-tile nt + DH/16 of the same thread.
@@ -117,15 +149,15 @@ __device__ __forceinline__ void rope_bwd_acc(float (&acc)[DH / 8][4], int s0, in
 }
 
 // ---------------------------------------------------------------------------------------
-// forward: CTA = 64 queries of one (b, head), 4 warps x 16 query rows, 64-key blocks
+// forward: CTA = 64 queries of one (b, head), 4 warps x 16 query rows, 64-key blocks that
+// stream through a two-stage ring (block j + 1 is copied while block j is used)
 // ---------------------------------------------------------------------------------------
 template <int DH>
 __global__ void __launch_bounds__(128) attn_fwd_mma_kernel(AttnArgs a) {
   constexpr int LD = DH + 8, NB = 64;
   extern __shared__ __align__(16) uint8_t smraw[];
   bf16* Qs = reinterpret_cast<bf16*>(smraw);
-  bf16* Ks = Qs + 64 * LD;
-  bf16* Vs = Ks + NB * LD;
+  bf16* KV = Qs + 64 * LD;  // [2 stages][K, V][NB][LD]
   const int bh = blockIdx.y, b = bh / a.n_heads, hh = bh % a.n_heads;
   const int H = a.n_heads * DH, ldq = 3 * H;
   const int q0 = blockIdx.x * 64;
@@ -133,24 +165,38 @@ __global__ void __launch_bounds__(128) attn_fwd_mma_kernel(AttnArgs a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
   const float sl2 = a.scale * kLog2e;
 
-  load_tile<DH>(Qs, qkv, ldq, b, a.S, q0, 64, hh * DH, a.rope, a.rope_theta);
-  __syncthreads();
-  uint32_t qf[DH / 16][4];
-#pragma unroll
-  for (int ks = 0; ks < DH / 16; ++ks) frag_a(qf[ks], Qs, LD, warp * 16, ks * 16, lane);
+  const int kend = a.causal ? min(a.S, q0 + 64) : a.S;
+  auto stage_kv = [&](int k0, int st) {
+    bf16* Kd = KV + (size_t)st * 2 * NB * LD;
+    stage_tile<DH>(Kd, qkv, ldq, b, a.S, k0, NB, H + hh * DH, a.rope, a.rope_theta);
+    stage_tile<DH>(Kd + NB * LD, qkv, ldq, b, a.S, k0, NB, 2 * H + hh * DH, false, 0.f);
+  };
+  stage_tile<DH>(Qs, qkv, ldq, b, a.S, q0, 64, hh * DH, a.rope, a.rope_theta);
+  stage_kv(0, 0);
+  cp_async_commit();
 
   const int qr0 = q0 + warp * 16 + g, qr1 = qr0 + 8;
   float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
   float o[DH / 8][4];
 #pragma unroll
   for (int i = 0; i < DH / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  uint32_t qf[DH / 16][4];
 
-  const int kend = a.causal ? min(a.S, q0 + 64) : a.S;
-  for (int k0 = 0; k0 < kend; k0 += NB) {
+  for (int k0 = 0, it = 0; k0 < kend; k0 += NB, ++it) {
+    if (k0 + NB < kend) {
+      stage_kv(k0 + NB, (it + 1) & 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
     __syncthreads();
-    load_tile<DH>(Ks, qkv, ldq, b, a.S, k0, NB, H + hh * DH, a.rope, a.rope_theta);
-    load_tile<DH>(Vs, qkv, ldq, b, a.S, k0, NB, 2 * H + hh * DH, false, 0.f);
-    __syncthreads();
+    if (it == 0) {
+#pragma unroll
+      for (int ks = 0; ks < DH / 16; ++ks) frag_a(qf[ks], Qs, LD, warp * 16, ks * 16, lane);
+    }
+    const bf16* Ks = KV + (size_t)(it & 1) * 2 * NB * LD;
+    const bf16* Vs = Ks + NB * LD;
     float s[NB / 8][4];
 #pragma unroll
     for (int i = 0; i < NB / 8; ++i) s[i][0] = s[i][1] = s[i][2] = s[i][3] = 0.f;
@@ -220,6 +266,7 @@ __global__ void __launch_bounds__(128) attn_fwd_mma_kernel(AttnArgs a) {
         mma16816(o[2 * np + 1], pa, bb[2], bb[3]);
       }
     }
+    __syncthreads();  // this stage is refilled by the next iteration's copies
   }
   bf16* O = reinterpret_cast<bf16*>(a.O);
   const float i0 = l0 > 0.f ? 1.f / l0 : 0.f, i1 = l1 > 0.f ? 1.f / l1 : 0.f;
@@ -237,17 +284,17 @@ __global__ void __launch_bounds__(128) attn_fwd_mma_kernel(AttnArgs a) {
 
 // ---------------------------------------------------------------------------------------
 // backward dK, dV: CTA = 64 keys of one (b, head) (4 warps x 16 keys); query blocks of QB
+// (q, dO, the row log-sum-exp and D) stream through a two-stage ring.  Rows beyond S are
+// zero-filled: their q and dO rows are zero, so they add nothing to dK and dV.
 // ---------------------------------------------------------------------------------------
 template <int DH, int QB>
 __global__ void __launch_bounds__(128) attn_bwd_dkdv_mma_kernel(AttnArgs a) {
   constexpr int LD = DH + 8;
+  constexpr int STAGE = 2 * QB * LD * 2 + 2 * QB * 4;  // bytes: q, dO, L, D of one block
   extern __shared__ __align__(16) uint8_t smraw[];
   bf16* Ks = reinterpret_cast<bf16*>(smraw);
   bf16* Vs = Ks + 64 * LD;
-  bf16* Qs = Vs + 64 * LD;
-  bf16* Ds_ = Qs + QB * LD;  // dO tile
-  float* Ls = reinterpret_cast<float*>(Ds_ + QB * LD);
-  float* Dd = Ls + QB;
+  uint8_t* ring = reinterpret_cast<uint8_t*>(Vs + 64 * LD);
   const int bh = blockIdx.y, b = bh / a.n_heads, hh = bh % a.n_heads;
   const int H = a.n_heads * DH, ldq = 3 * H;
   const int k0 = blockIdx.x * 64;
@@ -256,8 +303,8 @@ __global__ void __launch_bounds__(128) attn_bwd_dkdv_mma_kernel(AttnArgs a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
   const float sl2 = a.scale * kLog2e;
 
-  load_tile<DH>(Ks, qkv, ldq, b, a.S, k0, 64, H + hh * DH, a.rope, a.rope_theta);
-  load_tile<DH>(Vs, qkv, ldq, b, a.S, k0, 64, 2 * H + hh * DH, false, 0.f);
+  stage_tile<DH>(Ks, qkv, ldq, b, a.S, k0, 64, H + hh * DH, a.rope, a.rope_theta);
+  stage_tile<DH>(Vs, qkv, ldq, b, a.S, k0, 64, 2 * H + hh * DH, false, 0.f);
   const int kr0 = k0 + warp * 16 + g, kr1 = kr0 + 8;  // keys of accumulator rows
   float dk[DH / 8][4], dv[DH / 8][4];
 #pragma unroll
@@ -265,22 +312,35 @@ __global__ void __launch_bounds__(128) attn_bwd_dkdv_mma_kernel(AttnArgs a) {
 #pragma unroll
     for (int j = 0; j < 4; ++j) dk[i][j] = dv[i][j] = 0.f;
 
-  const int qstart = a.causal ? (k0 / QB) * QB : 0;
-  for (int q0 = qstart; q0 < a.S; q0 += QB) {
-    __syncthreads();
-    load_tile<DH>(Qs, qkv, ldq, b, a.S, q0, QB, hh * DH, a.rope, a.rope_theta);
-    for (int e = threadIdx.x; e < QB * (DH / 8); e += blockDim.x) {
-      const int r = e / (DH / 8), c = (e % (DH / 8)) * 8, s = q0 + r;
-      uint4 v = make_uint4(0, 0, 0, 0);
-      if (s < a.S) v = *reinterpret_cast<const uint4*>(dO + (size_t)(b * a.S + s) * H + hh * DH + c);
-      *reinterpret_cast<uint4*>(Ds_ + r * LD + c) = v;
-    }
+  auto stage_q = [&](int q0, int st) {
+    uint8_t* base = ring + (size_t)st * STAGE;
+    bf16* Qd = reinterpret_cast<bf16*>(base);
+    stage_tile<DH>(Qd, qkv, ldq, b, a.S, q0, QB, hh * DH, a.rope, a.rope_theta);
+    stage_tile<DH>(Qd + QB * LD, dO, H, b, a.S, q0, QB, hh * DH, false, 0.f);
+    float* Ld = reinterpret_cast<float*>(Qd + 2 * QB * LD);
     for (int e = threadIdx.x; e < QB; e += blockDim.x) {
       const int s = q0 + e;
-      Ls[e] = s < a.S ? a.lse[(size_t)bh * a.S + s] * kLog2e : INFINITY;
-      Dd[e] = s < a.S ? a.Dscratch[(size_t)bh * a.S + s] : 0.f;
+      const bool ok = s < a.S;
+      cp_async4(Ld + e, a.lse + (size_t)bh * a.S + (ok ? s : 0), ok);
+      cp_async4(Ld + QB + e, a.Dscratch + (size_t)bh * a.S + (ok ? s : 0), ok);
+    }
+  };
+  const int qstart = a.causal ? (k0 / QB) * QB : 0;
+  stage_q(qstart, 0);
+  cp_async_commit();
+  for (int q0 = qstart, it = 0; q0 < a.S; q0 += QB, ++it) {
+    if (q0 + QB < a.S) {
+      stage_q(q0 + QB, (it + 1) & 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
     }
     __syncthreads();
+    const bf16* Qs = reinterpret_cast<const bf16*>(ring + (size_t)(it & 1) * STAGE);
+    const bf16* Ds_ = Qs + QB * LD;  // dO tile
+    const float* Ls = reinterpret_cast<const float*>(Qs + 2 * QB * LD);  // natural-log lse
+    const float* Dd = Ls + QB;
     // S^T = K Q^T and dP^T = V dO^T (16 keys x QB queries per warp)
     float st[QB / 8][4], dpt[QB / 8][4];
 #pragma unroll
@@ -309,7 +369,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dkdv_mma_kernel(AttnArgs a) {
 #pragma unroll
       for (int j = 0; j < 2; ++j) {
         const int ql = nt * 8 + 2 * t + j, q = q0 + ql;
-        const float L = Ls[ql], Dv = Dd[ql];
+        const float L = Ls[ql] * kLog2e, Dv = Dd[ql];
         const bool ok0 = kr0 < a.S && (!a.causal || kr0 <= q);
         const bool ok1 = kr1 < a.S && (!a.causal || kr1 <= q);
         const float p0 = ok0 ? exp2f(st[nt][j] * sl2 - L) : 0.f;
@@ -338,6 +398,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dkdv_mma_kernel(AttnArgs a) {
         mma16816(dk[2 * np + 1], da, bq[2], bq[3]);
       }
     }
+    __syncthreads();  // this stage is refilled by the next iteration's copies
   }
 #pragma unroll
   for (int i = 0; i < DH / 8; ++i)
@@ -363,6 +424,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dkdv_mma_kernel(AttnArgs a) {
 
 // ---------------------------------------------------------------------------------------
 // backward dQ: CTA = 64 queries of one (b, head) (4 warps x 16 queries); 64-key blocks
+// streaming through a two-stage ring
 // ---------------------------------------------------------------------------------------
 template <int DH>
 __global__ void __launch_bounds__(128) attn_bwd_dq_mma_kernel(AttnArgs a) {
@@ -370,8 +432,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_mma_kernel(AttnArgs a) {
   extern __shared__ __align__(16) uint8_t smraw[];
   bf16* Qs = reinterpret_cast<bf16*>(smraw);
   bf16* Os = Qs + 64 * LD;   // dO tile
-  bf16* Ks = Os + 64 * LD;
-  bf16* Vs = Ks + NB * LD;
+  bf16* KV = Os + 64 * LD;   // [2 stages][K, V][NB][LD]
   const int bh = blockIdx.y, b = bh / a.n_heads, hh = bh % a.n_heads;
   const int H = a.n_heads * DH, ldq = 3 * H;
   const int q0 = blockIdx.x * 64;
@@ -380,13 +441,16 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_mma_kernel(AttnArgs a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
   const float sl2 = a.scale * kLog2e;
 
-  load_tile<DH>(Qs, qkv, ldq, b, a.S, q0, 64, hh * DH, a.rope, a.rope_theta);
-  for (int e = threadIdx.x; e < 64 * (DH / 8); e += blockDim.x) {
-    const int r = e / (DH / 8), c = (e % (DH / 8)) * 8, s = q0 + r;
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (s < a.S) v = *reinterpret_cast<const uint4*>(dO + (size_t)(b * a.S + s) * H + hh * DH + c);
-    *reinterpret_cast<uint4*>(Os + r * LD + c) = v;
-  }
+  const int kend = a.causal ? min(a.S, q0 + 64) : a.S;
+  auto stage_kv = [&](int k0, int st) {
+    bf16* Kd = KV + (size_t)st * 2 * NB * LD;
+    stage_tile<DH>(Kd, qkv, ldq, b, a.S, k0, NB, H + hh * DH, a.rope, a.rope_theta);
+    stage_tile<DH>(Kd + NB * LD, qkv, ldq, b, a.S, k0, NB, 2 * H + hh * DH, false, 0.f);
+  };
+  stage_tile<DH>(Qs, qkv, ldq, b, a.S, q0, 64, hh * DH, a.rope, a.rope_theta);
+  stage_tile<DH>(Os, dO, H, b, a.S, q0, 64, hh * DH, false, 0.f);
+  stage_kv(0, 0);
+  cp_async_commit();
   const int qr0 = q0 + warp * 16 + g, qr1 = qr0 + 8;
   const float L0 = qr0 < a.S ? a.lse[(size_t)bh * a.S + qr0] * kLog2e : INFINITY;
   const float L1 = qr1 < a.S ? a.lse[(size_t)bh * a.S + qr1] * kLog2e : INFINITY;
@@ -396,12 +460,17 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_mma_kernel(AttnArgs a) {
 #pragma unroll
   for (int i = 0; i < DH / 8; ++i) dq[i][0] = dq[i][1] = dq[i][2] = dq[i][3] = 0.f;
 
-  const int kend = a.causal ? min(a.S, q0 + 64) : a.S;
-  for (int k0 = 0; k0 < kend; k0 += NB) {
+  for (int k0 = 0, it = 0; k0 < kend; k0 += NB, ++it) {
+    if (k0 + NB < kend) {
+      stage_kv(k0 + NB, (it + 1) & 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
     __syncthreads();
-    load_tile<DH>(Ks, qkv, ldq, b, a.S, k0, NB, H + hh * DH, a.rope, a.rope_theta);
-    load_tile<DH>(Vs, qkv, ldq, b, a.S, k0, NB, 2 * H + hh * DH, false, 0.f);
-    __syncthreads();
+    const bf16* Ks = KV + (size_t)(it & 1) * 2 * NB * LD;
+    const bf16* Vs = Ks + NB * LD;
     float s[NB / 8][4], dp[NB / 8][4];
 #pragma unroll
     for (int i = 0; i < NB / 8; ++i)
@@ -448,6 +517,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_mma_kernel(AttnArgs a) {
         mma16816(dq[2 * np + 1], da, bk[2], bk[3]);
       }
     }
+    __syncthreads();  // this stage is refilled by the next iteration's copies
   }
 #pragma unroll
   for (int i = 0; i < DH / 8; ++i)
@@ -466,7 +536,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_mma_kernel(AttnArgs a) {
 template <int DH>
 cudaError_t fwd(const AttnArgs& a, cudaStream_t st) {
   constexpr int LD = DH + 8;
-  const size_t smem = (size_t)3 * 64 * LD * 2;
+  const size_t smem = (size_t)5 * 64 * LD * 2;
   auto k = attn_fwd_mma_kernel<DH>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
@@ -478,7 +548,7 @@ cudaError_t fwd(const AttnArgs& a, cudaStream_t st) {
 template <int DH>
 cudaError_t bwd(const AttnArgs& a, cudaStream_t st) {
   constexpr int LD = DH + 8, QB = DH == 128 ? 32 : 64;
-  const size_t smem1 = (size_t)(128 + 2 * QB) * LD * 2 + 2 * QB * 4;
+  const size_t smem1 = (size_t)128 * LD * 2 + 2 * ((size_t)2 * QB * LD * 2 + 2 * QB * 4);
   auto k1 = attn_bwd_dkdv_mma_kernel<DH, QB>;
   cudaError_t e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
   if (e != cudaSuccess) return e;
@@ -486,7 +556,7 @@ cudaError_t bwd(const AttnArgs& a, cudaStream_t st) {
   note_launch(1);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const size_t smem2 = (size_t)4 * 64 * LD * 2;
+  const size_t smem2 = (size_t)6 * 64 * LD * 2;
   auto k2 = attn_bwd_dq_mma_kernel<DH>;
   e = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
   if (e != cudaSuccess) return e;
