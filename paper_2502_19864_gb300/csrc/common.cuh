@@ -82,6 +82,17 @@ __device__ __forceinline__ float2 gelu2(float2 x) {
   const float2 h = __fmul2_rn(x, f2(0.5f));
   return __ffma2_rn(h, erf2_as7128(__fmul2_rn(x, f2(0.70710678118654752f))), h);
 }
+// GELU(x) and GELU'(x) together (one erf): the same per-component operations as gelu2 and
+// gelu_grad2
+__device__ __forceinline__ void gelu_both2(float2 x, float2& y, float2& dy) {
+  const float2 erf = erf2_as7128(__fmul2_rn(x, f2(0.70710678118654752f)));
+  const float2 h = __fmul2_rn(x, f2(0.5f));
+  y = __ffma2_rn(h, erf, h);
+  const float2 Phi = __ffma2_rn(erf, f2(0.5f), f2(0.5f));
+  const float2 q = __fmul2_rn(__fmul2_rn(x, f2(-0.5f)), x);
+  const float2 ex = make_float2(__expf(q.x), __expf(q.y));
+  dy = __fadd2_rn(Phi, __fmul2_rn(__fmul2_rn(x, ex), f2(0.39894228040143268f)));
+}
 __device__ __forceinline__ float2 gelu_grad2(float2 x) {
   const float2 Phi = __ffma2_rn(erf2_as7128(__fmul2_rn(x, f2(0.70710678118654752f))), f2(0.5f), f2(0.5f));
   const float2 q = __fmul2_rn(__fmul2_rn(x, f2(-0.5f)), x);

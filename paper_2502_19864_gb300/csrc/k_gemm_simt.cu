@@ -38,9 +38,14 @@ __device__ __forceinline__ void epilogue(const GemmArgs& g, int m, int n, float 
       if (g.C) st_dt(g.C, g.c_dtype, (int64_t)m * g.ldc + n, u);
       st_dt(g.C2, g.c2_dtype, (int64_t)m * g.ldc2 + n, gelu_f(u));
     } break;
-    case EPI_DGELU: {
-      float u = ld_dt(g.aux, g.aux_dtype, (int64_t)m * g.ldaux + n);
-      st_dt(g.C, g.c_dtype, (int64_t)m * g.ldc + n, acc * gelu_grad_f(u));
+    case EPI_BIAS_GELU_G: {
+      float u = acc + (g.bias ? g.bias[n] : 0.f);
+      if (g.C) st_dt(g.C, g.c_dtype, (int64_t)m * g.ldc + n, gelu_grad_f(u));
+      st_dt(g.C2, g.c2_dtype, (int64_t)m * g.ldc2 + n, gelu_f(u));
+    } break;
+    case EPI_MUL: {
+      float f = ld_dt(g.aux, g.aux_dtype, (int64_t)m * g.ldaux + n);
+      st_dt(g.C, g.c_dtype, (int64_t)m * g.ldc + n, acc * f);
     } break;
     case EPI_RESID: {
       float r = ld_dt(g.aux, g.aux_dtype, (int64_t)m * g.ldaux + n);

@@ -43,11 +43,11 @@ constexpr int SLOT_BYTES = 4096, NSLOT = 1;
 // epilogues that read a saved operand per output element (GELU', residual, SwiGLU')
 template <int EPI>
 struct EpiTraits {
-  static constexpr bool AUX = EPI == EPI_DGELU || EPI == EPI_RESID || EPI == EPI_DSWIGLU;
+  static constexpr bool AUX = EPI == EPI_MUL || EPI == EPI_RESID || EPI == EPI_DSWIGLU;
 };
 
 // Every epilogue stages through 4 KB per warp, which keeps the full operand ring.  AUX
-// epilogues TMA-load their operand chunk into that area: bf16 GELU' operands use two 2 KB
+// epilogues TMA-load their operand chunk into that area: bf16 factor operands use two 2 KB
 // regions (the next chunk loads while this one computes); 4 KB operands (fp32 residual,
 // packed gate|up) use one region, whose first chunk per tile loads during the main loop.
 template <int BN, bool AUX>
@@ -325,15 +325,20 @@ __device__ __noinline__ F8 gelu8(F8 x) {
   }
   return x;
 }
-// g * GELU'(u) for 8 values, out of line for the same reason
-__device__ __noinline__ F8 dgelu8(F8 g, F8 u) {
+// GELU(u) into x and GELU'(u) into d for 8 values, out of line for the same reason
+struct F8x2 {
+  F8 y, d;
+};
+__device__ __noinline__ F8x2 gelu_both8(F8 x) {
+  F8x2 r;
 #pragma unroll
   for (int i = 0; i < 8; i += 2) {
-    const float2 y = __fmul2_rn(make_float2(g.v[i], g.v[i + 1]), gelu_grad2(make_float2(u.v[i], u.v[i + 1])));
-    g.v[i] = y.x;
-    g.v[i + 1] = y.y;
+    float2 y, d;
+    gelu_both2(make_float2(x.v[i], x.v[i + 1]), y, d);
+    r.y.v[i] = y.x; r.y.v[i + 1] = y.y;
+    r.d.v[i] = d.x; r.d.v[i + 1] = d.y;
   }
-  return g;
+  return r;
 }
 
 // One warp's 32 x 32 chunk of output C of the STORE and BIAS_GELU epilogues: rows row0..,
@@ -362,6 +367,19 @@ __device__ __forceinline__ void epi_chunk(const TcParams& p, const CUtensorMap* 
 #pragma unroll
       for (int i = 0; i < 8; ++i) v[j + i] = x.v[i];
     }
+    store_chunk(tmC2, staging, slot_i, p.c2_dtype, lane, v, n, row0, ts);
+  } else if (EPI == EPI_BIAS_GELU_G) {
+    float d[32];
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) {
+      F8 x;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) x.v[i] = v[j + i];
+      const F8x2 r = gelu_both8(x);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) { v[j + i] = r.y.v[i]; d[j + i] = r.d.v[i]; }
+    }
+    if (p.C) store_chunk(tmC, staging, slot_i, p.c_dtype, lane, d, n, row0, ts);
     store_chunk(tmC2, staging, slot_i, p.c2_dtype, lane, v, n, row0, ts);
   }
 }
@@ -507,7 +525,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     int aux_waited = 0;                    // AUX chunks whose load this warp has waited for
     uint64_t* abar = aux_bar[warp - 2];
     // AUX: TMA load of the operand chunk (rows row0.., output columns n..) into a region
-    const int rbytes = (EPI == EPI_DGELU && p.aux_dtype == DT_BF16) ? SLOT_BYTES / 2 : SLOT_BYTES;
+    const int rbytes = (EPI == EPI_MUL && p.aux_dtype == DT_BF16) ? SLOT_BYTES / 2 : SLOT_BYTES;
     const int nreg = SLOT_BYTES / rbytes;
     auto aux_issue = [&](int row0_, int n_) {
       const int reg = aux_i % nreg;
@@ -539,7 +557,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       // bias of this warp's columns (BN / 2 floats, one 128-byte line per 32) brought into L1
       // while the accumulator is still being produced; the chunks then read it with
       // broadcast vector loads
-      if ((EPI == EPI_STORE || EPI == EPI_BIAS_GELU) && p.bias && lane < BN / 64 &&
+      if ((EPI == EPI_STORE || EPI == EPI_BIAS_GELU || EPI == EPI_BIAS_GELU_G) && p.bias && lane < BN / 64 &&
           n0 + cbeg + 32 * lane < p.N)
         asm volatile("prefetch.global.L1 [%0];" ::"l"(p.bias + n0 + cbeg + 32 * lane));
       if (!mbar_wait(&tfull_bar[acc], acc_phase, &abort_sh, p.err)) break;
@@ -588,15 +606,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           if (more && nreg == 2) aux_issue(row0, n0 + c0 + 32);
           tmem_wait32(r);
           float* v = reinterpret_cast<float*>(r);
-          if (EPI == EPI_DGELU) {
+          if (EPI == EPI_MUL) {
 #pragma unroll
-            for (int j = 0; j < 32; j += 8) {
-              F8 g8, u8;
-#pragma unroll
-              for (int i = 0; i < 8; ++i) { g8.v[i] = v[j + i]; u8.v[i] = x1[j + i]; }
-              g8 = dgelu8(g8, u8);
-#pragma unroll
-              for (int i = 0; i < 8; ++i) v[j + i] = g8.v[i];
+            for (int i = 0; i < 32; i += 2) {
+              const float2 y = __fmul2_rn(make_float2(v[i], v[i + 1]), make_float2(x1[i], x1[i + 1]));
+              v[i] = y.x;
+              v[i + 1] = y.y;
             }
             store_chunk(&tmC, region, slot_i, p.c_dtype, lane, v, n0 + c0, row0, false);
           } else if (EPI == EPI_RESID) {
@@ -663,7 +678,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           chunk(ci + 1, rb);
         }
       }
-      if (EPI == EPI_STORE || EPI == EPI_BIAS_GELU) {  // released above
+      if (EPI == EPI_STORE || EPI == EPI_BIAS_GELU || EPI == EPI_BIAS_GELU_G) {  // released above
         if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
         continue;
       }
@@ -807,7 +822,8 @@ cudaError_t dispatch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorM
   switch (p.epi) {
     case EPI_STORE: return launch<BN, EPI_STORE>(a, b, c, c2, x, p, grid, st);
     case EPI_BIAS_GELU: return launch<BN, EPI_BIAS_GELU>(a, b, c, c2, x, p, grid, st);
-    case EPI_DGELU: return launch<BN, EPI_DGELU>(a, b, c, c2, x, p, grid, st);
+    case EPI_MUL: return launch<BN, EPI_MUL>(a, b, c, c2, x, p, grid, st);
+    case EPI_BIAS_GELU_G: return launch<BN, EPI_BIAS_GELU_G>(a, b, c, c2, x, p, grid, st);
     case EPI_RESID: return launch<BN, EPI_RESID>(a, b, c, c2, x, p, grid, st);
     case EPI_SWIGLU: return launch<BN, EPI_SWIGLU>(a, b, c, c2, x, p, grid, st);
     case EPI_DSWIGLU: return launch<BN, EPI_DSWIGLU>(a, b, c, c2, x, p, grid, st);
@@ -849,7 +865,8 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   if (g.aux && (!aligned16(g.aux) || g.ldaux % 8)) return cudaErrorNotSupported;
   if (g.epi == EPI_SWIGLU && (g.N % 128 || !g.C2)) return cudaErrorNotSupported;
   if (g.epi == EPI_DSWIGLU && g.N % 64) return cudaErrorNotSupported;
-  if (!has_c && g.epi != EPI_BIAS_GELU && g.epi != EPI_SWIGLU) return cudaErrorNotSupported;
+  if (!has_c && g.epi != EPI_BIAS_GELU && g.epi != EPI_BIAS_GELU_G && g.epi != EPI_SWIGLU)
+    return cudaErrorNotSupported;
 
   const int sms = device_sm_count();
   const int m_tiles = (g.M + BM - 1) / BM;
@@ -880,7 +897,7 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   }
   // operand map of the GELU' / residual / SwiGLU' epilogues: [M, N], or the packed
   // [M, 2N] gate|up of SwiGLU' (always bf16)
-  if (g.epi == EPI_DGELU || g.epi == EPI_RESID || g.epi == EPI_DSWIGLU) {
+  if (g.epi == EPI_MUL || g.epi == EPI_RESID || g.epi == EPI_DSWIGLU) {
     if (!g.aux) return cudaErrorNotSupported;
     if (g.epi == EPI_DSWIGLU && g.aux_dtype != DT_BF16) return cudaErrorNotSupported;
     const int64_t xw = g.epi == EPI_DSWIGLU ? 2LL * g.N : g.N;

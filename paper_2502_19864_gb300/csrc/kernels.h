@@ -22,12 +22,14 @@ long long launches_so_far();
 enum EpiKind : int {
   EPI_STORE = 0,     // C = acc (+ bias)
   EPI_BIAS_GELU,     // C = acc + bias (pre-activation u, optional), C2 = GELU(u)
-  EPI_DGELU,         // C = acc * GELU'(aux)           (aux = saved u)
+  EPI_MUL,           // C = acc * aux                  (aux = GELU'(u) saved by BIAS_GELU_G)
   EPI_RESID,         // C = acc + aux                  (aux = fp32 residual)
   EPI_DSWIGLU,       // N = F: acc is d(h) at col j; aux = packed [gate|up] [M, 2F];
                      // C (width 2F, packed like aux) gets d(gate), d(up)
   EPI_SWIGLU,        // N = 2F packed [gate|up]: C = packed pre-activations (optional),
                      // C2 [M, F] = silu(gate) * up
+  EPI_BIAS_GELU_G,   // u = acc + bias: C = GELU'(u) (optional), C2 = GELU(u) -- the factor the
+                     // backward multiplies by (EPI_MUL), evaluated once in the forward
 };
 
 struct GemmArgs {

@@ -45,7 +45,8 @@ struct LayerWOff {  // offsets into the weights region
 typedef uint16_t bf16_t;  // storage of the bf16 adapter shadows (host side never reads them)
 
 struct SlotOff {  // offsets of one saved-activation slot, relative to the slot base
-  size_t qkv, O, lse, a, zA, xhat1, rstd1, u, f, zF, xhat2, rstd2;  // encoder
+  // encoder (gp: GELU'(u) of the FFN pre-activation u, saved for the backward)
+  size_t qkv, O, lse, a, zA, xhat1, rstd1, gp, f, zF, xhat2, rstd2;
   size_t x_in, x1, gu;                                               // decoder extras
   size_t full_bytes, lowest_bytes, slot_bytes;
 };
@@ -258,7 +259,7 @@ void plan(ra_ctx* c) {
   if (!c->dec) {
     s.xhat1 = sl.take(T * H * es);
     s.rstd1 = sl.take(T * 4);
-    s.u = sl.take(T * F * es);
+    s.gp = sl.take(T * F * es);
     s.f = sl.take(T * H * es);
     s.zF = sl.take(T * m * 4);
     s.xhat2 = sl.take(T * H * es);
@@ -606,7 +607,7 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     float* zA = saved ? (float*)(sb + so.zA) : nullptr;
     void* xhat1 = saved ? sb + so.xhat1 : nullptr;
     float* rstd1 = saved ? (float*)(sb + so.rstd1) : nullptr;
-    void* u = saved ? sb + so.u : nullptr;
+    void* gp = saved ? sb + so.gp : nullptr;
     void* f = saved ? sb + so.f : ctx->ws<char>(ctx->s_f);
     float* zF = saved ? (float*)(sb + so.zF) : nullptr;
     void* xhat2 = saved ? sb + so.xhat2 : nullptr;
@@ -636,7 +637,7 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     ad.y = y1; ad.xhat = xhat1; ad.rstd = rstd1;
     CU(P_adapter_fwd(ctx, ad, st));
     g = gemm_args(ctx, y1, H, ctx->w(o.W1), H, T, F, H);
-    g.epi = EPI_BIAS_GELU; g.C = u; g.ldc = F; g.c_dtype = act; g.bias = ctx->w<float>(o.b1);
+    g.epi = EPI_BIAS_GELU_G; g.C = gp; g.ldc = F; g.c_dtype = act; g.bias = ctx->w<float>(o.b1);
     g.C2 = hbuf; g.ldc2 = F; g.c2_dtype = act;
     CU(P_gemm(ctx, g, st));
     g = gemm_args(ctx, hbuf, F, ctx->w(o.W2), F, T, H, F);
@@ -835,10 +836,10 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       ab.dh = ctx->ws(ctx->b_df); ab.dh_dtype = act;
       ab.dWd = Gl + (size_t)2 * H * m; ab.dWu = Gl + (size_t)3 * H * m;
       CU(P_adapter_bwd(ctx, ab, st));
-      // du = (df W2) * GELU'(u)
+      // du = (df W2) * GELU'(u), the factor saved by the forward's FFN-up epilogue
       GemmArgs g = gemm_args(ctx, ctx->ws(ctx->b_df), H, ctx->w(o.W2T), H, T, F, H);
-      g.epi = EPI_DGELU; g.C = ctx->ws(ctx->b_du); g.ldc = F; g.c_dtype = act;
-      g.aux = sb + so.u; g.ldaux = F; g.aux_dtype = act;
+      g.epi = EPI_MUL; g.C = ctx->ws(ctx->b_du); g.ldc = F; g.c_dtype = act;
+      g.aux = sb + so.gp; g.ldaux = F; g.aux_dtype = act;
       CU(P_gemm(ctx, g, st));
       // dy1 = ds2 + du W1
       float* dy1 = ctx->ws<float>(ctx->b_dy1);
