@@ -316,13 +316,13 @@ int dw_chunks(int T, int H) {
 // Norms
 // ---------------------------------------------------------------------------------------
 template <typename T>
-__global__ void layernorm_bwd_kernel(const float* dy, const void* xhat, const float* rstd,
+__global__ void layernorm_bwd_kernel(const float* dy, const float* dy2, const void* xhat, const float* rstd,
                                      const float* gamma, float* ds, int Tn, int H) {
   int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (t >= Tn) return;
   float s1 = 0.f, s2 = 0.f;
   for (int i = lane; i < H; i += 32) {
-    float gy = dy[(int64_t)t * H + i] * gamma[i];
+    float gy = (dy[(int64_t)t * H + i] + (dy2 ? dy2[(int64_t)t * H + i] : 0.f)) * gamma[i];
     float xh = ldf<T>(xhat, (int64_t)t * H + i);
     s1 += gy;
     s2 += gy * xh;
@@ -331,7 +331,7 @@ __global__ void layernorm_bwd_kernel(const float* dy, const void* xhat, const fl
   s2 = warp_sum(s2) / H;
   float r = rstd[t];
   for (int i = lane; i < H; i += 32) {
-    float gy = dy[(int64_t)t * H + i] * gamma[i];
+    float gy = (dy[(int64_t)t * H + i] + (dy2 ? dy2[(int64_t)t * H + i] : 0.f)) * gamma[i];
     float xh = ldf<T>(xhat, (int64_t)t * H + i);
     ds[(int64_t)t * H + i] = r * (gy - s1 - xh * s2);
   }
@@ -397,8 +397,8 @@ template <> __device__ __forceinline__ void st4<bf16>(void* p, int64_t i, float4
 }
 
 template <typename TX, int V>
-__global__ void __launch_bounds__(256) layernorm_bwd_vec_kernel(const float* dy, const void* xhat,
-    const float* rstd, const float* gamma, float* ds, int Tn, int H) {
+__global__ void __launch_bounds__(256) layernorm_bwd_vec_kernel(const float* dy, const float* dy2,
+    const void* xhat, const float* rstd, const float* gamma, float* ds, int Tn, int H) {
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= Tn) return;
   const int64_t base = (int64_t)row * H;
@@ -407,7 +407,12 @@ __global__ void __launch_bounds__(256) layernorm_bwd_vec_kernel(const float* dy,
 #pragma unroll
   for (int v = 0; v < V; ++v) {
     const int c = (v * 32 + lane) * 4;
-    const float4 d = ld4<float>(dy, base + c), gm = ld4<float>(gamma, c);
+    float4 d = ld4<float>(dy, base + c);
+    if (dy2) {
+      const float4 d2 = ld4<float>(dy2, base + c);
+      d = make_float4(d.x + d2.x, d.y + d2.y, d.z + d2.z, d.w + d2.w);
+    }
+    const float4 gm = ld4<float>(gamma, c);
     g[v] = make_float4(d.x * gm.x, d.y * gm.y, d.z * gm.z, d.w * gm.w);
     x[v] = ld4<TX>(xhat, base + c);
     s1 += g[v].x + g[v].y + g[v].z + g[v].w;
@@ -793,17 +798,17 @@ cudaError_t adapter_bwd(const AdapterBwdArgs& a, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-cudaError_t layernorm_bwd(const float* dy, const void* xhat, const float* rstd,
+cudaError_t layernorm_bwd(const float* dy, const float* dy2, const void* xhat, const float* rstd,
                           const float* gamma, float* ds, int T, int H, int dtype,
                           cudaStream_t st) {
   unsigned grid = blocks_for((int64_t)T * 32, 256);
   if (const int V = row_vec(H)) {
-    if (dtype == DT_BF16) RA_VEC_SWITCH(V, (layernorm_bwd_vec_kernel<bf16, VV><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H)))
-    else RA_VEC_SWITCH(V, (layernorm_bwd_vec_kernel<float, VV><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H)))
+    if (dtype == DT_BF16) RA_VEC_SWITCH(V, (layernorm_bwd_vec_kernel<bf16, VV><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, T, H)))
+    else RA_VEC_SWITCH(V, (layernorm_bwd_vec_kernel<float, VV><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, T, H)))
   } else if (dtype == DT_BF16) {
-    layernorm_bwd_kernel<bf16><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H);
+    layernorm_bwd_kernel<bf16><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, T, H);
   } else {
-    layernorm_bwd_kernel<float><<<grid, 256, 0, st>>>(dy, xhat, rstd, gamma, ds, T, H);
+    layernorm_bwd_kernel<float><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, T, H);
   }
   note_launch(1);
   return cudaGetLastError();

@@ -144,8 +144,9 @@ cudaError_t adapter_dw_reduce(const float* partials, int nchunk, int H, int m, f
                               float* dWu, cudaStream_t st);
 
 // LayerNorm backward with frozen gamma: ds = rstd * (gy - mean(gy) - xhat mean(gy xhat)),
-// gy = dy * gamma.  dy f32, xhat act, ds f32.
-cudaError_t layernorm_bwd(const float* dy, const void* xhat, const float* rstd,
+// gy = (dy + dy2) * gamma.  dy, dy2 (nullable: 0) f32, xhat act, ds f32.  The second input
+// lets a residual-stream gradient join here instead of in the producing GEMM's epilogue.
+cudaError_t layernorm_bwd(const float* dy, const float* dy2, const void* xhat, const float* rstd,
                           const float* gamma, float* ds, int T, int H, int dtype,
                           cudaStream_t st);
 // RMSNorm forward: n = x * rstd * gamma; x given as act (x_act) or f32 (x_f32);

@@ -815,6 +815,9 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
                          ctx->w<float>(ctx->head_rmsf), nullptr, dY, T, H, st);
     }));
   }
+  // encoder: the layer-output gradient arrives as two parts, dY = (dqkv Wqkv) + ds1 of the
+  // layer above; the LayerNorm backward adds them as it loads (null: dY is whole)
+  const float* dY2 = nullptr;
   for (int l = L - 1; l >= k; --l) {
     const LayerWOff& o = ctx->lw[l];
     const bool lowest = l == k;
@@ -827,8 +830,8 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
     ab.partials = ctx->ws<float>(ctx->b_part);
     if (!ctx->dec) {
       float* ds2 = ctx->ws<float>(ctx->b_ds2);
-      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * (8 + dtype_size(act)), st,
-              [&] { return layernorm_bwd(dY, sb + so.xhat2, (float*)(sb + so.rstd2), ctx->w<float>(o.g2), ds2, T, H, act, st); }));
+      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * (8 + dtype_size(act) + (dY2 ? 4 : 0)), st,
+              [&] { return layernorm_bwd(dY, dY2, sb + so.xhat2, (float*)(sb + so.rstd2), ctx->w<float>(o.g2), ds2, T, H, act, st); }));
       // FFN-branch adapter: g = ds2, input f, z_F
       ab.g = ds2; ab.h = sb + so.f; ab.z = (float*)(sb + so.zF);
       ab.WuT = PTl + (size_t)3 * H * m; ab.WdT = PTl + (size_t)2 * H * m;
@@ -841,15 +844,14 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       g.epi = EPI_MUL; g.C = ctx->ws(ctx->b_du); g.ldc = F; g.c_dtype = act;
       g.aux = sb + so.gp; g.ldaux = F; g.aux_dtype = act;
       CU(P_gemm(ctx, g, st));
-      // dy1 = ds2 + du W1
+      // dy1 = ds2 + du W1: the GEMM writes du W1, the LayerNorm backward adds ds2
       float* dy1 = ctx->ws<float>(ctx->b_dy1);
       g = gemm_args(ctx, ctx->ws(ctx->b_du), F, ctx->w(o.W1T), F, T, H, F);
-      g.epi = EPI_RESID; g.C = dy1; g.ldc = H; g.c_dtype = DT_F32;
-      g.aux = ds2; g.ldaux = H; g.aux_dtype = DT_F32;
+      g.C = dy1; g.ldc = H; g.c_dtype = DT_F32;
       CU(P_gemm(ctx, g, st));
       float* ds1 = ctx->ws<float>(ctx->b_ds1);
-      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * (8 + dtype_size(act)), st,
-              [&] { return layernorm_bwd(dy1, sb + so.xhat1, (float*)(sb + so.rstd1), ctx->w<float>(o.g1), ds1, T, H, act, st); }));
+      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * (12 + dtype_size(act)), st,
+              [&] { return layernorm_bwd(dy1, ds2, sb + so.xhat1, (float*)(sb + so.rstd1), ctx->w<float>(o.g1), ds1, T, H, act, st); }));
       // attention-branch adapter
       ab.g = ds1; ab.h = sb + so.a; ab.z = (float*)(sb + so.zA);
       ab.WuT = PTl + (size_t)H * m; ab.WdT = PTl;
@@ -867,10 +869,12 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       at.lse = (float*)(sb + so.lse); at.dO = ctx->ws(ctx->b_dO); at.Dscratch = ctx->ws<float>(ctx->b_D);
       at.dqkv = ctx->ws(ctx->b_dqkv); at.err = ctx->ws<unsigned>(ctx->ws_err);
       CU(P_attn_bwd(ctx, at, st));
+      // dX = ds1 + dqkv Wqkv: the GEMM writes dqkv Wqkv; the next layer's LayerNorm backward
+      // adds ds1
       g = gemm_args(ctx, ctx->ws(ctx->b_dqkv), 3 * H, ctx->w(o.WqkvT), 3 * H, T, H, 3 * H);
-      g.epi = EPI_RESID; g.C = dX; g.ldc = H; g.c_dtype = DT_F32;
-      g.aux = ds1; g.ldaux = H; g.aux_dtype = DT_F32;
+      g.C = dX; g.ldc = H; g.c_dtype = DT_F32;
       CU(P_gemm(ctx, g, st));
+      dY2 = ds1;
     } else {
       // FFN-branch adapter: g = dY (= d x2), input f, z_F
       ab.g = dY; ab.h = sb + so.f; ab.z = (float*)(sb + so.zF);
