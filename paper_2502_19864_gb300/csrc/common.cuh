@@ -105,6 +105,15 @@ __device__ __forceinline__ float silu_grad_f(float x) {
   return s * (1.0f + x * (1.0f - s));
 }
 
+// ---- programmatic dependent launch ----------------------------------------------------
+// A kernel started with launch_pdl may begin while the kernel before it in the stream is
+// still finishing.  pdl_wait() blocks until that kernel has completed and its writes are
+// visible; it precedes every access to memory that earlier kernels write or read.
+// pdl_trigger() lets the next kernel of the stream be scheduled (its CTAs then wait in their
+// own pdl_wait).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ---- error word written by kernels whose bounded waits ran out -------------------------
 // Bit 0: a wait timed out.  The host reads and clears it in ra_sync_status.
 enum : unsigned { RA_DEVERR_TIMEOUT = 1u, RA_DEVERR_BOUNDS = 2u };

@@ -202,6 +202,8 @@ __host__ __device__ constexpr int size_class(int H) { return H <= 768 ? 0 : H <=
 template <int MB, bool DEC, int SZ>
 __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
   extern __shared__ __align__(16) uint8_t sm[];
+  pdl_wait();
+  pdl_trigger();
   const int H = p.H, W = H / COLS_PER_WARP;
   const int KS = phase1_slice(H, MB), W1 = H / KS;
   const int lda = H + 8, lds = MB + 8;
@@ -361,6 +363,8 @@ struct BwdArgs {
 template <int MB, int SZ>
 __global__ void RA_ROWS_BOUNDS(SZ) adapter_bwd_rows_mma_kernel(BwdArgs p) {
   extern __shared__ __align__(16) uint8_t sm[];
+  pdl_wait();
+  pdl_trigger();
   const int H = p.H;
   const int KS = phase1_slice(H, MB), W1 = H / KS;
   const int ldg = H + 8, lds = MB + 8;
@@ -425,6 +429,8 @@ constexpr int DWC = 64, DWR = 32;
 
 template <int MB>
 __global__ void __launch_bounds__(256) adapter_dw_mma_kernel(DwArgs p) {
+  pdl_wait();
+  pdl_trigger();
   // 4 warps per output matrix: with m >= 64 each owns m/64 tiles of 16 bottleneck rows and
   // all 64 columns; with m = 32 each owns one 16-row tile and one 32-column half
   constexpr int LDJ = MB + 8, LDI = DWC + 8;
@@ -544,9 +550,9 @@ cudaError_t launch_fwd(FwdArgs p, cudaStream_t st) {
          : sz == 1 ? adapter_fwd_mma_kernel<MB, DEC, 1> : adapter_fwd_mma_kernel<MB, DEC, 2>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k<<<(p.T + R - 1) / R, (p.H / COLS_PER_WARP) * 32, smem, st>>>(p);
+  e = launch_pdl(k, dim3((p.T + R - 1) / R), dim3((p.H / COLS_PER_WARP) * 32), smem, st, p);
   note_launch(1);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 template <int MB>
@@ -557,9 +563,9 @@ cudaError_t launch_bwd(const BwdArgs& p, cudaStream_t st) {
          : sz == 1 ? adapter_bwd_rows_mma_kernel<MB, 1> : adapter_bwd_rows_mma_kernel<MB, 2>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k<<<(p.T + R - 1) / R, (p.H / COLS_PER_WARP) * 32, smem, st>>>(p);
+  e = launch_pdl(k, dim3((p.T + R - 1) / R), dim3((p.H / COLS_PER_WARP) * 32), smem, st, p);
   note_launch(1);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace
@@ -609,11 +615,11 @@ cudaError_t adapter_bwd_mma(const AdapterBwdArgs& a, const void* Wu_b, const voi
   const int nchunk = adapter_dw_chunks(a.T, a.H);
   d.chunk = (a.T + nchunk - 1) / nchunk;
   dim3 grid(a.H / DWC, nchunk);
-  if (a.m == 32) adapter_dw_mma_kernel<32><<<grid, 256, 0, st>>>(d);
-  else if (a.m == 64) adapter_dw_mma_kernel<64><<<grid, 256, 0, st>>>(d);
-  else adapter_dw_mma_kernel<128><<<grid, 256, 0, st>>>(d);
+  if (a.m == 32) e = launch_pdl(adapter_dw_mma_kernel<32>, grid, dim3(256), (size_t)0, st, d);
+  else if (a.m == 64) e = launch_pdl(adapter_dw_mma_kernel<64>, grid, dim3(256), (size_t)0, st, d);
+  else e = launch_pdl(adapter_dw_mma_kernel<128>, grid, dim3(256), (size_t)0, st, d);
   note_launch(1);
-  e = cudaGetLastError();
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   return adapter_dw_reduce(a.partials, nchunk, a.H, a.m, a.dWd, a.dWu, st);
 }

@@ -128,6 +128,8 @@ __global__ void __launch_bounds__(256) attn_fwd_kernel(AttnArgs a) {
 // D[b, h, s] = sum_d dO * O  (one warp per (token, head))
 template <typename T>
 __global__ void attn_bwd_pre_kernel(AttnArgs a) {
+  pdl_wait();
+  pdl_trigger();
   int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   int T_ = a.B * a.S;
   if (gw >= T_ * a.n_heads) return;
@@ -334,8 +336,10 @@ template <typename T>
 cudaError_t bwd_impl(const AttnArgs& a, cudaStream_t st) {
   int T_ = a.B * a.S;
   int64_t warps = (int64_t)T_ * a.n_heads;
-  attn_bwd_pre_kernel<T><<<(unsigned)((warps * 32 + 255) / 256), 256, 0, st>>>(a);
+  cudaError_t le = launch_pdl(attn_bwd_pre_kernel<T>, dim3((unsigned)((warps * 32 + 255) / 256)), dim3(256),
+                              (size_t)0, st, a);
   note_launch(1);
+  if (le != cudaSuccess) return le;
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (attention_mma_ok(a)) return attention_bwd_mma(a, st);

@@ -164,6 +164,8 @@ __global__ void __launch_bounds__(128) attn_fwd_mma_kernel(AttnArgs a) {
   const bf16* qkv = reinterpret_cast<const bf16*>(a.qkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
   const float sl2 = a.scale * kLog2e;
+  pdl_wait();
+  pdl_trigger();
 
   const int kend = a.causal ? min(a.S, q0 + 64) : a.S;
   auto stage_kv = [&](int k0, int st) {
@@ -302,6 +304,8 @@ __global__ void __launch_bounds__(128) attn_bwd_dkdv_mma_kernel(AttnArgs a) {
   const bf16* dO = reinterpret_cast<const bf16*>(a.dO);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
   const float sl2 = a.scale * kLog2e;
+  pdl_wait();
+  pdl_trigger();
 
   stage_tile<DH>(Ks, qkv, ldq, b, a.S, k0, 64, H + hh * DH, a.rope, a.rope_theta);
   stage_tile<DH>(Vs, qkv, ldq, b, a.S, k0, 64, 2 * H + hh * DH, false, 0.f);
@@ -440,6 +444,8 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_mma_kernel(AttnArgs a) {
   const bf16* dO = reinterpret_cast<const bf16*>(a.dO);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
   const float sl2 = a.scale * kLog2e;
+  pdl_wait();
+  pdl_trigger();
 
   const int kend = a.causal ? min(a.S, q0 + 64) : a.S;
   auto stage_kv = [&](int k0, int st) {
@@ -540,9 +546,9 @@ cudaError_t fwd(const AttnArgs& a, cudaStream_t st) {
   auto k = attn_fwd_mma_kernel<DH>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k<<<dim3((a.S + 63) / 64, a.B * a.n_heads), 128, smem, st>>>(a);
+  e = launch_pdl(k, dim3((a.S + 63) / 64, a.B * a.n_heads), dim3(128), smem, st, a);
   note_launch(1);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 template <int DH>
@@ -552,17 +558,17 @@ cudaError_t bwd(const AttnArgs& a, cudaStream_t st) {
   auto k1 = attn_bwd_dkdv_mma_kernel<DH, QB>;
   cudaError_t e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
   if (e != cudaSuccess) return e;
-  k1<<<dim3((a.S + 63) / 64, a.B * a.n_heads), 128, smem1, st>>>(a);
+  e = launch_pdl(k1, dim3((a.S + 63) / 64, a.B * a.n_heads), dim3(128), smem1, st, a);
   note_launch(1);
-  e = cudaGetLastError();
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const size_t smem2 = (size_t)6 * 64 * LD * 2;
   auto k2 = attn_bwd_dq_mma_kernel<DH>;
   e = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
   if (e != cudaSuccess) return e;
-  k2<<<dim3((a.S + 63) / 64, a.B * a.n_heads), 128, smem2, st>>>(a);
+  e = launch_pdl(k2, dim3((a.S + 63) / 64, a.B * a.n_heads), dim3(128), smem2, st, a);
   note_launch(1);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace

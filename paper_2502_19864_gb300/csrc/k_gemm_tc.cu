@@ -448,6 +448,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = tmem_base_sh;
+  // the set-up above overlaps the previous kernel's tail; operands are read only after it
+  pdl_wait();
+  pdl_trigger();
 
   if (warp == 0) {
     // ------------------------------------------------------------------ TMA producer
@@ -810,9 +813,10 @@ cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  gemm_tc_kernel<BN, EPI><<<grid, NTHREADS, TileCfg<BN, EpiTraits<EPI>::AUX>::SMEM, st>>>(a, b, c, c2, x, p);
+  const cudaError_t e = launch_pdl(gemm_tc_kernel<BN, EPI>, dim3(grid), dim3(NTHREADS),
+                                   (size_t)TileCfg<BN, EpiTraits<EPI>::AUX>::SMEM, st, a, b, c, c2, x, p);
   note_launch(1);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 template <int BN>

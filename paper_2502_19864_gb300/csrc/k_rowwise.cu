@@ -287,6 +287,8 @@ __global__ void __launch_bounds__(256) adapter_dw_partial_kernel(AdapterBwdArgs 
 // Fixed-order sum of the partials: dW_up[j][i] and dW_down[i][j].
 __global__ void adapter_dw_reduce_kernel(const float* partials, int nchunk, int H, int m,
                                          float* dWd, float* dWu) {
+  pdl_wait();
+  pdl_trigger();
   int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   int64_t n = (int64_t)H * m;
   if (e >= 2 * n) return;
@@ -399,6 +401,8 @@ template <> __device__ __forceinline__ void st4<bf16>(void* p, int64_t i, float4
 template <typename TX, int V>
 __global__ void __launch_bounds__(256) layernorm_bwd_vec_kernel(const float* dy, const float* dy2,
     const void* xhat, const float* rstd, const float* gamma, float* ds, int Tn, int H) {
+  pdl_wait();
+  pdl_trigger();
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= Tn) return;
   const int64_t base = (int64_t)row * H;
@@ -432,6 +436,8 @@ __global__ void __launch_bounds__(256) layernorm_bwd_vec_kernel(const float* dy,
 template <typename TX, typename TN, int V>
 __global__ void __launch_bounds__(256) rmsnorm_fwd_vec_kernel(const void* x, const float* gamma, float eps,
     void* n, float* rstd, float* xf, int Tn, int H) {
+  pdl_wait();
+  pdl_trigger();
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= Tn) return;
   const int64_t base = (int64_t)row * H;
@@ -456,6 +462,8 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_vec_kernel(const void* x, con
 template <int V>
 __global__ void __launch_bounds__(256) rmsnorm_bwd_vec_kernel(const float* dy, const float* x, const float* rstd,
     const float* gamma, const float* resid, float* dx, int Tn, int H) {
+  pdl_wait();
+  pdl_trigger();
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= Tn) return;
   const int64_t base = (int64_t)row * H;
@@ -764,7 +772,7 @@ int adapter_dw_chunks(int T, int H) { return dw_chunks(T, H); }
 cudaError_t adapter_dw_reduce(const float* partials, int nchunk, int H, int m, float* dWd,
                               float* dWu, cudaStream_t st) {
   int64_t n = 2LL * H * m;
-  adapter_dw_reduce_kernel<<<blocks_for(n, 256), 256, 0, st>>>(partials, nchunk, H, m, dWd, dWu);
+  (void)launch_pdl(adapter_dw_reduce_kernel, dim3(blocks_for(n, 256)), dim3(256), (size_t)0, st, partials, nchunk, H, m, dWd, dWu);
   note_launch(1);
   return cudaGetLastError();
 }
@@ -793,7 +801,7 @@ cudaError_t adapter_bwd(const AdapterBwdArgs& a, cudaStream_t st) {
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   int64_t n = 2LL * a.H * a.m;
-  adapter_dw_reduce_kernel<<<blocks_for(n, 256), 256, 0, st>>>(a.partials, nchunk, a.H, a.m, a.dWd, a.dWu);
+  (void)launch_pdl(adapter_dw_reduce_kernel, dim3(blocks_for(n, 256)), dim3(256), (size_t)0, st, a.partials, nchunk, a.H, a.m, a.dWd, a.dWu);
   note_launch(3);
   return cudaGetLastError();
 }
@@ -803,8 +811,8 @@ cudaError_t layernorm_bwd(const float* dy, const float* dy2, const void* xhat, c
                           cudaStream_t st) {
   unsigned grid = blocks_for((int64_t)T * 32, 256);
   if (const int V = row_vec(H)) {
-    if (dtype == DT_BF16) RA_VEC_SWITCH(V, (layernorm_bwd_vec_kernel<bf16, VV><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, T, H)))
-    else RA_VEC_SWITCH(V, (layernorm_bwd_vec_kernel<float, VV><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, T, H)))
+    if (dtype == DT_BF16) RA_VEC_SWITCH(V, ((void)launch_pdl(layernorm_bwd_vec_kernel<bf16, VV>, dim3(grid), dim3(256), (size_t)0, st, dy, dy2, xhat, rstd, gamma, ds, T, H)))
+    else RA_VEC_SWITCH(V, ((void)launch_pdl(layernorm_bwd_vec_kernel<float, VV>, dim3(grid), dim3(256), (size_t)0, st, dy, dy2, xhat, rstd, gamma, ds, T, H)))
   } else if (dtype == DT_BF16) {
     layernorm_bwd_kernel<bf16><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, T, H);
   } else {
@@ -820,13 +828,13 @@ cudaError_t rmsnorm_fwd(const void* x, int x_dtype, const float* gamma, float ep
   unsigned grid = blocks_for((int64_t)T * 32, 256);
   if (const int V = row_vec(H)) {
     if (x_dtype == DT_BF16 && n_dtype == DT_BF16)
-      RA_VEC_SWITCH(V, (rmsnorm_fwd_vec_kernel<bf16, bf16, VV><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H)))
+      RA_VEC_SWITCH(V, ((void)launch_pdl(rmsnorm_fwd_vec_kernel<bf16, bf16, VV>, dim3(grid), dim3(256), (size_t)0, st, x, gamma, eps, n, rstd, x_f32_out, T, H)))
     else if (x_dtype == DT_F32 && n_dtype == DT_BF16)
-      RA_VEC_SWITCH(V, (rmsnorm_fwd_vec_kernel<float, bf16, VV><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H)))
+      RA_VEC_SWITCH(V, ((void)launch_pdl(rmsnorm_fwd_vec_kernel<float, bf16, VV>, dim3(grid), dim3(256), (size_t)0, st, x, gamma, eps, n, rstd, x_f32_out, T, H)))
     else if (x_dtype == DT_BF16)
-      RA_VEC_SWITCH(V, (rmsnorm_fwd_vec_kernel<bf16, float, VV><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H)))
+      RA_VEC_SWITCH(V, ((void)launch_pdl(rmsnorm_fwd_vec_kernel<bf16, float, VV>, dim3(grid), dim3(256), (size_t)0, st, x, gamma, eps, n, rstd, x_f32_out, T, H)))
     else
-      RA_VEC_SWITCH(V, (rmsnorm_fwd_vec_kernel<float, float, VV><<<grid, 256, 0, st>>>(x, gamma, eps, n, rstd, x_f32_out, T, H)))
+      RA_VEC_SWITCH(V, ((void)launch_pdl(rmsnorm_fwd_vec_kernel<float, float, VV>, dim3(grid), dim3(256), (size_t)0, st, x, gamma, eps, n, rstd, x_f32_out, T, H)))
     note_launch(1);
     return cudaGetLastError();
   }
@@ -845,7 +853,7 @@ cudaError_t rmsnorm_fwd(const void* x, int x_dtype, const float* gamma, float ep
 cudaError_t rmsnorm_bwd(const float* dy, const float* x, const float* rstd, const float* gamma,
                         const float* resid, float* dx, int T, int H, cudaStream_t st) {
   if (const int V = row_vec(H))
-    RA_VEC_SWITCH(V, (rmsnorm_bwd_vec_kernel<VV><<<blocks_for((int64_t)T * 32, 256), 256, 0, st>>>(dy, x, rstd, gamma, resid, dx, T, H)))
+    RA_VEC_SWITCH(V, ((void)launch_pdl(rmsnorm_bwd_vec_kernel<VV>, dim3(blocks_for((int64_t)T * 32, 256)), dim3(256), (size_t)0, st, dy, x, rstd, gamma, resid, dx, T, H)))
   else
     rmsnorm_bwd_kernel<<<blocks_for((int64_t)T * 32, 256), 256, 0, st>>>(dy, x, rstd, gamma, resid, dx, T, H);
   note_launch(1);

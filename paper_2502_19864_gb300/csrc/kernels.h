@@ -11,6 +11,25 @@ enum DType : int { DT_F32 = 0, DT_BF16 = 1 };
 
 inline size_t dtype_size(int dt) { return dt == DT_BF16 ? 2 : 4; }
 
+// Launches kernel k with programmatic stream serialisation: it may start while the previous
+// kernel of the stream finishes, and must call pdl_wait() before touching memory that earlier
+// kernels use.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k, args...);
+}
+
 // Counts kernels launched by this library (process-wide), for launch accounting.
 void note_launch(int n);
 long long launches_so_far();
