@@ -232,6 +232,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 // layout the store map uses: bf16 rows are 64 B under the 64-byte swizzle (16-byte chunk q
 // of row r at q ^ ((r >> 1) & 3)), f32 rows 128 B under the 128-byte swizzle (q ^ (r & 7)).
 // Lanes 0..7 then hit eight different bank groups for every q: no bank conflicts.
+// (Output chunks use stage_half for f32; the 128-byte form serves the f32 operand staging.)
 __device__ __forceinline__ void stage_row(uint8_t* slot, int dt, int lane, const float* x) {
   if (dt == DT_BF16) {
     uint8_t* row = slot + lane * 64;
@@ -283,26 +284,41 @@ __device__ __forceinline__ void unstage_row(const uint8_t* slot, int dt, int lan
   }
 }
 
+// 16 f32 values of this thread's row as one 64-byte row of a 32 x 16 f32 box (the same
+// 64-byte swizzle as a bf16 32-column row)
+__device__ __forceinline__ void stage_half(uint8_t* slot, int lane, const float* x) {
+  uint8_t* row = slot + lane * 64;
+  const int sw = (lane >> 1) & 3;
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+    *reinterpret_cast<float4*>(row + ((q ^ sw) << 4)) = make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3]);
+}
+
 // Stores one 32-row x 32-column chunk (rows row0.., columns col..) of this warp through the
-// staging area and a TMA tensor store.  `slot_i` counts the warp's stores; two_slots: every
-// output of the kernel is bf16, so the area holds two chunks.
+// staging area and TMA tensor stores: bf16 as one 2 KB box, f32 as two 32 x 16 boxes of 2 KB.
+// `slot_i` counts the warp's stores; two_slots: the area holds two 2 KB slots, used in turn,
+// so a box is staged while the previous one is still being read.
 __device__ __forceinline__ void store_chunk(const CUtensorMap* tm, uint8_t* staging, int& slot_i,
                                            int dt, int lane, const float* x, int col, int row0,
                                            bool two_slots) {
-  uint8_t* slot = staging + (two_slots ? (slot_i & 1) * (SLOT_BYTES / 2) : 0);
-  if (lane == 0) {  // the store that last used this slot has read it
-    if (two_slots) bulk_wait_read<1>();
-    else bulk_wait_read<0>();
+#pragma unroll
+  for (int h = 0; h < (dt == DT_BF16 ? 1 : 2); ++h) {
+    uint8_t* slot = staging + (two_slots ? (slot_i & 1) * (SLOT_BYTES / 2) : 0);
+    if (lane == 0) {  // the store that last used this slot has read it
+      if (two_slots) bulk_wait_read<1>();
+      else bulk_wait_read<0>();
+    }
+    __syncwarp();
+    if (dt == DT_BF16) stage_row(slot, dt, lane, x);
+    else stage_half(slot, lane, x + 16 * h);
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(tm, (uint32_t)__cvta_generic_to_shared(slot), col + 16 * h, row0);
+      bulk_commit();
+    }
+    ++slot_i;
   }
-  __syncwarp();
-  stage_row(slot, dt, lane, x);
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-  __syncwarp();
-  if (lane == 0) {
-    tma_store_2d(tm, (uint32_t)__cvta_generic_to_shared(slot), col, row0);
-    bulk_commit();
-  }
-  ++slot_i;
 }
 
 // Bias of one row's 32-column chunk [n, n + 32) (read from registers of the warp).
@@ -519,7 +535,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     const int quad = warp & 3;             // TMEM lanes 32*quad .. 32*quad + 31
     const int half = (warp - 2) >> 2;      // which half of the tile's columns
     uint8_t* staging = smem + STAGES * Cfg::STAGE_BYTES + (warp - 2) * Cfg::WARP_STAGING;
-    const bool two_slots = (!p.C || p.c_dtype == DT_BF16) && (!p.C2 || p.c2_dtype == DT_BF16);
+    const bool two_slots = true;  // every output box is 2 KB
     int slot_i = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
@@ -553,7 +569,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       int mt, nt;
       tile_coords(tile, p.m_tiles, p.n_tiles_n, mt, nt);
       const int m0 = mt * BM, n0 = nt * BN;
-      const int row0 = m0 + quad * 32, row = row0 + lane;
+      const int row0 = m0 + quad * 32;
       const int cbeg = half * (BN / 2), cend = cbeg + BN / 2;
       // the first operand chunk is fetched while the main loop of this tile still runs
       if (EpiTraits<EPI>::AUX && n0 + cbeg < p.N && row0 < p.M) aux_issue(row0, n0 + cbeg);
@@ -767,8 +783,9 @@ struct MapKeyHash {
 
 // Row-major [rows, cols] matrix with leading dimension ld (elements of dtype); box of
 // box_cols x box_rows.  Operand loads (box 64 bf16 columns) use the 128-byte swizzle the
-// MMA descriptors expect; output stores (box 32 columns) use the swizzle whose span is one
-// box row (64 B for bf16, 128 B for f32), matching stage_row.
+// MMA descriptors expect; output stores (32 bf16 or 16 f32 columns: 64-byte rows) and operand
+// loads of the epilogues (32 columns) use the swizzle whose span is one box row, matching
+// stage_row, stage_half and unstage_row.
 bool make_map(CUtensorMap* out, const void* ptr, int64_t rows, int64_t cols, int64_t ld,
               int box_cols, int box_rows, int dtype) {
   static std::mutex mu;
@@ -893,11 +910,14 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   // [M, 2N]; C2 is [M, N] (bias+GELU) or [M, N / 2] (h of the SwiGLU epilogue)
   if (has_c) {
     const int64_t cw = g.epi == EPI_DSWIGLU ? 2LL * g.N : g.N;
-    if (!make_map(&mc, g.C, g.M, cw, g.ldc, 32, 32, g.c_dtype)) return cudaErrorNotSupported;
+    // output boxes: 32 rows x 32 bf16 or x 16 f32 columns (64-byte rows)
+    if (!make_map(&mc, g.C, g.M, cw, g.ldc, g.c_dtype == DT_BF16 ? 32 : 16, 32, g.c_dtype))
+      return cudaErrorNotSupported;
   }
   if (g.C2) {
     const int64_t cw2 = g.epi == EPI_SWIGLU ? g.N / 2 : g.N;
-    if (!make_map(&mc2, g.C2, g.M, cw2, g.ldc2, 32, 32, g.c2_dtype)) return cudaErrorNotSupported;
+    if (!make_map(&mc2, g.C2, g.M, cw2, g.ldc2, g.c2_dtype == DT_BF16 ? 32 : 16, 32, g.c2_dtype))
+      return cudaErrorNotSupported;
   }
   // operand map of the GELU' / residual / SwiGLU' epilogues: [M, N], or the packed
   // [M, 2N] gate|up of SwiGLU' (always bf16)
