@@ -578,6 +578,7 @@ bool attention_mma_ok(const AttnArgs& a) {
 }
 
 cudaError_t attention_fwd_mma(const AttnArgs& a, cudaStream_t st) {
+  if (attention_tc_ok(a)) return attention_fwd_tc(a, st);
   return a.head_dim == 64 ? fwd<64>(a, st) : fwd<128>(a, st);
 }
 

@@ -101,6 +101,9 @@ cudaError_t attention_bwd(const AttnArgs& a, cudaStream_t st);
 bool attention_mma_ok(const AttnArgs& a);
 cudaError_t attention_fwd_mma(const AttnArgs& a, cudaStream_t st);
 cudaError_t attention_bwd_mma(const AttnArgs& a, cudaStream_t st);
+// tcgen05 forward (bf16, head_dim 64, no mask or RoPE, S <= 256)
+bool attention_tc_ok(const AttnArgs& a);
+cudaError_t attention_fwd_tc(const AttnArgs& a, cudaStream_t st);
 
 // ---------------------------------------------------------------------------------------
 // Row-wise fused kernels
