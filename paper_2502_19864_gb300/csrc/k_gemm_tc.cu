@@ -36,7 +36,7 @@ namespace {
 
 using namespace tc;
 
-constexpr int BM = 128, BK = 64, NTHREADS = 320, EPI_WARPS = 8;
+constexpr int BM = 128, BK = 64;
 
 // epilogue staging: 4 KB per warp, one 32 x 32 f32 chunk or two 32 x 32 bf16 chunks (then
 // a second store can be staged while the first is still being read); this keeps the full
@@ -46,6 +46,11 @@ constexpr int SLOT_BYTES = 4096, NSLOT = 1;
 // epilogues that read a saved operand per output element (GELU', residual, SwiGLU')
 template <int EPI>
 struct EpiTraits {
+  // the GELU epilogue evaluates erf per element: 12 epilogue warps (three per TMEM lane
+  // quadrant) for it, 8 for the others (GELU + GELU' needs more registers than 12 warps
+  // leave)
+  static constexpr int WARPS = EPI == EPI_BIAS_GELU ? 12 : 8;
+  static constexpr int THREADS = (2 + WARPS) * 32;
   static constexpr bool AUX = EPI == EPI_MUL || EPI == EPI_RESID || EPI == EPI_DSWIGLU;
 };
 
@@ -53,15 +58,16 @@ struct EpiTraits {
 // epilogues TMA-load their operand chunk into that area: bf16 factor operands use two 2 KB
 // regions (the next chunk loads while this one computes); 4 KB operands (fp32 residual,
 // packed gate|up) use one region, whose first chunk per tile loads during the main loop.
-template <int BN, bool AUX>
+template <int BN, bool AUX, int EW = 8>
 struct TileCfg {
-  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  // the operand ring gives up a stage to the staging of the extra epilogue warps
+  static constexpr int STAGES = BN == 256 ? (EW > 8 ? 3 : 4) : (EW > 8 ? 5 : 6);
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
   static constexpr int WARP_STAGING = NSLOT * SLOT_BYTES;
-  static constexpr int STAGING = EPI_WARPS * WARP_STAGING;
+  static constexpr int STAGING = EW * WARP_STAGING;
   static constexpr int SMEM = STAGES * STAGE_BYTES + STAGING + 1024;  // + alignment slack
 };
 
@@ -288,16 +294,17 @@ __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, 
 
 // ---- the kernel -------------------------------------------------------------------------------
 template <int BN, int EPI>
-__global__ void __launch_bounds__(NTHREADS, 1)
+__global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmC2,
                    const __grid_constant__ CUtensorMap tmX, const TcParams p) {
-  using Cfg = TileCfg<BN, EpiTraits<EPI>::AUX>;
+  constexpr int EW = EpiTraits<EPI>::WARPS;
+  using Cfg = TileCfg<BN, EpiTraits<EPI>::AUX, EW>;
   constexpr int STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES];
   __shared__ __align__(8) uint64_t tfull_bar[2], tempty_bar[2], drain_bar;
-  __shared__ __align__(8) uint64_t aux_bar[EPI_WARPS][2];  // TMA loads of AUX operands
+  __shared__ __align__(8) uint64_t aux_bar[EW][2];  // TMA loads of AUX operands
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_sh;
 
@@ -313,10 +320,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull_bar[a], 1);
-      mbar_init(&tempty_bar[a], EPI_WARPS);
+      mbar_init(&tempty_bar[a], EW);
     }
     mbar_init(&drain_bar, 1);
-    for (int w = 0; w < EPI_WARPS; ++w) {
+    for (int w = 0; w < EW; ++w) {
       mbar_init(&aux_bar[w][0], 1);
       mbar_init(&aux_bar[w][1], 1);
     }
@@ -408,7 +415,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   } else {
     // ------------------------------------------------------------------ epilogue (warps 2..9)
     const int quad = warp & 3;             // TMEM lanes 32*quad .. 32*quad + 31
-    const int half = (warp - 2) >> 2;      // which half of the tile's columns
+    const int half = (warp - 2) >> 2;      // which part of the tile's columns (EW / 4 parts)
+    constexpr int PARTS = EW / 4;
     uint8_t* staging = smem + STAGES * Cfg::STAGE_BYTES + (warp - 2) * Cfg::WARP_STAGING;
     const bool two_slots = true;  // every output box is 2 KB
     int slot_i = 0;
@@ -451,9 +459,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       // bias of this warp's columns (BN / 2 floats, one 128-byte line per 32) brought into L1
       // while the accumulator is still being produced; the chunks then read it with
       // broadcast vector loads
-      if ((EPI == EPI_STORE || EPI == EPI_BIAS_GELU || EPI == EPI_BIAS_GELU_G) && p.bias && lane < BN / 64 &&
-          n0 + cbeg + 32 * lane < p.N)
-        asm volatile("prefetch.global.L1 [%0];" ::"l"(p.bias + n0 + cbeg + 32 * lane));
+      // (STORE / GELU: this warp's chunks are half, half + PARTS, ... of the tile's BN / 32)
+      if ((EPI == EPI_STORE || EPI == EPI_BIAS_GELU || EPI == EPI_BIAS_GELU_G) && p.bias &&
+          half + PARTS * lane < BN / 32 && n0 + 32 * (half + PARTS * lane) < p.N)
+        asm volatile("prefetch.global.L1 [%0];" ::"l"(p.bias + n0 + 32 * (half + PARTS * lane)));
       if (!mbar_wait(&tfull_bar[acc], acc_phase, &abort_sh, p.err)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
@@ -530,10 +539,16 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         // STORE / BIAS_GELU: the TMEM load of chunk i + 1 is in flight while chunk i is
         // computed and stored; the accumulator is released as soon as its last chunk is in
         // registers, so the next tile's MMAs need not wait for these stores
-        constexpr int NCH = BN / 64;  // 2 or 4 chunks of 32 columns per warp
+        // this warp's chunks: tile columns 32 (half + PARTS i), i < nch
+        const int nch = (BN / 32 - half + PARTS - 1) / PARTS;
         uint32_t ra[32], rb[32];
-        auto chunk = [&](int ci, uint32_t* r) {
-          const int c0 = cbeg + 32 * ci;
+        auto col = [&](int i) { return 32 * (half + PARTS * i); };
+        auto release = [&]() {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+        };
+        auto chunk = [&](int c0, uint32_t* r) {
           // chunks entirely right of N or below M are skipped (warp-uniform); partial ones
           // are clipped by the tensor store
           if (n0 + c0 < p.N && row0 < p.M) {
@@ -547,29 +562,27 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                 b0 = __ldg(reinterpret_cast<const float4*>(p.bias + c));
                 b1 = __ldg(reinterpret_cast<const float4*>(p.bias + c + 4));
               }
-              float* b = in.bias + 8 * g8;
-              b[0] = b0.x; b[1] = b0.y; b[2] = b0.z; b[3] = b0.w;
-              b[4] = b1.x; b[5] = b1.y; b[6] = b1.z; b[7] = b1.w;
+              float* bb = in.bias + 8 * g8;
+              bb[0] = b0.x; bb[1] = b0.y; bb[2] = b0.z; bb[3] = b0.w;
+              bb[4] = b1.x; bb[5] = b1.y; bb[6] = b1.z; bb[7] = b1.w;
             }
             epi_chunk<EPI>(p, &tmC, &tmC2, staging, slot_i, lane, row0, n0 + c0,
                            reinterpret_cast<float*>(r), in, two_slots);
           }
         };
-        tmem_ld32_issue(tbase + cbeg, ra);
+        tmem_ld32_issue(tbase + col(0), ra);
 #pragma unroll 1
-        for (int ci = 0; ci < NCH; ci += 2) {
+        for (int i = 0; i < nch; i += 2) {
           tmem_wait32(ra);
-          tmem_ld32_issue(tbase + cbeg + 32 * (ci + 1), rb);
-          chunk(ci, ra);
-          tmem_wait32(rb);
-          if (ci + 2 < NCH) {
-            tmem_ld32_issue(tbase + cbeg + 32 * (ci + 2), ra);
-          } else {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+          if (i + 1 < nch) tmem_ld32_issue(tbase + col(i + 1), rb);
+          else release();
+          chunk(col(i), ra);
+          if (i + 1 < nch) {
+            tmem_wait32(rb);
+            if (i + 2 < nch) tmem_ld32_issue(tbase + col(i + 2), ra);
+            else release();
+            chunk(col(i + 1), rb);
           }
-          chunk(ci + 1, rb);
         }
       }
       if (EPI == EPI_STORE || EPI == EPI_BIAS_GELU || EPI == EPI_BIAS_GELU_G) {  // released above
@@ -701,12 +714,13 @@ cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         TileCfg<BN, EpiTraits<EPI>::AUX>::SMEM);
+                                         TileCfg<BN, EpiTraits<EPI>::AUX, EpiTraits<EPI>::WARPS>::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  const cudaError_t e = launch_pdl(gemm_tc_kernel<BN, EPI>, dim3(grid), dim3(NTHREADS),
-                                   (size_t)TileCfg<BN, EpiTraits<EPI>::AUX>::SMEM, st, a, b, c, c2, x, p);
+  const cudaError_t e = launch_pdl(gemm_tc_kernel<BN, EPI>, dim3(grid), dim3(EpiTraits<EPI>::THREADS),
+                                   (size_t)TileCfg<BN, EpiTraits<EPI>::AUX, EpiTraits<EPI>::WARPS>::SMEM, st,
+                                   a, b, c, c2, x, p);
   note_launch(1);
   return e != cudaSuccess ? e : cudaGetLastError();
 }

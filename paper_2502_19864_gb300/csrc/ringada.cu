@@ -637,7 +637,9 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     ad.y = y1; ad.xhat = xhat1; ad.rstd = rstd1;
     CU(P_adapter_fwd(ctx, ad, st));
     g = gemm_args(ctx, y1, H, ctx->w(o.W1), H, T, F, H);
-    g.epi = EPI_BIAS_GELU_G; g.C = gp; g.ldc = F; g.c_dtype = act; g.bias = ctx->w<float>(o.b1);
+    // saved layers also keep GELU'(u) for the backward; frozen layers need GELU(u) only
+    g.epi = gp ? EPI_BIAS_GELU_G : EPI_BIAS_GELU;
+    g.C = gp; g.ldc = F; g.c_dtype = act; g.bias = ctx->w<float>(o.b1);
     g.C2 = hbuf; g.ldc2 = F; g.c2_dtype = act;
     CU(P_gemm(ctx, g, st));
     g = gemm_args(ctx, hbuf, F, ctx->w(o.W2), F, T, H, F);
