@@ -147,6 +147,38 @@ __global__ void attn_bwd_pre_kernel(AttnArgs a) {
   if (lane == 0) a.Dscratch[((int64_t)b * a.n_heads + hh) * a.S + s] = acc;
 }
 
+// bf16, head_dim 64 or 128: G = head_dim / 8 threads per (token, head), 16-byte loads
+template <int G>
+__global__ void __launch_bounds__(256) attn_bwd_pre_vec_kernel(AttnArgs a) {
+  pdl_wait();
+  pdl_trigger();
+  const int64_t gi = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / G;
+  const int r = threadIdx.x % G;
+  const int T_ = a.B * a.S;
+  // groups past the end stay for the shuffles below (full warps) but touch no memory
+  const bool live = gi < (int64_t)T_ * a.n_heads;
+  const int t = live ? (int)(gi / a.n_heads) : 0, hh = live ? (int)(gi % a.n_heads) : 0;
+  const int b = t / a.S, s = t % a.S;
+  const int dh = 8 * G, H = a.n_heads * dh;
+  const int64_t i = (int64_t)t * H + hh * dh + 8 * r;
+  uint4 o = make_uint4(0, 0, 0, 0), g = o;
+  if (live) {
+    o = __ldg(reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(a.O) + i));
+    g = __ldg(reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(a.dO) + i));
+  }
+  const __nv_bfloat162* o2 = reinterpret_cast<const __nv_bfloat162*>(&o);
+  const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&g);
+  float acc = 0.f;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float2 x = __bfloat1622float2(o2[k]), y = __bfloat1622float2(g2[k]);
+    acc += x.x * y.x + x.y * y.y;
+  }
+#pragma unroll
+  for (int off = G / 2; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  if (live && r == 0) a.Dscratch[((int64_t)b * a.n_heads + hh) * a.S + s] = acc;
+}
+
 // thread-group layout of the backward: 8 threads per key (or query); thread r of a group
 // owns dims r, r+8, r+16, ... so both members of every RoPE pair (d, d + dh/2) stay in it.
 constexpr int GRP = 8;
@@ -336,8 +368,16 @@ template <typename T>
 cudaError_t bwd_impl(const AttnArgs& a, cudaStream_t st) {
   int T_ = a.B * a.S;
   int64_t warps = (int64_t)T_ * a.n_heads;
-  cudaError_t le = launch_pdl(attn_bwd_pre_kernel<T>, dim3((unsigned)((warps * 32 + 255) / 256)), dim3(256),
-                              (size_t)0, st, a);
+  cudaError_t le;
+  if (a.dtype == DT_BF16 && (a.head_dim == 64 || a.head_dim == 128)) {
+    const int G = a.head_dim / 8;
+    const unsigned blocks = (unsigned)((warps * G + 255) / 256);
+    le = G == 8 ? launch_pdl(attn_bwd_pre_vec_kernel<8>, dim3(blocks), dim3(256), (size_t)0, st, a)
+                : launch_pdl(attn_bwd_pre_vec_kernel<16>, dim3(blocks), dim3(256), (size_t)0, st, a);
+  } else {
+    le = launch_pdl(attn_bwd_pre_kernel<T>, dim3((unsigned)((warps * 32 + 255) / 256)), dim3(256),
+                    (size_t)0, st, a);
+  }
   note_launch(1);
   if (le != cudaSuccess) return le;
   cudaError_t e = cudaGetLastError();

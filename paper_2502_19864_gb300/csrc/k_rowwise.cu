@@ -294,8 +294,18 @@ __global__ void adapter_dw_reduce_kernel(const float* partials, int nchunk, int 
   if (e >= 2 * n) return;
   bool up = e < n;
   int64_t idx = up ? e : e - n;  // index into [m][H]
+  const float* src = partials + (up ? 0 : n) + idx;
+  const size_t stride = (size_t)2 * n;
   float s = 0.f;
-  for (int c = 0; c < nchunk; ++c) s += partials[(size_t)c * 2 * n + (up ? 0 : n) + idx];
+  int c = 0;
+  for (; c + 8 <= nchunk; c += 8) {  // eight loads in flight, summed in chunk order
+    float v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = src[(size_t)(c + k) * stride];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) s += v[k];
+  }
+  for (; c < nchunk; ++c) s += src[(size_t)c * stride];
   if (up) dWu[idx] = s;
   else {
     int j = (int)(idx / H), i = (int)(idx % H);
