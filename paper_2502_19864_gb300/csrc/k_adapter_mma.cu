@@ -83,7 +83,8 @@ __device__ __forceinline__ void load_a(uint32_t* a, const bf16* s, int ld, int r
 // slice [kbase, kbase + ks_len) of H, where Bw is [m, H] bf16 in the tiled fragment layout (B
 // fragments read directly, 16 bytes per thread per two k16 steps; the matrix is small and
 // stays in L1/L2).  The m output columns
-// are produced in groups of 8 n-tiles to bound the registers.
+// are produced in groups of 8 n-tiles to bound the registers.  Rows of part are MB + 8 floats
+// apart, so the float2 stores of one half-warp fall in distinct banks.
 template <int MB>
 __device__ __forceinline__ void phase1_store(const bf16* Xs, int ldx, const bf16* Bw, int H,
                                              int kbase, int ks_len, float* part, int lane) {
@@ -109,8 +110,8 @@ __device__ __forceinline__ void phase1_store(const bf16* Xs, int ldx, const bf16
 #pragma unroll
     for (int nt = 0; nt < NTG; ++nt) {
       const int c = ng * 64 + nt * 8 + 2 * t;
-      *reinterpret_cast<float2*>(part + g * MB + c) = make_float2(acc[nt][0], acc[nt][1]);
-      *reinterpret_cast<float2*>(part + (g + 8) * MB + c) = make_float2(acc[nt][2], acc[nt][3]);
+      *reinterpret_cast<float2*>(part + g * (MB + 8) + c) = make_float2(acc[nt][0], acc[nt][1]);
+      *reinterpret_cast<float2*>(part + (g + 8) * (MB + 8) + c) = make_float2(acc[nt][2], acc[nt][3]);
     }
   }
 }
@@ -184,13 +185,22 @@ __device__ __forceinline__ void load_rows_bf16_async(bf16* dst, int ld, const bf
 }
 __device__ __forceinline__ void load_rows_f32_as_bf16(bf16* dst, int ld, const float* src, int t0,
                                                       int T, int H, int R) {
-  const int vec = H / 4;
-  for (int e = threadIdx.x; e < R * vec; e += blockDim.x) {
-    const int r = e / vec, c = (e % vec) * 4;
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (t0 + r < T) v = *reinterpret_cast<const float4*>(src + (size_t)(t0 + r) * H + c);
-    uint2 q = make_uint2(pack2(v.x, v.y), pack2(v.z, v.w));
-    *reinterpret_cast<uint2*>(dst + (size_t)r * ld + c) = q;
+  const int vec = H / 4, n = R * vec, step = blockDim.x;
+  // up to eight 16-byte loads in flight per thread before any conversion
+  for (int e0 = threadIdx.x; e0 < n; e0 += 8 * step) {
+    float4 v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int e = e0 + k * step, r = e / vec, c = (e % vec) * 4;
+      v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (e < n && t0 + r < T) v[k] = __ldg(reinterpret_cast<const float4*>(src + (size_t)(t0 + r) * H + c));
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int e = e0 + k * step, r = e / vec, c = (e % vec) * 4;
+      if (e < n)
+        *reinterpret_cast<uint2*>(dst + (size_t)r * ld + c) = make_uint2(pack2(v[k].x, v[k].y), pack2(v[k].z, v[k].w));
+    }
   }
 }
 
@@ -208,8 +218,8 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
   const int KS = phase1_slice(H, MB), W1 = H / KS;
   const int lda = H + 8, lds = MB + 8;
   bf16* As = reinterpret_cast<bf16*>(sm);                         // [R][H + 8]
-  float* part = reinterpret_cast<float*>(As + (size_t)R * lda);   // [W1][R][MB]
-  bf16* Ss = reinterpret_cast<bf16*>(part + (size_t)W1 * R * MB); // [R][MB + 8]
+  float* part = reinterpret_cast<float*>(As + (size_t)R * lda);         // [W1][R][MB + 8]
+  bf16* Ss = reinterpret_cast<bf16*>(part + (size_t)W1 * R * (MB + 8)); // [R][MB + 8]
   float* stat = reinterpret_cast<float*>(Ss + (size_t)R * lds);   // [W][16]
   float* rowv = stat + W * 16;                                    // [16]
   bf16* Rs = reinterpret_cast<bf16*>(rowv + 16);                  // encoder: [R][H + 8] residual
@@ -223,12 +233,12 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
     load_rows_bf16_async(Rs, lda, reinterpret_cast<const bf16*>(p.resid), t0, p.T, H, R);
   cp_async_wait_all();
   __syncthreads();
-  if (warp < W1) phase1_store<MB>(As, lda, p.WdT, H, warp * KS, KS, part + (size_t)warp * R * MB, lane);
+  if (warp < W1) phase1_store<MB>(As, lda, p.WdT, H, warp * KS, KS, part + (size_t)warp * R * (MB + 8), lane);
   __syncthreads();
   for (int e = threadIdx.x; e < R * MB; e += blockDim.x) {
     const int r = e / MB, j = e % MB;
     float zs = 0.f;
-    for (int w = 0; w < W1; ++w) zs += part[((size_t)w * R + r) * MB + j];
+    for (int w = 0; w < W1; ++w) zs += part[((size_t)w * R + r) * (MB + 8) + j];
     if (p.z && t0 + r < p.T) p.z[(size_t)(t0 + r) * MB + j] = zs;
     Ss[r * lds + j] = __float2bfloat16_rn(gelu_f(zs));
   }
@@ -370,19 +380,19 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_bwd_rows_mma_kernel(BwdArgs p) {
   const int ldg = H + 8, lds = MB + 8;
   bf16* Gs = reinterpret_cast<bf16*>(sm);
   float* part = reinterpret_cast<float*>(Gs + (size_t)R * ldg);
-  bf16* Ds = reinterpret_cast<bf16*>(part + (size_t)W1 * R * MB);
+  bf16* Ds = reinterpret_cast<bf16*>(part + (size_t)W1 * R * (MB + 8));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, t = lane & 3;
   const int t0 = blockIdx.x * R;
 
   load_rows_f32_as_bf16(Gs, ldg, p.g, t0, p.T, H, R);
   __syncthreads();
-  if (warp < W1) phase1_store<MB>(Gs, ldg, p.Wu, H, warp * KS, KS, part + (size_t)warp * R * MB, lane);
+  if (warp < W1) phase1_store<MB>(Gs, ldg, p.Wu, H, warp * KS, KS, part + (size_t)warp * R * (MB + 8), lane);
   __syncthreads();
   for (int e = threadIdx.x; e < R * MB; e += blockDim.x) {
     const int r = e / MB, j = e % MB;
     float ds = 0.f;
-    for (int w = 0; w < W1; ++w) ds += part[((size_t)w * R + r) * MB + j];
+    for (int w = 0; w < W1; ++w) ds += part[((size_t)w * R + r) * (MB + 8) + j];
     float dz = 0.f;
     if (t0 + r < p.T) {
       dz = ds * gelu_grad_f(p.z[(size_t)(t0 + r) * MB + j]);
@@ -537,7 +547,7 @@ __global__ void __launch_bounds__(256) adapter_dw_mma_kernel(DwArgs p) {
 // shared memory of the row kernels; the encoder forward also stages the residual rows
 size_t rows_smem(int H, int m, bool resid_rows = false) {
   const int W = H / COLS_PER_WARP, W1 = H / phase1_slice(H, m);
-  return (size_t)R * (H + 8) * 2 + (size_t)W1 * R * m * 4 + (size_t)R * (m + 8) * 2 + (W * 16 + 16) * 4 +
+  return (size_t)R * (H + 8) * 2 + (size_t)W1 * R * (m + 8) * 4 + (size_t)R * (m + 8) * 2 + (W * 16 + 16) * 4 +
          (resid_rows ? (size_t)R * (H + 8) * 2 : 0);
 }
 
