@@ -52,9 +52,6 @@ __device__ __forceinline__ void cp_async16(void* smem, const void* gmem, bool va
 __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
 }
-__device__ __forceinline__ uint32_t ld_u32(const bf16* p) {
-  return __ldg(reinterpret_cast<const unsigned int*>(p));
-}
 // B fragments of n8 tile `ntile` (rows 8 ntile .. + 7) for the two k16 steps at k0 (a
 // multiple of 32) of a [R, C] bf16 weight in the tiled fragment layout (8 x 32 blocks of 256
 // contiguous elements, each row of a block in fragment order): lane l reads elements
@@ -127,7 +124,6 @@ __host__ __device__ inline int phase1_slice(int H, int m) {
 template <int MB>
 __device__ __forceinline__ void phase2(float (&acc)[8][4], const bf16* Ss, int lds,
                                        const bf16* Bn, int m, int nbase, int lane) {
-  const int g = lane >> 2, t = lane & 3;
 #pragma unroll
   for (int nt = 0; nt < 8; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
 #pragma unroll
@@ -158,20 +154,9 @@ struct FwdArgs {
   float* x_out;           // decoder residual stream out
   bf16* xhat;             // encoder, nullable
   float* rstd;            // nullable
-  bool stage_resid;       // encoder: residual rows staged in shared memory (when they fit)
+  bool stage_gb;          // gamma (and beta) staged in shared memory
 };
 
-// Loads R rows of a bf16 [T, H] matrix into smem (ld = H + 8); rows >= T read as zero.
-__device__ __forceinline__ void load_rows_bf16(bf16* dst, int ld, const bf16* src, int t0, int T,
-                                               int H, int R) {
-  const int vec = H / 8;
-  for (int e = threadIdx.x; e < R * vec; e += blockDim.x) {
-    const int r = e / vec, c = (e % vec) * 8;
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (t0 + r < T) v = *reinterpret_cast<const uint4*>(src + (size_t)(t0 + r) * H + c);
-    *reinterpret_cast<uint4*>(dst + (size_t)r * ld + c) = v;
-  }
-}
 // Issues cp.async copies of R rows of a bf16 [T, H] matrix into smem (ld = H + 8); rows >= T
 // are zero-filled.  The caller waits (cp_async_wait_all) and synchronises.
 __device__ __forceinline__ void load_rows_bf16_async(bf16* dst, int ld, const bf16* src, int t0, int T,
@@ -209,6 +194,49 @@ __device__ __forceinline__ void load_rows_f32_as_bf16(bf16* dst, int ld, const f
 #define RA_ROWS_BOUNDS(SZ) __launch_bounds__((SZ) == 0 ? 384 : (SZ) == 1 ? 512 : 1024, (SZ) == 2 ? 1 : 2)
 __host__ __device__ constexpr int size_class(int H) { return H <= 768 ? 0 : H <= 1024 ? 1 : 2; }
 
+// Shared-memory layout of the forward kernel (byte offsets):
+//   [0, part)       a rows [R][H + 8] bf16; after the norm, the output y of each warp's columns
+//   [part, s)       per-warp partials of z [W1][R][MB + 8] f32; once z is summed (encoder) the
+//                   residual rows [R][H + 8] bf16, then xhat of each warp's columns
+//   [s, stat)       GELU(z) [R][MB + 8] bf16
+//   [stat, gb)      per-warp row statistics [W][16] and the row values [16], f32
+//   [gb, bytes)     gamma (and beta) staged at the start, when they fit without costing a CTA
+struct FwdLayout { int part, s, stat, gb, bytes; };
+__host__ __device__ inline FwdLayout fwd_layout(int H, int m, int gb_floats) {
+  const int W = H / COLS_PER_WARP, W1 = H / phase1_slice(H, m);
+  const int zpart = W1 * R * (m + 8) * 4, rows = R * (H + 8) * 2;
+  FwdLayout L;
+  L.part = rows;
+  L.s = L.part + (zpart > rows ? zpart : rows);
+  L.stat = L.s + R * (m + 8) * 2;
+  L.gb = L.stat + (W * 16 + 16) * 4;
+  L.bytes = L.gb + gb_floats * 4;
+  return L;
+}
+
+// cp.async of the 16 x 64 block of rows [t0, t0 + 16) and this warp's columns [c0, c0 + 64)
+// of a bf16 [T, H] matrix (rows >= T zero-filled); four 16-byte copies per lane
+__device__ __forceinline__ void load_block_async(bf16* dst, int ld, const bf16* src, int t0, int T,
+                                                 int H, int c0, int lane) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int e = lane + 32 * i, r = e >> 3, c = c0 + (e & 7) * 8;
+    const bool ok = t0 + r < T;
+    cp_async16(dst + (size_t)r * ld + c, src + (size_t)(ok ? t0 + r : 0) * H + c, ok);
+  }
+}
+// copies the warp's 16 x 64 block from shared memory to rows [t0, t0 + 16) of a bf16 [T, H]
+// matrix: every store instruction writes four whole 128-byte row segments
+__device__ __forceinline__ void store_block(bf16* dst, int H, const bf16* src, int ld, int t0, int T,
+                                            int c0, int lane) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int e = lane + 32 * i, r = e >> 3, c = c0 + (e & 7) * 8;
+    if (t0 + r < T)
+      *reinterpret_cast<uint4*>(dst + (size_t)(t0 + r) * H + c) = *reinterpret_cast<const uint4*>(src + (size_t)r * ld + c);
+  }
+}
+
 template <int MB, bool DEC, int SZ>
 __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
   extern __shared__ __align__(16) uint8_t sm[];
@@ -217,20 +245,27 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
   const int H = p.H, W = H / COLS_PER_WARP;
   const int KS = phase1_slice(H, MB), W1 = H / KS;
   const int lda = H + 8, lds = MB + 8;
-  bf16* As = reinterpret_cast<bf16*>(sm);                         // [R][H + 8]
-  float* part = reinterpret_cast<float*>(As + (size_t)R * lda);         // [W1][R][MB + 8]
-  bf16* Ss = reinterpret_cast<bf16*>(part + (size_t)W1 * R * (MB + 8)); // [R][MB + 8]
-  float* stat = reinterpret_cast<float*>(Ss + (size_t)R * lds);   // [W][16]
-  float* rowv = stat + W * 16;                                    // [16]
-  bf16* Rs = reinterpret_cast<bf16*>(rowv + 16);                  // encoder: [R][H + 8] residual
+  const FwdLayout L = fwd_layout(H, MB, 0);
+  bf16* As = reinterpret_cast<bf16*>(sm);
+  float* part = reinterpret_cast<float*>(sm + L.part);
+  bf16* Rs = reinterpret_cast<bf16*>(sm + L.part);
+  bf16* Ss = reinterpret_cast<bf16*>(sm + L.s);
+  float* stat = reinterpret_cast<float*>(sm + L.stat);
+  float* rowv = stat + W * 16;
+  float* gbs = reinterpret_cast<float*>(sm + L.gb);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, t = lane & 3;
   const int t0 = blockIdx.x * R;
+  const int nbase = warp * COLS_PER_WARP;
 
-  // the row tile and (encoder) the residual rows are all in flight at once
   load_rows_bf16_async(As, lda, p.a, t0, p.T, H, R);
-  if (!DEC && p.stage_resid)
-    load_rows_bf16_async(Rs, lda, reinterpret_cast<const bf16*>(p.resid), t0, p.T, H, R);
+  if (p.stage_gb) {
+    const int nv = (DEC ? 1 : 2) * (H / 4);
+    for (int e = threadIdx.x; e < nv; e += blockDim.x) {
+      const float* src = e < H / 4 ? p.gamma + 4 * e : p.beta + 4 * (e - H / 4);
+      cp_async16(gbs + 4 * e, src, true);
+    }
+  }
   cp_async_wait_all();
   __syncthreads();
   if (warp < W1) phase1_store<MB>(As, lda, p.WdT, H, warp * KS, KS, part + (size_t)warp * R * (MB + 8), lane);
@@ -243,9 +278,15 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
     Ss[r * lds + j] = __float2bfloat16_rn(gelu_f(zs));
   }
   __syncthreads();
-  const int nbase = warp * COLS_PER_WARP;
+  // encoder: the residual rows of this warp's columns land in the (now free) partial buffer
+  // while phase 2 runs
+  if (!DEC) load_block_async(Rs, lda, reinterpret_cast<const bf16*>(p.resid), t0, p.T, H, nbase, lane);
   float v[8][4];
   phase2<MB>(v, Ss, lds, p.WuT, MB, nbase, lane);
+  if (!DEC) {
+    cp_async_wait_all();
+    __syncwarp();
+  }
   const int rl0 = g, rl1 = g + 8;  // local rows of c0/c1 and c2/c3
   const int r0 = t0 + rl0, r1 = t0 + rl1;
   float s0 = 0.f, s1 = 0.f;
@@ -259,13 +300,9 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
       const float* rs = reinterpret_cast<const float*>(p.resid);
       if (r0 < p.T) q0 = *reinterpret_cast<const float2*>(rs + (size_t)r0 * H + c);
       if (r1 < p.T) q1 = *reinterpret_cast<const float2*>(rs + (size_t)r1 * H + c);
-    } else if (p.stage_resid) {
+    } else {
       q0 = unpack2(*reinterpret_cast<const uint32_t*>(Rs + (size_t)rl0 * lda + c));
       q1 = unpack2(*reinterpret_cast<const uint32_t*>(Rs + (size_t)rl1 * lda + c));
-    } else {
-      const bf16* rs = reinterpret_cast<const bf16*>(p.resid);
-      if (r0 < p.T) q0 = unpack2(*reinterpret_cast<const uint32_t*>(rs + (size_t)r0 * H + c));
-      if (r1 < p.T) q1 = unpack2(*reinterpret_cast<const uint32_t*>(rs + (size_t)r1 * H + c));
     }
     v[nt][0] += a0.x + q0.x; v[nt][1] += a0.y + q0.y;
     v[nt][2] += a1.x + q1.x; v[nt][3] += a1.y + q1.y;
@@ -290,23 +327,21 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
     rowv[threadIdx.x] = s / H;
   }
   __syncthreads();
+  const float* gam = p.stage_gb ? gbs : p.gamma;
   if (DEC) {
     const float rs0 = rsqrtf(rowv[g] + p.eps), rs1 = rsqrtf(rowv[g + 8] + p.eps);
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
       const int c = nbase + nt * 8 + 2 * t;
-      const float2 gm = *reinterpret_cast<const float2*>(p.gamma + c);
-      if (r0 < p.T) {
-        *reinterpret_cast<float2*>(p.x_out + (size_t)r0 * H + c) = make_float2(v[nt][0], v[nt][1]);
-        *reinterpret_cast<uint32_t*>(p.y + (size_t)r0 * H + c) =
-            pack2(v[nt][0] * rs0 * gm.x, v[nt][1] * rs0 * gm.y);
-      }
-      if (r1 < p.T) {
-        *reinterpret_cast<float2*>(p.x_out + (size_t)r1 * H + c) = make_float2(v[nt][2], v[nt][3]);
-        *reinterpret_cast<uint32_t*>(p.y + (size_t)r1 * H + c) =
-            pack2(v[nt][2] * rs1 * gm.x, v[nt][3] * rs1 * gm.y);
-      }
+      const float2 gm = *reinterpret_cast<const float2*>(gam + c);
+      if (r0 < p.T) *reinterpret_cast<float2*>(p.x_out + (size_t)r0 * H + c) = make_float2(v[nt][0], v[nt][1]);
+      if (r1 < p.T) *reinterpret_cast<float2*>(p.x_out + (size_t)r1 * H + c) = make_float2(v[nt][2], v[nt][3]);
+      // y goes through this warp's columns of the a rows (read above by this thread only)
+      *reinterpret_cast<uint32_t*>(As + (size_t)rl0 * lda + c) = pack2(v[nt][0] * rs0 * gm.x, v[nt][1] * rs0 * gm.y);
+      *reinterpret_cast<uint32_t*>(As + (size_t)rl1 * lda + c) = pack2(v[nt][2] * rs1 * gm.x, v[nt][3] * rs1 * gm.y);
     }
+    __syncwarp();
+    store_block(p.y, H, As, lda, t0, p.T, nbase, lane);
     if (p.rstd && warp == 0 && t == 0) {
       if (r0 < p.T) p.rstd[r0] = rs0;
       if (r1 < p.T) p.rstd[r1] = rs1;
@@ -334,22 +369,23 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
     }
     __syncthreads();
     const float rs0 = rowv[g], rs1 = rowv[g + 8];
+    const float* bet = p.stage_gb ? gbs + H : p.beta;
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
       const int c = nbase + nt * 8 + 2 * t;
-      const float2 gm = *reinterpret_cast<const float2*>(p.gamma + c);
-      const float2 bt = *reinterpret_cast<const float2*>(p.beta + c);
+      const float2 gm = *reinterpret_cast<const float2*>(gam + c);
+      const float2 bt = *reinterpret_cast<const float2*>(bet + c);
       const float x00 = v[nt][0] * rs0, x01 = v[nt][1] * rs0;
       const float x10 = v[nt][2] * rs1, x11 = v[nt][3] * rs1;
-      if (r0 < p.T) {
-        *reinterpret_cast<uint32_t*>(p.y + (size_t)r0 * H + c) = pack2(x00 * gm.x + bt.x, x01 * gm.y + bt.y);
-        if (p.xhat) *reinterpret_cast<uint32_t*>(p.xhat + (size_t)r0 * H + c) = pack2(x00, x01);
-      }
-      if (r1 < p.T) {
-        *reinterpret_cast<uint32_t*>(p.y + (size_t)r1 * H + c) = pack2(x10 * gm.x + bt.x, x11 * gm.y + bt.y);
-        if (p.xhat) *reinterpret_cast<uint32_t*>(p.xhat + (size_t)r1 * H + c) = pack2(x10, x11);
-      }
+      // y and xhat go through this warp's columns of the a rows and of the residual rows
+      *reinterpret_cast<uint32_t*>(As + (size_t)rl0 * lda + c) = pack2(x00 * gm.x + bt.x, x01 * gm.y + bt.y);
+      *reinterpret_cast<uint32_t*>(As + (size_t)rl1 * lda + c) = pack2(x10 * gm.x + bt.x, x11 * gm.y + bt.y);
+      *reinterpret_cast<uint32_t*>(Rs + (size_t)rl0 * lda + c) = pack2(x00, x01);
+      *reinterpret_cast<uint32_t*>(Rs + (size_t)rl1 * lda + c) = pack2(x10, x11);
     }
+    __syncwarp();
+    store_block(p.y, H, As, lda, t0, p.T, nbase, lane);
+    if (p.xhat) store_block(p.xhat, H, Rs, lda, t0, p.T, nbase, lane);
     if (p.rstd && warp == 0 && t == 0) {
       if (r0 < p.T) p.rstd[r0] = rs0;
       if (r1 < p.T) p.rstd[r1] = rs1;
@@ -406,18 +442,18 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_bwd_rows_mma_kernel(BwdArgs p) {
   float v[8][4];
   phase2<MB>(v, Ds, lds, p.Wd, MB, nbase, lane);
   const int r0 = t0 + g, r1 = r0 + 8;
+  // dh goes through this warp's columns of the staged g rows, then out in whole row segments
 #pragma unroll
   for (int nt = 0; nt < 8; ++nt) {
     const int c = nbase + nt * 8 + 2 * t;
-    if (r0 < p.T) {
-      const float2 q = *reinterpret_cast<const float2*>(p.g + (size_t)r0 * H + c);
-      *reinterpret_cast<uint32_t*>(p.dh + (size_t)r0 * H + c) = pack2(v[nt][0] + q.x, v[nt][1] + q.y);
-    }
-    if (r1 < p.T) {
-      const float2 q = *reinterpret_cast<const float2*>(p.g + (size_t)r1 * H + c);
-      *reinterpret_cast<uint32_t*>(p.dh + (size_t)r1 * H + c) = pack2(v[nt][2] + q.x, v[nt][3] + q.y);
-    }
+    float2 q0 = make_float2(0.f, 0.f), q1 = make_float2(0.f, 0.f);
+    if (r0 < p.T) q0 = *reinterpret_cast<const float2*>(p.g + (size_t)r0 * H + c);
+    if (r1 < p.T) q1 = *reinterpret_cast<const float2*>(p.g + (size_t)r1 * H + c);
+    *reinterpret_cast<uint32_t*>(Gs + (size_t)g * ldg + c) = pack2(v[nt][0] + q0.x, v[nt][1] + q0.y);
+    *reinterpret_cast<uint32_t*>(Gs + (size_t)(g + 8) * ldg + c) = pack2(v[nt][2] + q1.x, v[nt][3] + q1.y);
   }
+  __syncwarp();
+  store_block(p.dh, H, Gs, ldg, t0, p.T, nbase, lane);
 }
 
 // ---------------------------------------------------------------------------------------
@@ -544,17 +580,35 @@ __global__ void __launch_bounds__(256) adapter_dw_mma_kernel(DwArgs p) {
     }
 }
 
-// shared memory of the row kernels; the encoder forward also stages the residual rows
-size_t rows_smem(int H, int m, bool resid_rows = false) {
+// shared memory of the backward row kernel
+size_t rows_smem(int H, int m) {
   const int W = H / COLS_PER_WARP, W1 = H / phase1_slice(H, m);
-  return (size_t)R * (H + 8) * 2 + (size_t)W1 * R * (m + 8) * 4 + (size_t)R * (m + 8) * 2 + (W * 16 + 16) * 4 +
-         (resid_rows ? (size_t)R * (H + 8) * 2 : 0);
+  return (size_t)R * (H + 8) * 2 + (size_t)W1 * R * (m + 8) * 4 + (size_t)R * (m + 8) * 2 + (W * 16 + 16) * 4;
+}
+
+int smem_per_sm() {
+  static int v = -1;
+  if (v < 0) {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&n, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) == cudaSuccess)
+      v = n;
+    else
+      v = 0;
+  }
+  return v;
 }
 
 template <int MB, bool DEC>
 cudaError_t launch_fwd(FwdArgs p, cudaStream_t st) {
-  p.stage_resid = !DEC && rows_smem(p.H, MB, true) <= 220 * 1024;
-  const size_t smem = rows_smem(p.H, MB, p.stage_resid);
+  // gamma (and beta) go to shared memory when that keeps the CTAs per SM (1 KB reserved each)
+  const int gbf = (DEC ? 1 : 2) * p.H;
+  const size_t s0 = fwd_layout(p.H, MB, 0).bytes, s1 = fwd_layout(p.H, MB, gbf).bytes;
+  const int per_sm = smem_per_sm();
+  const bool aligned = ((uintptr_t)p.gamma & 15) == 0 && (DEC || ((uintptr_t)p.beta & 15) == 0);
+  p.stage_gb = aligned && s1 <= 220 * 1024 && per_sm > 0 &&
+               per_sm / (int)(s1 + 1024) == per_sm / (int)(s0 + 1024);
+  const size_t smem = p.stage_gb ? s1 : s0;
   const int sz = size_class(p.H);
   auto k = sz == 0 ? adapter_fwd_mma_kernel<MB, DEC, 0>
          : sz == 1 ? adapter_fwd_mma_kernel<MB, DEC, 1> : adapter_fwd_mma_kernel<MB, DEC, 2>;
@@ -582,7 +636,7 @@ cudaError_t launch_bwd(const BwdArgs& p, cudaStream_t st) {
 
 bool adapter_mma_ok(int H, int m) {
   return H % 128 == 0 && H <= 2048 && (m == 32 || m == 64 || m == 128) &&
-         rows_smem(H, m) <= 220 * 1024;
+         rows_smem(H, m) <= 220 * 1024 && fwd_layout(H, m, 0).bytes <= 220 * 1024;
 }
 
 cudaError_t adapter_fwd_mma(const AdapterFwdArgs& a, const void* WdT_b, const void* WuT_b,
