@@ -199,7 +199,7 @@ __host__ __device__ constexpr int size_class(int H) { return H <= 768 ? 0 : H <=
 //   [part, s)       per-warp partials of z [W1][R][MB + 8] f32; once z is summed (encoder) the
 //                   residual rows [R][H + 8] bf16, then xhat of each warp's columns
 //   [s, stat)       GELU(z) [R][MB + 8] bf16
-//   [stat, gb)      per-warp row statistics [W][16] and the row values [16], f32
+//   [stat, gb)      per-warp row summaries [W][16] float2
 //   [gb, bytes)     gamma (and beta) staged at the start, when they fit without costing a CTA
 struct FwdLayout { int part, s, stat, gb, bytes; };
 __host__ __device__ inline FwdLayout fwd_layout(int H, int m, int gb_floats) {
@@ -209,7 +209,7 @@ __host__ __device__ inline FwdLayout fwd_layout(int H, int m, int gb_floats) {
   L.part = rows;
   L.s = L.part + (zpart > rows ? zpart : rows);
   L.stat = L.s + R * (m + 8) * 2;
-  L.gb = L.stat + (W * 16 + 16) * 4;
+  L.gb = L.stat + W * 16 * 8;
   L.bytes = L.gb + gb_floats * 4;
   return L;
 }
@@ -250,8 +250,7 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
   float* part = reinterpret_cast<float*>(sm + L.part);
   bf16* Rs = reinterpret_cast<bf16*>(sm + L.part);
   bf16* Ss = reinterpret_cast<bf16*>(sm + L.s);
-  float* stat = reinterpret_cast<float*>(sm + L.stat);
-  float* rowv = stat + W * 16;
+  float2* stat = reinterpret_cast<float2*>(sm + L.stat);
   float* gbs = reinterpret_cast<float*>(sm + L.gb);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, t = lane & 3;
@@ -314,22 +313,61 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
       s1 += v[nt][2] + v[nt][3];
     }
   }
-  // row sums across the quad, then across warps (fixed order)
   s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
   s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
   s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
   s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
-  if (t == 0) { stat[warp * 16 + g] = s0; stat[warp * 16 + g + 8] = s1; }
-  __syncthreads();
-  if (threadIdx.x < 16) {
-    float s = 0.f;
-    for (int w = 0; w < W; ++w) s += stat[w * 16 + threadIdx.x];
-    rowv[threadIdx.x] = s / H;
+  // Row statistics with one barrier.  Each warp publishes a summary of its 64 columns of the
+  // 16 rows; after the barrier lanes 0-15 of every warp merge the W summaries of one row in
+  // warp order (the same order in every warp) and the quads fetch their two rows by shuffle.
+  //   RMSNorm:   the sum of squares;
+  //   LayerNorm: the mean and the centred sum of squares of the 64 columns, merged with the
+  //              pairwise update of Chan, Golub and LeVeque for equal counts,
+  //              M2 = sum_w M2_w + 64 sum_w (mean_w - mean)^2.
+  float mu0 = 0.f, mu1 = 0.f;
+  if (!DEC) {
+    mu0 = s0 * (1.f / COLS_PER_WARP);
+    mu1 = s1 * (1.f / COLS_PER_WARP);
+    s0 = s1 = 0.f;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      const float d0 = v[nt][0] - mu0, d1 = v[nt][1] - mu0, d2 = v[nt][2] - mu1, d3 = v[nt][3] - mu1;
+      s0 += d0 * d0 + d1 * d1;
+      s1 += d2 * d2 + d3 * d3;
+    }
+    s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
+    s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+    s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
+    s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+  }
+  if (t == 0) {
+    stat[warp * 16 + rl0] = make_float2(mu0, s0);
+    stat[warp * 16 + rl1] = make_float2(mu1, s1);
   }
   __syncthreads();
+  float mean = 0.f, rstd = 0.f;
+  if (lane < 16) {
+    if (DEC) {
+      float q = 0.f;
+      for (int w = 0; w < W; ++w) q += stat[w * 16 + lane].y;
+      rstd = rsqrtf(q / H + p.eps);
+    } else {
+      float sm = 0.f;
+      for (int w = 0; w < W; ++w) sm += stat[w * 16 + lane].x;
+      mean = sm / W;
+      float q = 0.f, dd = 0.f;
+      for (int w = 0; w < W; ++w) {
+        const float2 st = stat[w * 16 + lane];
+        const float d = st.x - mean;
+        q += st.y;
+        dd += d * d;
+      }
+      rstd = rsqrtf((q + COLS_PER_WARP * dd) / H + p.eps);
+    }
+  }
+  const float rs0 = __shfl_sync(0xffffffffu, rstd, rl0), rs1 = __shfl_sync(0xffffffffu, rstd, rl1);
   const float* gam = p.stage_gb ? gbs : p.gamma;
   if (DEC) {
-    const float rs0 = rsqrtf(rowv[g] + p.eps), rs1 = rsqrtf(rowv[g + 8] + p.eps);
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
       const int c = nbase + nt * 8 + 2 * t;
@@ -342,41 +380,16 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
     }
     __syncwarp();
     store_block(p.y, H, As, lda, t0, p.T, nbase, lane);
-    if (p.rstd && warp == 0 && t == 0) {
-      if (r0 < p.T) p.rstd[r0] = rs0;
-      if (r1 < p.T) p.rstd[r1] = rs1;
-    }
   } else {
-    const float mu0 = rowv[g], mu1 = rowv[g + 8];
-    float q0 = 0.f, q1 = 0.f;
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-      v[nt][0] -= mu0; v[nt][1] -= mu0; v[nt][2] -= mu1; v[nt][3] -= mu1;
-      q0 += v[nt][0] * v[nt][0] + v[nt][1] * v[nt][1];
-      q1 += v[nt][2] * v[nt][2] + v[nt][3] * v[nt][3];
-    }
-    q0 += __shfl_xor_sync(0xffffffffu, q0, 1);
-    q0 += __shfl_xor_sync(0xffffffffu, q0, 2);
-    q1 += __shfl_xor_sync(0xffffffffu, q1, 1);
-    q1 += __shfl_xor_sync(0xffffffffu, q1, 2);
-    __syncthreads();  // everyone has read rowv
-    if (t == 0) { stat[warp * 16 + g] = q0; stat[warp * 16 + g + 8] = q1; }
-    __syncthreads();
-    if (threadIdx.x < 16) {
-      float s = 0.f;
-      for (int w = 0; w < W; ++w) s += stat[w * 16 + threadIdx.x];
-      rowv[threadIdx.x] = rsqrtf(s / H + p.eps);
-    }
-    __syncthreads();
-    const float rs0 = rowv[g], rs1 = rowv[g + 8];
+    const float m0 = __shfl_sync(0xffffffffu, mean, rl0), m1 = __shfl_sync(0xffffffffu, mean, rl1);
     const float* bet = p.stage_gb ? gbs + H : p.beta;
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
       const int c = nbase + nt * 8 + 2 * t;
       const float2 gm = *reinterpret_cast<const float2*>(gam + c);
       const float2 bt = *reinterpret_cast<const float2*>(bet + c);
-      const float x00 = v[nt][0] * rs0, x01 = v[nt][1] * rs0;
-      const float x10 = v[nt][2] * rs1, x11 = v[nt][3] * rs1;
+      const float x00 = (v[nt][0] - m0) * rs0, x01 = (v[nt][1] - m0) * rs0;
+      const float x10 = (v[nt][2] - m1) * rs1, x11 = (v[nt][3] - m1) * rs1;
       // y and xhat go through this warp's columns of the a rows and of the residual rows
       *reinterpret_cast<uint32_t*>(As + (size_t)rl0 * lda + c) = pack2(x00 * gm.x + bt.x, x01 * gm.y + bt.y);
       *reinterpret_cast<uint32_t*>(As + (size_t)rl1 * lda + c) = pack2(x10 * gm.x + bt.x, x11 * gm.y + bt.y);
@@ -386,10 +399,10 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
     __syncwarp();
     store_block(p.y, H, As, lda, t0, p.T, nbase, lane);
     if (p.xhat) store_block(p.xhat, H, Rs, lda, t0, p.T, nbase, lane);
-    if (p.rstd && warp == 0 && t == 0) {
-      if (r0 < p.T) p.rstd[r0] = rs0;
-      if (r1 < p.T) p.rstd[r1] = rs1;
-    }
+  }
+  if (p.rstd && warp == 0 && t == 0) {
+    if (r0 < p.T) p.rstd[r0] = rs0;
+    if (r1 < p.T) p.rstd[r1] = rs1;
   }
 }
 
