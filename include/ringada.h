@@ -282,9 +282,10 @@ ra_status ra_adapter_backward(const float* g_dev, const float* h_dev, const floa
 size_t ra_adapter_backward_scratch_bytes(int32_t T, int32_t H, int32_t m);
 
 /* Same computation as ra_adapter_backward, for callers that cannot allocate device memory:
- * a caller that is capturing its stream into a CUDA graph (cudaMalloc is not allowed
- * during capture), or a host that passes a kernel only its inputs and outputs and has no
- * allocator to offer.  The paper has no counterpart; this is a deployment variant.
+ * plug-in hosts that hand a kernel only its input and output buffers and expose no
+ * allocator (custom-operator slots of serving runtimes), and loops that forbid allocation
+ * once running, because cudaMalloc can block, synchronise the device or fail at any time.
+ * The paper has no counterpart; this is a deployment variant.
  * Scratch: a fixed 16 MiB device array inside the library (ra_adapter_backward_noalloc_
  * capacity() bytes), held on every GPU that loads the library until the process exits;
  * the call allocates nothing and frees nothing.  Sizes whose scratch need

@@ -1,11 +1,10 @@
 // k_noalloc.cu -- an allocation-free variant of the stand-alone adapter backward.
 //
 // ra_adapter_backward takes a caller-provided scratch buffer.  Some callers cannot provide
-// one: a caller that is in the middle of capturing its stream into a CUDA graph may not
-// call cudaMalloc (allocation is not a stream operation and breaks the capture), and
-// plug-in hosts that hand a kernel only its input and output buffers (custom-op slots of
-// inference servers, real-time loops that forbid allocation after start-up) have no
-// allocator to call.  This variant keeps its scratch in a fixed device array instead.
+// one: plug-in hosts that hand a kernel only its input and output buffers (custom-operator
+// slots of serving runtimes) have no allocator to call, and loops that forbid allocation
+// once running cannot afford cudaMalloc, which can block, synchronise the device or fail
+// at any time.  This variant keeps its scratch in a fixed device array instead.
 #include <cuda_runtime.h>
 
 #include <mutex>

@@ -1,6 +1,6 @@
 """The allocation-free adapter backward (ra_adapter_backward_noalloc), for callers that
-cannot allocate device memory (e.g. while capturing a CUDA graph, or inside a host that
-hands over only inputs and outputs).  Checked through the C ABI against the existing
+cannot allocate device memory: plug-in hosts that hand over only inputs and outputs, and
+loops that forbid allocation once running.  Checked through the C ABI against the existing
 ra_adapter_backward on two calls in a row with different inputs, since the fixed scratch
 array is shared by every call and keeps the previous call's contents.  Named to run last."""
 import numpy as np
