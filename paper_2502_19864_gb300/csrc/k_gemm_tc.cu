@@ -7,8 +7,9 @@
 // step.
 //
 // Structure (one persistent CTA per SM, 320 threads):
-//   warp 0      TMA producer: 128 x 64 A tiles and BN x 64 B tiles (128-byte swizzle) into
-//               a STAGES-deep shared-memory ring, completion tracked by mbarrier tx counts;
+//   warp 0      TMA producer: 128 x 64 A tiles and BN x 64 B tiles (BN = 128, 192 or 256;
+//               128-byte swizzle) into a STAGES-deep shared-memory ring, completion tracked
+//               by mbarrier tx counts;
 //   warp 1      allocates 2*BN TMEM columns (two accumulators); one thread issues
 //               tcgen05.mma (M = 128, N = BN, K = 16) and tcgen05.commit to free each stage
 //               and to publish each finished accumulator;
@@ -60,12 +61,14 @@ struct EpiTraits {
 // packed gate|up) use one region, whose first chunk per tile loads during the main loop.
 template <int BN, bool AUX, int EW = 8>
 struct TileCfg {
-  // the operand ring gives up a stage to the staging of the extra epilogue warps
-  static constexpr int STAGES = BN == 256 ? (EW > 8 ? 3 : 4) : (EW > 8 ? 5 : 6);
+  // the operand ring gives up a stage to the staging of the extra epilogue warps (a
+  // 192-wide ring keeps 4 stages either way: 40 KB stages)
+  static constexpr int STAGES = BN == 256 ? (EW > 8 ? 3 : 4) : BN == 192 ? 4 : (EW > 8 ? 5 : 6);
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int TMEM_COLS = 2 * BN;
+  // two accumulators of BN columns; the allocation is a power of two
+  static constexpr int TMEM_COLS = 2 * BN <= 256 ? 256 : 512;
   static constexpr int WARP_STAGING = NSLOT * SLOT_BYTES;
   static constexpr int STAGING = EW * WARP_STAGING;
   static constexpr int SMEM = STAGES * STAGE_BYTES + STAGING + 1024;  // + alignment slack
@@ -735,8 +738,14 @@ cudaError_t dispatch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorM
     case EPI_MUL: return launch<BN, EPI_MUL>(a, b, c, c2, x, p, grid, st);
     case EPI_BIAS_GELU_G: return launch<BN, EPI_BIAS_GELU_G>(a, b, c, c2, x, p, grid, st);
     case EPI_RESID: return launch<BN, EPI_RESID>(a, b, c, c2, x, p, grid, st);
-    case EPI_SWIGLU: return launch<BN, EPI_SWIGLU>(a, b, c, c2, x, p, grid, st);
-    case EPI_DSWIGLU: return launch<BN, EPI_DSWIGLU>(a, b, c, c2, x, p, grid, st);
+    case EPI_SWIGLU:
+    case EPI_DSWIGLU:
+      // the gate|up epilogues work on 128-column blocks: 128- and 256-wide tiles only
+      if constexpr (BN % 128 == 0) {
+        if (p.epi == EPI_SWIGLU) return launch<BN, EPI_SWIGLU>(a, b, c, c2, x, p, grid, st);
+        return launch<BN, EPI_DSWIGLU>(a, b, c, c2, x, p, grid, st);
+      }
+      break;
   }
   return cudaErrorNotSupported;
 }
@@ -780,14 +789,19 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
 
   const int sms = device_sm_count();
   const int m_tiles = (g.M + BM - 1) / BM;
-  // tile width: fewer waves of 128 x BN tiles, weighting 128-wide tiles by the higher
-  // shared-memory traffic per flop they carry
+  // tile width: fewest waves of 128 x BN tiles (time ~ waves x BN), weighting the narrower
+  // tiles by their measured cost per column: a 128-wide tile carries more shared-memory
+  // operand traffic per flop, and a 192-wide tile takes about as long as a 256-wide one
+  // (measured: 0.96x the time of a 256-wide tile).  So 192 wins only where it saves a
+  // whole wave at equal count, e.g. N = 768 at 4096 rows: 128 tiles in one wave instead of
+  // 96 tiles of 256 columns on a third fewer SMs.
   auto cost = [&](int bn) {
     int tiles = m_tiles * ((g.N + bn - 1) / bn);
     int waves = (tiles + sms - 1) / sms;
-    return (double)waves * bn * (bn == 128 ? 1.15 : 1.0);
+    return (double)waves * bn * (bn == 128 ? 1.15 : bn == 192 ? 1.27 : 1.0);
   };
-  const int BNsel = (g.N <= 128 || cost(128) < cost(256)) ? 128 : 256;
+  int BNsel = (g.N <= 128 || cost(128) < cost(256)) ? 128 : 256;
+  if (g.N > 128 && g.epi != EPI_SWIGLU && g.epi != EPI_DSWIGLU && cost(192) < cost(BNsel)) BNsel = 192;
 
   CUtensorMap ma, mb, mc, mc2, mx;
   memset(&mc, 0, sizeof mc);
@@ -830,6 +844,7 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   p.err = g.err;
   const int grid = p.num_tiles < sms ? p.num_tiles : sms;
   return BNsel == 256 ? dispatch<256>(ma, mb, mc, mc2, mx, p, grid, st)
+       : BNsel == 192 ? dispatch<192>(ma, mb, mc, mc2, mx, p, grid, st)
                       : dispatch<128>(ma, mb, mc, mc2, mx, p, grid, st);
 }
 

@@ -62,9 +62,19 @@ def test_gemm_step_shapes(M, N, K):
     _check(C, ref)
 
 
-def test_gemm_bias_and_gelu_epilogue():
+# shapes whose tiles are 192 columns wide (N = 768 at 4096 rows; a ragged last tile,
+# 760 = 3 x 192 + 184, with ragged rows), and N = 3072 at 8192 rows
+@pytest.mark.parametrize("M,N,K", [(4096, 768, 768), (8192, 3072, 1024), (4000, 760, 200)])
+def test_gemm_192_wide_tiles(M, N, K):
+    C, _, ref = _run(M, N, K)
+    _check(C, ref)
+
+
+# (4096, 768): the bias+GELU epilogue on 192-wide tiles
+@pytest.mark.parametrize("M,N,K", [(520, 384, 256), (4096, 768, 256)])
+def test_gemm_bias_and_gelu_epilogue(M, N, K):
     import torch
-    C, G, ref = _run(520, 384, 256, bias=True, gelu=True)
+    C, G, ref = _run(M, N, K, bias=True, gelu=True)
     _check(C, ref)
     _check(G, torch.nn.functional.gelu(ref), tol=1e-2)
 
