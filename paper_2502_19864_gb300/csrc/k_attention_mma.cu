@@ -149,6 +149,43 @@ __device__ __forceinline__ void rope_bwd_acc(float (&acc)[DH / 8][4], int s0, in
 }
 
 // ---------------------------------------------------------------------------------------
+// RoPE once, in place, on the q and k columns of qkv [T, 3H]: thread = 8 consecutive pair
+// indices i of one (token, head); the 8 angles serve both q and k.  The rotated values are
+// rounded to bf16 exactly as the staging path rounds them.
+// ---------------------------------------------------------------------------------------
+template <int DH>
+__global__ void __launch_bounds__(256) rope_qk_kernel(bf16* qkv, int T, int S, int n_heads, float theta) {
+  pdl_wait();
+  pdl_trigger();
+  constexpr int HALF = DH / 2, G = HALF / 8;
+  const int H = n_heads * DH;
+  const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= (int64_t)T * n_heads * G) return;
+  const int gi = (int)(e % G);
+  const int64_t th = e / G;
+  const int hh = (int)(th % n_heads), tk = (int)(th / n_heads);
+  const int s = tk % S, i0 = gi * 8;
+  float cs[8], sn[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) sincosf((float)s * inv_freq(i0 + j, DH, theta), &sn[j], &cs[j]);
+#pragma unroll
+  for (int part = 0; part < 2; ++part) {
+    bf16* p = qkv + (size_t)tk * 3 * H + (size_t)part * H + (size_t)hh * DH + i0;
+    uint4 u1 = *reinterpret_cast<const uint4*>(p), u2 = *reinterpret_cast<const uint4*>(p + HALF);
+    __nv_bfloat16* x1 = reinterpret_cast<__nv_bfloat16*>(&u1);
+    __nv_bfloat16* x2 = reinterpret_cast<__nv_bfloat16*>(&u2);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float a1 = __bfloat162float(x1[j]), a2 = __bfloat162float(x2[j]);
+      x1[j] = __float2bfloat16_rn(a1 * cs[j] - a2 * sn[j]);
+      x2[j] = __float2bfloat16_rn(a2 * cs[j] + a1 * sn[j]);
+    }
+    *reinterpret_cast<uint4*>(p) = u1;
+    *reinterpret_cast<uint4*>(p + HALF) = u2;
+  }
+}
+
+// ---------------------------------------------------------------------------------------
 // forward: CTA = 64 queries of one (b, head), 4 warps x 16 query rows, 64-key blocks that
 // stream through a two-stage ring (block j + 1 is copied while block j is used)
 // ---------------------------------------------------------------------------------------
@@ -170,10 +207,10 @@ __global__ void __launch_bounds__(128) attn_fwd_mma_kernel(AttnArgs a) {
   const int kend = a.causal ? min(a.S, q0 + 64) : a.S;
   auto stage_kv = [&](int k0, int st) {
     bf16* Kd = KV + (size_t)st * 2 * NB * LD;
-    stage_tile<DH>(Kd, qkv, ldq, b, a.S, k0, NB, H + hh * DH, a.rope, a.rope_theta);
+    stage_tile<DH>(Kd, qkv, ldq, b, a.S, k0, NB, H + hh * DH, a.rope && !a.qk_rotated, a.rope_theta);
     stage_tile<DH>(Kd + NB * LD, qkv, ldq, b, a.S, k0, NB, 2 * H + hh * DH, false, 0.f);
   };
-  stage_tile<DH>(Qs, qkv, ldq, b, a.S, q0, 64, hh * DH, a.rope, a.rope_theta);
+  stage_tile<DH>(Qs, qkv, ldq, b, a.S, q0, 64, hh * DH, a.rope && !a.qk_rotated, a.rope_theta);
   stage_kv(0, 0);
   cp_async_commit();
 
@@ -307,7 +344,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dkdv_mma_kernel(AttnArgs a) {
   pdl_wait();
   pdl_trigger();
 
-  stage_tile<DH>(Ks, qkv, ldq, b, a.S, k0, 64, H + hh * DH, a.rope, a.rope_theta);
+  stage_tile<DH>(Ks, qkv, ldq, b, a.S, k0, 64, H + hh * DH, a.rope && !a.qk_rotated, a.rope_theta);
   stage_tile<DH>(Vs, qkv, ldq, b, a.S, k0, 64, 2 * H + hh * DH, false, 0.f);
   const int kr0 = k0 + warp * 16 + g, kr1 = kr0 + 8;  // keys of accumulator rows
   float dk[DH / 8][4], dv[DH / 8][4];
@@ -319,7 +356,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dkdv_mma_kernel(AttnArgs a) {
   auto stage_q = [&](int q0, int st) {
     uint8_t* base = ring + (size_t)st * STAGE;
     bf16* Qd = reinterpret_cast<bf16*>(base);
-    stage_tile<DH>(Qd, qkv, ldq, b, a.S, q0, QB, hh * DH, a.rope, a.rope_theta);
+    stage_tile<DH>(Qd, qkv, ldq, b, a.S, q0, QB, hh * DH, a.rope && !a.qk_rotated, a.rope_theta);
     stage_tile<DH>(Qd + QB * LD, dO, H, b, a.S, q0, QB, hh * DH, false, 0.f);
     float* Ld = reinterpret_cast<float*>(Qd + 2 * QB * LD);
     for (int e = threadIdx.x; e < QB; e += blockDim.x) {
@@ -450,10 +487,10 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_mma_kernel(AttnArgs a) {
   const int kend = a.causal ? min(a.S, q0 + 64) : a.S;
   auto stage_kv = [&](int k0, int st) {
     bf16* Kd = KV + (size_t)st * 2 * NB * LD;
-    stage_tile<DH>(Kd, qkv, ldq, b, a.S, k0, NB, H + hh * DH, a.rope, a.rope_theta);
+    stage_tile<DH>(Kd, qkv, ldq, b, a.S, k0, NB, H + hh * DH, a.rope && !a.qk_rotated, a.rope_theta);
     stage_tile<DH>(Kd + NB * LD, qkv, ldq, b, a.S, k0, NB, 2 * H + hh * DH, false, 0.f);
   };
-  stage_tile<DH>(Qs, qkv, ldq, b, a.S, q0, 64, hh * DH, a.rope, a.rope_theta);
+  stage_tile<DH>(Qs, qkv, ldq, b, a.S, q0, 64, hh * DH, a.rope && !a.qk_rotated, a.rope_theta);
   stage_tile<DH>(Os, dO, H, b, a.S, q0, 64, hh * DH, false, 0.f);
   stage_kv(0, 0);
   cp_async_commit();
@@ -575,6 +612,19 @@ cudaError_t bwd(const AttnArgs& a, cudaStream_t st) {
 
 bool attention_mma_ok(const AttnArgs& a) {
   return a.dtype == DT_BF16 && (a.head_dim == 64 || a.head_dim == 128);
+}
+
+cudaError_t rope_qk_inplace(const AttnArgs& a, cudaStream_t st) {
+  if (!attention_mma_ok(a) || !a.rope || a.qk_rotated) return cudaErrorInvalidValue;
+  const int T = a.B * a.S;
+  const int64_t n = (int64_t)T * a.n_heads * (a.head_dim / 16);
+  const unsigned blocks = (unsigned)((n + 255) / 256);
+  bf16* qkv = reinterpret_cast<bf16*>(const_cast<void*>(a.qkv));
+  const cudaError_t e = a.head_dim == 64
+      ? launch_pdl(rope_qk_kernel<64>, dim3(blocks), dim3(256), (size_t)0, st, qkv, T, a.S, a.n_heads, a.rope_theta)
+      : launch_pdl(rope_qk_kernel<128>, dim3(blocks), dim3(256), (size_t)0, st, qkv, T, a.S, a.n_heads, a.rope_theta);
+  note_launch(1);
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t attention_fwd_mma(const AttnArgs& a, cudaStream_t st) {

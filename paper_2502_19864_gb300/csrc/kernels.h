@@ -85,6 +85,9 @@ struct AttnArgs {
   int dtype = DT_F32;
   bool causal = false;
   bool rope = false;          // rotate-half RoPE on q and k inside the kernel
+  bool qk_rotated = false;    // q and k in qkv already carry the rotation (rope_qk_inplace):
+                              // the kernels stage them as they are, and the backward only
+                              // applies the rotation's transpose to dq and dk
   float rope_theta = 10000.f;
   float scale = 1.f;
   void* O = nullptr;          // [T, H]
@@ -99,6 +102,10 @@ cudaError_t attention_fwd(const AttnArgs& a, cudaStream_t st);
 cudaError_t attention_bwd(const AttnArgs& a, cudaStream_t st);
 // tensor-core versions (bf16, head_dim 64 or 128); the backward expects D in a.Dscratch
 bool attention_mma_ok(const AttnArgs& a);
+// Rotates the q and k columns of a.qkv (bf16, head_dim 64 or 128) in place with RoPE
+// (rotate-half pairs (i, i + dh/2), angle s * theta^(-2i/dh)), once per forward, so that
+// every query block of the attention kernels can stage them with plain copies.
+cudaError_t rope_qk_inplace(const AttnArgs& a, cudaStream_t st);
 cudaError_t attention_fwd_mma(const AttnArgs& a, cudaStream_t st);
 cudaError_t attention_bwd_mma(const AttnArgs& a, cudaStream_t st);
 // tcgen05 forward (bf16, head_dim 64, no mask or RoPE, S <= 256)

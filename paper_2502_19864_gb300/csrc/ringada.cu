@@ -717,6 +717,12 @@ ra_status decoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     at.dtype = act; at.causal = true; at.rope = true; at.rope_theta = ctx->cfg.rope_theta;
     at.scale = 1.f / sqrtf((float)ctx->dh); at.O = O; at.lse = lse;
     at.err = ctx->ws<unsigned>(ctx->ws_err);
+    if (attention_mma_ok(at)) {
+      // q and k rotated once, in place (the saved qkv of this layer then holds them rotated)
+      CU(prof(ctx, RA_PROF_ATTN_FWD, 0, (double)T * 2 * H * 2 * esz(act), st,
+              [&] { return rope_qk_inplace(at, st); }));
+      at.qk_rotated = true;
+    }
     CU(P_attn_fwd(ctx, at, st));
     g = gemm_args(ctx, O, H, ctx->w(o.Wo), H, T, H, H);
     g.C = a; g.ldc = H; g.c_dtype = act;
@@ -910,6 +916,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       AttnArgs at;
       at.qkv = sb + so.qkv; at.B = B; at.S = S; at.n_heads = ctx->nh; at.head_dim = ctx->dh;
       at.dtype = act; at.causal = true; at.rope = true; at.rope_theta = ctx->cfg.rope_theta;
+      at.qk_rotated = attention_mma_ok(at);  // the forward rotated the saved q and k in place
       at.scale = 1.f / sqrtf((float)ctx->dh); at.O = sb + so.O;
       at.lse = (float*)(sb + so.lse); at.dO = ctx->ws(ctx->b_dO); at.Dscratch = ctx->ws<float>(ctx->b_D);
       at.dqkv = ctx->ws(ctx->b_dqkv); at.err = ctx->ws<unsigned>(ctx->ws_err);
