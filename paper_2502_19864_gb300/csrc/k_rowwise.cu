@@ -518,20 +518,36 @@ inline int row_vec(int H) {
 // Heads
 // ---------------------------------------------------------------------------------------
 constexpr int MAXC = 32, MAXB = 256;
-// forward: logits = y[b, 0, :] Wh^T + bh, mean CE, dlogits = (softmax - onehot) / B
-template <typename T>
-__global__ void __launch_bounds__(256) encoder_head_fwd_kernel(const void* y, const float* Wh,
+constexpr int HEAD_FWD_THREADS = 512, HEAD_BWD_THREADS = 128;
+// forward: logits = y[b, 0, :] Wh^T + bh, mean CE, dlogits = (softmax - onehot) / B.
+// One warp per batch row computes all C logits of the row at once, with eight loads of the
+// CLS row in flight per lane; then one thread per row takes the softmax.  CM >= C is the
+// number of class accumulators held in registers (2, 8 or MAXC).
+template <typename T, int CM>
+__global__ void __launch_bounds__(HEAD_FWD_THREADS) encoder_head_fwd_kernel(const void* y, const float* Wh,
     const float* bh, const int32_t* labels, int B, int S, int H, int C, float* loss,
     float* logits_out, float* dlogits, unsigned* err) {
   __shared__ float lg[MAXB * MAXC];
   __shared__ float red[MAXB];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int pc = warp; pc < B * C; pc += 8) {
-    int b = pc / C, c = pc % C;
-    float s = 0.f;
-    for (int i = lane; i < H; i += 32) s += ldf<T>(y, (int64_t)b * S * H + i) * Wh[(int64_t)c * H + i];
-    s = warp_sum(s);
-    if (lane == 0) lg[b * C + c] = s + bh[c];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  for (int b = warp; b < B; b += nw) {
+    const int64_t row = (int64_t)b * S * H;
+    float acc[CM];
+#pragma unroll
+    for (int c = 0; c < CM; ++c) acc[c] = 0.f;
+#pragma unroll 8
+    for (int i = lane; i < H; i += 32) {
+      const float x = ldf<T>(y, row + i);
+#pragma unroll
+      for (int c = 0; c < CM; ++c)
+        if (c < C) acc[c] += x * __ldg(Wh + (int64_t)c * H + i);
+    }
+#pragma unroll
+    for (int c = 0; c < CM; ++c)
+      if (c < C) {
+        const float s = warp_sum(acc[c]);
+        if (lane == 0) lg[b * C + c] = s + bh[c];
+      }
   }
   __syncthreads();
   for (int b = threadIdx.x; b < B; b += blockDim.x) {
@@ -557,24 +573,46 @@ __global__ void __launch_bounds__(256) encoder_head_fwd_kernel(const void* y, co
   }
 }
 
-// backward: dWh = dlogits^T cls, dbh = sum_b dlogits, dy[b, 0, :] = dlogits Wh
-template <typename T>
-__global__ void __launch_bounds__(256) encoder_head_bwd_kernel(const void* y, const float* Wh,
+// backward: dWh = dlogits^T cls, dbh = sum_b dlogits, dy[b, 0, :] = dlogits Wh.  One thread
+// per column i; the column's B CLS values are loaded eight at a time, so a thread waits on
+// B / 8 round trips instead of C * B.  CM >= C as in the forward.
+template <typename T, int CM>
+__global__ void __launch_bounds__(HEAD_BWD_THREADS) encoder_head_bwd_kernel(const void* y, const float* Wh,
     const float* dlogits, int B, int S, int H, int C, float* dWh, float* dbh, float* dy) {
   __shared__ float lg[MAXB * MAXC];
   for (int e = threadIdx.x; e < B * C; e += blockDim.x) lg[e] = dlogits[e];
   __syncthreads();
-  int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < H) {
-    for (int c = 0; c < C; ++c) {
-      float s = 0.f;
-      for (int b = 0; b < B; ++b) s += lg[b * C + c] * ldf<T>(y, (int64_t)b * S * H + i);
-      if (dWh) dWh[(int64_t)c * H + i] = s;
+    float w[CM], acc[CM];
+#pragma unroll
+    for (int c = 0; c < CM; ++c) {
+      acc[c] = 0.f;
+      w[c] = c < C ? __ldg(Wh + (int64_t)c * H + i) : 0.f;
     }
-    for (int b = 0; b < B; ++b) {
-      float s = 0.f;
-      for (int c = 0; c < C; ++c) s += lg[b * C + c] * Wh[(int64_t)c * H + i];
-      dy[(int64_t)b * S * H + i] = s;
+    for (int b0 = 0; b0 < B; b0 += 8) {
+      float x[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) x[k] = b0 + k < B ? ldf<T>(y, (int64_t)(b0 + k) * S * H + i) : 0.f;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (b0 + k < B) {
+          const float* l = lg + (b0 + k) * C;
+          float s = 0.f;
+#pragma unroll
+          for (int c = 0; c < CM; ++c)
+            if (c < C) {
+              acc[c] += l[c] * x[k];
+              s += l[c] * w[c];
+            }
+          dy[(int64_t)(b0 + k) * S * H + i] = s;
+        }
+      }
+    }
+    if (dWh) {
+#pragma unroll
+      for (int c = 0; c < CM; ++c)
+        if (c < C) dWh[(int64_t)c * H + i] = acc[c];
     }
   }
   if (dbh && blockIdx.x == 0 && threadIdx.x < C) {
@@ -874,10 +912,11 @@ cudaError_t encoder_head_fwd(const void* y, int dtype, const float* Wh, const fl
                              const int32_t* labels, int B, int S, int H, int C, float* loss,
                              float* logits_out, float* dlogits, unsigned* err, cudaStream_t st) {
   if (C > MAXC || B > MAXB) return cudaErrorInvalidValue;
-  if (dtype == DT_BF16)
-    encoder_head_fwd_kernel<bf16><<<1, 256, 0, st>>>(y, Wh, bh, labels, B, S, H, C, loss, logits_out, dlogits, err);
-  else
-    encoder_head_fwd_kernel<float><<<1, 256, 0, st>>>(y, Wh, bh, labels, B, S, H, C, loss, logits_out, dlogits, err);
+  auto k = dtype == DT_BF16 ? (C <= 2 ? encoder_head_fwd_kernel<bf16, 2>
+                               : C <= 8 ? encoder_head_fwd_kernel<bf16, 8> : encoder_head_fwd_kernel<bf16, MAXC>)
+                            : (C <= 2 ? encoder_head_fwd_kernel<float, 2>
+                               : C <= 8 ? encoder_head_fwd_kernel<float, 8> : encoder_head_fwd_kernel<float, MAXC>);
+  k<<<1, HEAD_FWD_THREADS, 0, st>>>(y, Wh, bh, labels, B, S, H, C, loss, logits_out, dlogits, err);
   note_launch(1);
   return cudaGetLastError();
 }
@@ -886,11 +925,12 @@ cudaError_t encoder_head_bwd(const void* y, int dtype, const float* Wh, const fl
                              int B, int S, int H, int C, float* dWh, float* dbh, float* dy,
                              cudaStream_t st) {
   if (C > MAXC || B > MAXB) return cudaErrorInvalidValue;
-  unsigned grid = blocks_for(H, 256);
-  if (dtype == DT_BF16)
-    encoder_head_bwd_kernel<bf16><<<grid, 256, 0, st>>>(y, Wh, dlogits, B, S, H, C, dWh, dbh, dy);
-  else
-    encoder_head_bwd_kernel<float><<<grid, 256, 0, st>>>(y, Wh, dlogits, B, S, H, C, dWh, dbh, dy);
+  unsigned grid = blocks_for(H, HEAD_BWD_THREADS);
+  auto k = dtype == DT_BF16 ? (C <= 2 ? encoder_head_bwd_kernel<bf16, 2>
+                               : C <= 8 ? encoder_head_bwd_kernel<bf16, 8> : encoder_head_bwd_kernel<bf16, MAXC>)
+                            : (C <= 2 ? encoder_head_bwd_kernel<float, 2>
+                               : C <= 8 ? encoder_head_bwd_kernel<float, 8> : encoder_head_bwd_kernel<float, MAXC>);
+  k<<<grid, HEAD_BWD_THREADS, 0, st>>>(y, Wh, dlogits, B, S, H, C, dWh, dbh, dy);
   note_launch(1);
   return cudaGetLastError();
 }
