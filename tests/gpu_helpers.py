@@ -23,12 +23,13 @@ def ra_cfg(cfg, max_depth=0, max_batch=None, max_seq=None):
 class GpuRun:
     """One context on cuda:0 loaded with a synthetic workload."""
 
-    def __init__(self, cfg, w, max_depth=0, want_logits=True):
+    def __init__(self, cfg, w, max_depth=0, want_logits=True, max_batch=None, max_seq=None):
         import torch
         self.torch = torch
         self.cfg = cfg
         self.w = w
-        self.model = R.Model(ra_cfg(cfg, max_depth), cfg.adapter_dim, device="cuda:0")
+        self.model = R.Model(ra_cfg(cfg, max_depth, max_batch, max_seq), cfg.adapter_dim,
+                             device="cuda:0")
         self.model.set_weights(w["layers"], w["head"])
         dt = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
         self.x = torch.tensor(w["x"], dtype=torch.float32).to(dt).cuda()
