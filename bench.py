@@ -102,7 +102,7 @@ def run_cpu_baseline(cfg_name, depth, batch, seconds):
 
 
 def reference_main(args):
-    rank = int(os.environ.get("RANK", "0"))
+    _, rank, _ = rank_env()
     if rank != 0:
         return 0
     import synth
@@ -301,12 +301,32 @@ class Runner:
         return ms, h2d, 4
 
 
+def rank_env():
+    """(world size, rank, local rank) from the torchrun environment; (1, 0, 0) without it."""
+    return (int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def max_over_ranks(dist, values, device):
+    """Element-wise maximum over the ranks of per-rank floats (the slowest rank's times);
+    the values themselves when there is no process group."""
+    if dist is None:
+        return [float(v) for v in values]
+    import torch
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def job_value(world, batch, ms):
+    """Whole-job samples/s: the samples of every replica over the slowest replica's step."""
+    return world * batch / (ms / 1000.0)
+
+
 def gpu_main(args):
     import torch
     import synth
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    world, rank, local = rank_env()
     dist = None
     if world > 1:
         import torch.distributed as dist
@@ -347,6 +367,9 @@ def gpu_main(args):
     clk = start_clock_sampler(torch.cuda.current_device())
     ms = run.time_steps(HEADLINE_D, steps, warmup)
     clocks = stop_clock_sampler(clk)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
     sweep[HEADLINE_D] = ms
     e2e_ms, h2d, d2h = run.time_e2e(HEADLINE_D, steps)
     # per-kernel device times: a second timed region, the same step with an event around
@@ -356,14 +379,14 @@ def gpu_main(args):
     saved_by_d = dict(run.saved)
     R.ra_set_unfrozen_depth(run.model.ctx, HEADLINE_D)
 
-    # max over ranks
-    if dist:
-        t = torch.tensor([ms, e2e_ms], device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, e2e_ms = t.tolist()
+    # the slowest rank's times (headline, end to end and every sweep point)
+    sweep_d = sorted(sweep)
+    red = max_over_ranks(dist, [ms, e2e_ms] + [sweep[d] for d in sweep_d], device)
+    ms, e2e_ms = red[0], red[1]
+    sweep = dict(zip(sweep_d, red[2:]))
 
     B = cfg.batch
-    value = world * B / (ms / 1000.0)
+    value = job_value(world, B, ms)
     g = prof["gemm"]
     gemm_tflops = g["flops"] / (g["ms"] / 1000.0) / 1e12 if g["ms"] > 0 else None
     traffic_per_flop, traffic_note = gemm_traffic()
@@ -407,7 +430,7 @@ def gpu_main(args):
                    "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2 (>1 GB streamed per step)",
                    "cuda_graph": True},
-        "sweep": {"d=%d" % d: {"samples_per_s": world * B / (sweep[d] / 1000.0),
+        "sweep": {"d=%d" % d: {"samples_per_s": job_value(world, B, sweep[d]),
                                "ms_per_step": sweep[d], "k": cfg.n_layers - d,
                                "saved_activation_bytes": saved_by_d[d]}
                   for d in sorted(sweep)},
@@ -416,7 +439,7 @@ def gpu_main(args):
         "roofline": roof,
         "phases_ms": phases,
         "clocks": clocks,
-        "e2e": {"value": world * B / (e2e_ms / 1000.0), "unit": UNIT,
+        "e2e": {"value": job_value(world, B, e2e_ms), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
         "gpu_launches": launches_headline * steps,
         "gpu_launches_per_step": launches_headline,
