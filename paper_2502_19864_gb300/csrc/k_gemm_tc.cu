@@ -47,10 +47,9 @@ constexpr int SLOT_BYTES = 4096, NSLOT = 1;
 // epilogues that read a saved operand per output element (GELU', residual, SwiGLU')
 template <int EPI>
 struct EpiTraits {
-  // the GELU epilogue evaluates erf per element: 12 epilogue warps (three per TMEM lane
-  // quadrant) for it, 8 for the others (GELU + GELU' needs more registers than 12 warps
-  // leave)
-  static constexpr int WARPS = EPI == EPI_BIAS_GELU ? 12 : 8;
+  // the GELU epilogues evaluate erf per element: 12 epilogue warps (three per TMEM lane
+  // quadrant) for them, 8 for the others
+  static constexpr int WARPS = (EPI == EPI_BIAS_GELU || EPI == EPI_BIAS_GELU_G) ? 12 : 8;
   static constexpr int THREADS = (2 + WARPS) * 32;
   static constexpr bool AUX = EPI == EPI_MUL || EPI == EPI_RESID || EPI == EPI_DSWIGLU;
 };
@@ -269,17 +268,45 @@ __device__ __forceinline__ void epi_chunk(const TcParams& p, const CUtensorMap* 
     }
     store_chunk(tmC2, staging, slot_i, p.c2_dtype, lane, v, n, row0, ts);
   } else if (EPI == EPI_BIAS_GELU_G) {
-    float d[32];
+    // GELU'(u) (bf16) goes into its staging slot 8 values at a time as they are computed, so
+    // no second 32-value array stays live (this is what lets the epilogue run 12 warps);
+    // GELU(u) replaces u in v and leaves through the usual chunk store
+    uint8_t* slot = staging + (ts ? (slot_i & 1) * (SLOT_BYTES / 2) : 0);
+    if (p.C) {
+      if (lane == 0) {  // the store that last used this slot has read it
+        if (ts) bulk_wait_read<1>();
+        else bulk_wait_read<0>();
+      }
+      __syncwarp();
+    }
+    uint8_t* row = slot + lane * 64;
+    const int sw = (lane >> 1) & 3;
 #pragma unroll
-    for (int j = 0; j < 32; j += 8) {
+    for (int q = 0; q < 4; ++q) {
       F8 x;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) x.v[i] = v[j + i];
+      for (int i = 0; i < 8; ++i) x.v[i] = v[8 * q + i];
       const F8x2 r = gelu_both8(x);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) { v[j + i] = r.y.v[i]; d[j + i] = r.d.v[i]; }
+      for (int i = 0; i < 8; ++i) v[8 * q + i] = r.y.v[i];
+      if (p.C) {
+        uint4 u;
+        u.x = pack_bf16x2(r.d.v[0], r.d.v[1]);
+        u.y = pack_bf16x2(r.d.v[2], r.d.v[3]);
+        u.z = pack_bf16x2(r.d.v[4], r.d.v[5]);
+        u.w = pack_bf16x2(r.d.v[6], r.d.v[7]);
+        *reinterpret_cast<uint4*>(row + ((q ^ sw) << 4)) = u;
+      }
     }
-    if (p.C) store_chunk(tmC, staging, slot_i, p.c_dtype, lane, d, n, row0, ts);
+    if (p.C) {
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d(tmC, (uint32_t)__cvta_generic_to_shared(slot), n, row0);
+        bulk_commit();
+      }
+      ++slot_i;
+    }
     store_chunk(tmC2, staging, slot_i, p.c2_dtype, lane, v, n, row0, ts);
   }
 }
@@ -783,6 +810,8 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   if (g.C2 && (!aligned16(g.C2) || g.ldc2 % 8)) return cudaErrorNotSupported;
   if (g.aux && (!aligned16(g.aux) || g.ldaux % 8)) return cudaErrorNotSupported;
   if (g.epi == EPI_SWIGLU && (g.N % 128 || !g.C2)) return cudaErrorNotSupported;
+  // the GELU' output of EPI_BIAS_GELU_G is staged as bf16
+  if (g.epi == EPI_BIAS_GELU_G && has_c && g.c_dtype != DT_BF16) return cudaErrorNotSupported;
   if (g.epi == EPI_DSWIGLU && g.N % 64) return cudaErrorNotSupported;
   if (!has_c && g.epi != EPI_BIAS_GELU && g.epi != EPI_BIAS_GELU_G && g.epi != EPI_SWIGLU)
     return cudaErrorNotSupported;
