@@ -454,7 +454,7 @@ def gpu_main(args):
 
 def large_gemm_check(torch, R, synth, device, peaks):
     """BERT-large-shaped step at d = 24 and d = 1: samples/s and the GEMMs' tensor throughput
-    (the spec bar is >= 60 % of dense bf16 peak in these GEMMs)."""
+    (the target for these GEMMs is >= 60 % of the dense bf16 peak)."""
     cfg = synth.CONFIGS["large"]
     run = Runner(cfg, cfg.n_layers, device)
     out = {}

@@ -1,4 +1,4 @@
-"""Parity of the CUDA path (through the C ABI) with the fp64 oracle, and the north-star
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle, and the step's
 invariants on the GPU: truncated gradients equal full-backprop gradients, nothing below k
 is written, frozen weights never change, the step is deterministic, checkpoints resume."""
 import numpy as np

@@ -287,7 +287,7 @@ def test_encoder_stack_matches_torch_layers_with_autograd():
 
 
 def test_encoder_without_adapters_matches_torch_layer_bitwise_identity_invariant():
-    """Spec invariant 1: zero W_up reproduces the frozen model exactly; the frozen
+    """Invariant: zero W_up reproduces the frozen model exactly (Eq. 1 adds 0); the frozen
     model itself matches torch's TransformerEncoderLayer."""
     cfg = _small_enc_cfg()
     w = synth.make_workload(cfg, 1)
