@@ -26,8 +26,9 @@ Readings where the paper is silent (each also listed in the design notes):
   sigma = exact erf GELU; adapters carry no biases; post-LN encoder blocks with LayerNorm
   (biased variance, eps 1e-12) and biased linears; pre-norm decoder blocks with RMSNorm
   (eps 1e-6), causal attention, rotate-half RoPE (theta 10000) and SwiGLU; attention scale
-  1/sqrt(head_dim) with no padding mask; encoder head on the token at position 0; mean
-  cross-entropy over rows; all gradients, including the one leaving the head, use the
+  1/sqrt(head_dim) with no padding mask; encoder head on the token at position 0, or a span
+  head (start and end logits at every token, the mean of the two cross-entropies over the
+  sequence positions); mean cross-entropy over rows; all gradients, including the one leaving the head, use the
   pre-update weights, and the head and adapters are updated together afterwards; Adam with
   PyTorch's default semantics and a per-parameter step count that starts at the first
   gradient a parameter receives.
@@ -317,6 +318,25 @@ def encoder_head(y, head, labels, cfg):
     return loss, logits, dy.reshape(B * S, H), grads
 
 
+def encoder_span_head(y, head, labels, cfg):
+    """Span head of extractive question answering (the paper's SQuAD task, Section IV):
+    start and end logits at every token, [B, S, 2] = y Wh^T + bh with Wh [2, H]; the loss is
+    the mean of the start and end cross-entropies, each a softmax over the S positions of a
+    sequence, averaged over the batch.  labels [B, 2] = (start, end).  Returns loss, logits
+    [B*S, 2], dy [B*S, H] (every position receives a gradient) and the head gradients."""
+    B, S, H = cfg.batch, cfg.seq, cfg.hidden
+    labels = np.asarray(labels).reshape(B, 2)
+    logits = y @ head["Wh"].T + head["bh"]                      # [B*S, 2]
+    z = logits.reshape(B, S, 2)
+    loss_start, d_start = cross_entropy(z[:, :, 0], labels[:, 0])
+    loss_end, d_end = cross_entropy(z[:, :, 1], labels[:, 1])
+    loss = 0.5 * (loss_start + loss_end)
+    dlogits = 0.5 * np.stack([d_start, d_end], axis=-1).reshape(B * S, 2)
+    dy = dlogits @ head["Wh"]
+    grads = dict(Wh=dlogits.T @ y, bh=dlogits.sum(axis=0))
+    return loss, logits, dy, grads
+
+
 def decoder_head(y, head, labels, cfg):
     """Final RMSNorm, frozen vocabulary projection, mean next-token cross-entropy over
     all B*S positions (label[b, t] is the target at position t)."""
@@ -357,7 +377,9 @@ def forward(cfg, layers, head, x, labels, d, adapters=True, start_layer=0, h0=No
         if l >= k:
             caches[l] = c
     labels = np.asarray(labels).astype(np.int64)
-    if cfg.arch == "encoder":
+    if cfg.arch == "encoder" and getattr(cfg, "head", "cls") == "span":
+        loss, logits, dy, hgrads = encoder_span_head(h, head, labels, cfg)
+    elif cfg.arch == "encoder":
         loss, logits, dy, hgrads = encoder_head(h, head, labels, cfg)
     else:
         loss, logits, dy, hgrads = decoder_head(h, head, labels, cfg)

@@ -11,7 +11,9 @@ Workload recipe (stands in for mBERT on SQuAD, Section IV, which is not availabl
     beta ~ N(0, 0.02); RMSNorm gamma ~ 1 + N(0, 0.02),
   * adapter down-projection ~ N(0, 0.02), up-projection ~ N(0, 1e-3) (Eq. 1 shapes
     W_down [H, m], W_up [m, H]),
-  * encoder: 2-class CLS head ~ N(0, 0.02), labels uniform in [0, 2);
+  * encoder: 2-class CLS head ~ N(0, 0.02), labels uniform in [0, 2); or a span head
+    (start and end logits at every token) ~ N(0, 0.02) with start and end positions drawn
+    independently and uniformly in [0, S);
     decoder: frozen vocabulary head, token labels uniform in [0, V),
   * one torch CPU generator, seed 0 unless stated, draws in the order of ``layer_keys``,
     then the head, then x, then the labels; every value is rounded once to the storage
@@ -41,6 +43,8 @@ class ModelCfg:
     head_trainable: bool = True
     norm_eps: float = 1e-12
     rope_theta: float = 10000.0
+    head: str = "cls"    # encoder head: "cls" (position 0, n_out classes) | "span" (start/end
+                         # logits at every position, n_out = 2)
 
     @property
     def head_dim(self) -> int:
@@ -53,6 +57,10 @@ class ModelCfg:
 
 def _enc(L, H, h, F, m, B, S, dtype, C=2):
     return ModelCfg("encoder", L, H, h, F, m, C, B, S, dtype, True, 1e-12)
+
+
+def _span(L, H, h, F, m, B, S, dtype):
+    return ModelCfg("encoder", L, H, h, F, m, 2, B, S, dtype, True, 1e-12, head="span")
 
 
 def _dec(L, H, h, F, m, V, B, S, dtype):
@@ -70,6 +78,9 @@ CONFIGS: Dict[str, ModelCfg] = {
     "small_enc_bf16": _enc(3, 256, 4, 1024, 32, 3, 100, "bf16"),
     "small_dec_bf16": _dec(3, 256, 2, 704, 32, 1000, 2, 200, "bf16"),
     "mid_enc_f32": _enc(3, 192, 3, 768, 24, 5, 77, "f32"),
+    # span (start/end) head over every token, the shape of extractive question answering
+    "tiny_span": _span(2, 128, 2, 512, 16, 4, 32, "f32"),
+    "small_span_bf16": _span(3, 256, 4, 1024, 32, 3, 100, "bf16"),
 }
 
 
@@ -135,7 +146,9 @@ def make_workload(cfg: ModelCfg, seed: int = 0):
     for key in head_keys(cfg):
         head[key] = round_to(_draw(gen, key, param_shape(cfg, key)), cfg.dtype)
     x = round_to(torch.randn((cfg.batch, cfg.seq, cfg.hidden), generator=gen), cfg.dtype)
-    if cfg.arch == "encoder":
+    if cfg.arch == "encoder" and cfg.head == "span":
+        labels = torch.randint(0, cfg.seq, (cfg.batch, 2), generator=gen)
+    elif cfg.arch == "encoder":
         labels = torch.randint(0, cfg.n_out, (cfg.batch,), generator=gen)
     else:
         labels = torch.randint(0, cfg.n_out, (cfg.batch, cfg.seq), generator=gen)
@@ -146,7 +159,11 @@ def make_batch(cfg: ModelCfg, seed: int):
     """A fresh (x, labels) batch from its own generator, for multi-step runs."""
     gen = torch.Generator().manual_seed(seed)
     x = round_to(torch.randn((cfg.batch, cfg.seq, cfg.hidden), generator=gen), cfg.dtype)
-    shape = (cfg.batch,) if cfg.arch == "encoder" else (cfg.batch, cfg.seq)
-    labels = torch.randint(0, cfg.n_out, shape, generator=gen).to(torch.int32).numpy()
+    if cfg.arch == "encoder" and cfg.head == "span":
+        labels = torch.randint(0, cfg.seq, (cfg.batch, 2), generator=gen)
+    else:
+        shape = (cfg.batch,) if cfg.arch == "encoder" else (cfg.batch, cfg.seq)
+        labels = torch.randint(0, cfg.n_out, shape, generator=gen)
+    labels = labels.to(torch.int32).numpy()
     return x, labels
 

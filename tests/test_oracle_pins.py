@@ -168,6 +168,34 @@ def test_cross_entropy_matches_torch():
     assert O.cross_entropy(np.zeros((3, 5)), np.array([0, 1, 4]))[0] == pytest.approx(np.log(5), rel=1e-15)
 
 
+def test_span_head_matches_torch_autograd():
+    """Span head (start/end logits at every token): loss, the gradient into every token and
+    the head gradients against torch's cross_entropy over the sequence positions."""
+    import dataclasses
+    cfg = dataclasses.replace(synth.CONFIGS["tiny_span"], batch=3, seq=11, hidden=16)
+    r = rng(12)
+    y = r.normal(size=(cfg.batch * cfg.seq, cfg.hidden))
+    head = dict(Wh=r.normal(size=(2, cfg.hidden)) * 0.3, bh=r.normal(size=2))
+    labels = r.integers(0, cfg.seq, size=(cfg.batch, 2))
+    loss, logits, dy, g = O.encoder_span_head(y, head, labels, cfg)
+    yt, Wt, bt = T(y, True), T(head["Wh"], True), T(head["bh"], True)
+    z = (yt @ Wt.T + bt).reshape(cfg.batch, cfg.seq, 2)
+    lab = torch.tensor(labels)
+    lt = 0.5 * (Fnn.cross_entropy(z[:, :, 0], lab[:, 0]) + Fnn.cross_entropy(z[:, :, 1], lab[:, 1]))
+    lt.backward()
+    assert loss == pytest.approx(lt.item(), rel=1e-14)
+    np.testing.assert_allclose(logits, z.detach().reshape(-1, 2).numpy(), rtol=1e-13, atol=1e-14)
+    np.testing.assert_allclose(dy, yt.grad.numpy(), rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(g["Wh"], Wt.grad.numpy(), rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(g["bh"], bt.grad.numpy(), rtol=1e-12, atol=1e-15)
+    # each sequence's start (and end) gradients sum to zero over its positions
+    d = dy @ np.linalg.pinv(head["Wh"])
+    assert np.abs(d.reshape(cfg.batch, cfg.seq, 2).sum(axis=1)).max() < 1e-12
+    # equal logits everywhere: the loss is ln S
+    flat = dict(Wh=np.zeros((2, cfg.hidden)), bh=np.zeros(2))
+    assert O.encoder_span_head(y, flat, labels, cfg)[0] == pytest.approx(np.log(cfg.seq), rel=1e-15)
+
+
 # ----------------------------------------------------------------------------------------
 # adapter (Eq. 1)
 # ----------------------------------------------------------------------------------------
@@ -353,7 +381,9 @@ def test_decoder_branch_wiring_special_cases():
 # finite differences (brute force) on the tiny configs
 # ----------------------------------------------------------------------------------------
 
-def _fd_check(cfg, w, d, n_coords=48, eps=1e-2, tol=1e-6, seed=0):
+def _fd_check(cfg, w, d, n_coords=48, eps=1e-2, tol=1e-6, seed=0, zero_keys=()):
+    """Central differences against the oracle's gradients.  ``zero_keys`` name head
+    parameters the loss does not depend on (their gradient must be zero both ways)."""
     layers, head = O.to_f64_params(w["layers"], w["head"])
     res = O.step(cfg, layers, head, w["x"], w["labels"], d)
     k = cfg.n_layers - d
@@ -387,6 +417,9 @@ def _fd_check(cfg, w, d, n_coords=48, eps=1e-2, tol=1e-6, seed=0):
             # Richardson extrapolation of the two central differences: O(e^4) truncation
             fd[j] = (4.0 * central[1] - central[0]) / 3.0
         an = grad.flat[idx]
+        if l == "head" and key in zero_keys:
+            assert np.abs(an).max() <= 1e-14 and np.abs(fd).max() <= 1e-8, (key, an, fd)
+            continue
         err = np.linalg.norm(fd - an) / np.linalg.norm(an)
         assert err <= tol, (l, key, err)
         # per coordinate, against the tensor's scale: a single wrong row or column fails here
@@ -402,6 +435,14 @@ def test_fd_tiny_encoder_top_layer():
 def test_fd_tiny_encoder_full_depth_stressed():
     cfg = synth.CONFIGS["tiny"]
     _fd_check(cfg, _stress_workload(cfg, 0), d=cfg.n_layers, n_coords=24)
+
+
+def test_fd_tiny_span_encoder_top_layer_and_full_depth():
+    # a common shift of all start (or end) logits of a sequence leaves its softmax
+    # unchanged, so the span head's bias gets no gradient at all
+    cfg = synth.CONFIGS["tiny_span"]
+    _fd_check(cfg, synth.make_workload(cfg, 0), d=1, n_coords=24, zero_keys=("bh",))
+    _fd_check(cfg, _stress_workload(cfg, 2), d=cfg.n_layers, n_coords=12, zero_keys=("bh",))
 
 
 def test_fd_tiny_decoder_top_layer_and_full_depth():
