@@ -58,15 +58,18 @@ typedef enum {
   RA_ERR_UNSUPPORTED = 8  /* no sm_103 device, or a feature this build does not have */
 } ra_status;
 
-enum { RA_ENCODER_POSTLN = 0, RA_DECODER_PRENORM = 1 };
+enum { RA_ENCODER_POSTLN = 0, RA_DECODER_PRENORM = 1, RA_ENCODER_POSTLN_SPAN = 2 };
 enum { RA_F32 = 0, RA_BF16 = 1 };
 
 /* Model shape.  Encoder: post-LN blocks (LayerNorm, biased linears, exact-GELU FFN), a
- * trainable n_out-class linear head on the token at position 0.  Decoder: pre-RMSNorm
+ * trainable n_out-class linear head on the token at position 0.  Span encoder
+ * (RA_ENCODER_POSTLN_SPAN): the same blocks with the extractive-QA head of the paper's SQuAD
+ * task (Section IV): start and end logits at every token (n_out = 2, max_seq <= 4096), loss
+ * = mean over the batch of (CE_start + CE_end) / 2, each a softmax over the sequence.  Decoder: pre-RMSNorm
  * blocks, causal attention with rotate-half RoPE, SwiGLU FFN (ffn % 64 == 0), final
  * RMSNorm and a frozen n_out-way vocabulary head over every position. */
 typedef struct {
-  int32_t arch;            /* RA_ENCODER_POSTLN | RA_DECODER_PRENORM */
+  int32_t arch;            /* RA_ENCODER_POSTLN | RA_DECODER_PRENORM | RA_ENCODER_POSTLN_SPAN */
   int32_t n_layers;        /* L >= 1 */
   int32_t hidden;          /* H, multiple of 64 */
   int32_t n_heads;         /* H / n_heads in {64, 128} for bf16, <= 128 for f32 */
@@ -149,9 +152,11 @@ ra_status ra_set_weights(ra_ctx* ctx, const ra_tensor_desc* list, int32_t n, ra_
 ra_status ra_set_unfrozen_depth(ra_ctx* ctx, int32_t d);
 
 /* Forward and loss (Algorithm 1 "Fw propagation", "calculates the loss").
- * x_dev [B, S, H] in the model dtype; labels_dev int32 [B] (encoder) or [B, S] (decoder);
- * loss_dev: one float (mean cross-entropy); logits_dev: nullable, float [B, n_out]
- * (encoder) or [B*S, n_out] (decoder).  Returns RA_ERR_SHAPE if B or S exceed capacity. */
+ * x_dev [B, S, H] in the model dtype; labels_dev int32 [B] (encoder), [B, 2] = (start,
+ * end) positions (span encoder) or [B, S] (decoder); loss_dev: one float (mean
+ * cross-entropy); logits_dev: nullable, float [B, n_out] (encoder) or [B*S, n_out] (span
+ * encoder, decoder).  Returns RA_ERR_SHAPE if B or S exceed capacity.  Labels out of range
+ * are read as 0 and reported by ra_sync_status. */
 ra_status ra_forward(ra_ctx* ctx, const void* x_dev, const int32_t* labels_dev, int32_t B,
                      int32_t S, float* loss_dev, float* logits_dev, ra_stream_t stream);
 

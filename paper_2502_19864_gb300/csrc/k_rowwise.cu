@@ -622,6 +622,130 @@ __global__ void __launch_bounds__(HEAD_BWD_THREADS) encoder_head_bwd_kernel(cons
   }
 }
 
+// ---------------------------------------------------------------------------------------
+// Span head: start and end logits at every token, loss = the mean over the batch of
+// (CE_start + CE_end) / 2, each a softmax over the S positions of one sequence.
+// ---------------------------------------------------------------------------------------
+constexpr int SPAN_CHUNKS = 32;   // token chunks of the deterministic dWh reduction
+// forward: one CTA per sequence b.  logits [S, 2] of its tokens (a warp per token, both
+// logits at once) into shared memory; warp c then takes the softmax over S of column c and
+// writes dlogits[t, c] = (p_c(s) - [s == label_c]) / (2 B); row_loss[b] = mean of the two
+// cross-entropies.
+template <typename T>
+__global__ void __launch_bounds__(256) span_head_fwd_kernel(const void* y, const float* Wh,
+    const float* bh, const int32_t* labels, int B, int S, int H, float* row_loss,
+    float* logits_out, float* dlogits, unsigned* err) {
+  extern __shared__ float zs[];  // [S][2]
+  __shared__ float part[2];
+  const int b = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  for (int s = warp; s < S; s += nw) {
+    const int64_t row = ((int64_t)b * S + s) * H;
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll 8
+    for (int i = lane; i < H; i += 32) {
+      const float x = ldf<T>(y, row + i);
+      a0 += x * __ldg(Wh + i);
+      a1 += x * __ldg(Wh + H + i);
+    }
+    a0 = warp_sum(a0);
+    a1 = warp_sum(a1);
+    if (lane == 0) {
+      zs[2 * s] = a0 + bh[0];
+      zs[2 * s + 1] = a1 + bh[1];
+    }
+  }
+  __syncthreads();
+  if (warp < 2) {
+    const int c = warp;
+    int lab = labels[2 * b + c];
+    if (lab < 0 || lab >= S) {
+      if (lane == 0) set_dev_error(err, RA_DEVERR_BOUNDS);
+      lab = 0;
+    }
+    float mx = -INFINITY;
+    for (int s = lane; s < S; s += 32) mx = fmaxf(mx, zs[2 * s + c]);
+    mx = warp_max(mx);
+    float se = 0.f;
+    for (int s = lane; s < S; s += 32) se += expf(zs[2 * s + c] - mx);
+    se = warp_sum(se);
+    const float lse = mx + logf(se);
+    const float inv = 1.f / (2.f * B);
+    for (int s = lane; s < S; s += 32) {
+      const int64_t t = (int64_t)b * S + s;
+      const float z = zs[2 * s + c];
+      if (logits_out) logits_out[2 * t + c] = z;
+      dlogits[2 * t + c] = (expf(z - lse) - (s == lab ? 1.f : 0.f)) * inv;
+    }
+    if (lane == 0) part[c] = lse - zs[2 * lab + c];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) row_loss[b] = 0.5f * (part[0] + part[1]);
+}
+
+// backward, every token's gradient: dy[t, :] = dlogits[t, 0] Wh[0, :] + dlogits[t, 1] Wh[1, :]
+// (a warp per token, 16-byte accesses; H % 4 == 0)
+__global__ void __launch_bounds__(256) span_head_dy_kernel(const float* Wh, const float* dlogits,
+                                                           int Tn, int H, float* dy) {
+  const int64_t t = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (t >= Tn) return;
+  const float d0 = dlogits[2 * t], d1 = dlogits[2 * t + 1];
+  for (int i = 4 * lane; i < H; i += 128) {
+    const float4 w0 = __ldg(reinterpret_cast<const float4*>(Wh + i));
+    const float4 w1 = __ldg(reinterpret_cast<const float4*>(Wh + H + i));
+    *reinterpret_cast<float4*>(dy + t * H + i) =
+        make_float4(d0 * w0.x + d1 * w1.x, d0 * w0.y + d1 * w1.y, d0 * w0.z + d1 * w1.z, d0 * w0.w + d1 * w1.w);
+  }
+}
+
+// backward, head weights: per chunk c of tokens, part[c][j][i] = sum over the chunk's tokens
+// (in token order) of dlogits[t, j] y[t, i] (a thread per column i, eight tokens' loads in
+// flight), and part_b[c][j] = the chunk's sum of dlogits[t, j]
+template <typename T>
+__global__ void __launch_bounds__(128) span_head_dw_kernel(const void* y, const float* dlogits,
+    int Tn, int H, int chunk, float* part, float* part_b) {
+  const int i = blockIdx.x * 128 + threadIdx.x, c = blockIdx.y;
+  const int t0 = c * chunk, t1 = min(Tn, t0 + chunk);
+  if (i < H) {
+    float a0 = 0.f, a1 = 0.f;
+    for (int t = t0; t < t1; t += 8) {
+      float x[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) x[k] = t + k < t1 ? ldf<T>(y, (int64_t)(t + k) * H + i) : 0.f;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (t + k < t1) {
+          a0 += dlogits[2 * (t + k)] * x[k];
+          a1 += dlogits[2 * (t + k) + 1] * x[k];
+        }
+      }
+    }
+    part[((size_t)c * 2) * H + i] = a0;
+    part[((size_t)c * 2 + 1) * H + i] = a1;
+  }
+  if (blockIdx.x == 0 && threadIdx.x < 2) {
+    float sb = 0.f;
+    for (int t = t0; t < t1; ++t) sb += dlogits[2 * t + threadIdx.x];
+    part_b[2 * c + threadIdx.x] = sb;
+  }
+}
+
+// fixed-order sum of the chunk partials: dWh [2, H], dbh [2]
+__global__ void __launch_bounds__(256) span_head_dw_reduce_kernel(const float* part, const float* part_b,
+    int nch, int H, float* dWh, float* dbh) {
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (dWh && j < 2 * H) {
+    float s = 0.f;
+    for (int c = 0; c < nch; ++c) s += part[(size_t)c * 2 * H + j];
+    dWh[j] = s;
+  }
+  if (dbh && blockIdx.x == 0 && threadIdx.x < 2) {
+    float s = 0.f;
+    for (int c = 0; c < nch; ++c) s += part_b[2 * c + threadIdx.x];
+    dbh[threadIdx.x] = s;
+  }
+}
+
 // one CTA per row: in-place dlogits = (softmax - onehot) / T
 template <typename T>
 __global__ void __launch_bounds__(256) vocab_ce_kernel(void* logits, int ld,
@@ -932,6 +1056,47 @@ cudaError_t encoder_head_bwd(const void* y, int dtype, const float* Wh, const fl
                                : C <= 8 ? encoder_head_bwd_kernel<float, 8> : encoder_head_bwd_kernel<float, MAXC>);
   k<<<grid, HEAD_BWD_THREADS, 0, st>>>(y, Wh, dlogits, B, S, H, C, dWh, dbh, dy);
   note_launch(1);
+  return cudaGetLastError();
+}
+
+int span_head_chunks() { return SPAN_CHUNKS; }
+
+cudaError_t span_head_fwd(const void* y, int dtype, const float* Wh, const float* bh,
+                          const int32_t* labels, int B, int S, int H, float* row_loss, float* loss,
+                          float* logits_out, float* dlogits, unsigned* err, cudaStream_t st) {
+  if (S < 1 || S > SPAN_MAX_SEQ || B < 1) return cudaErrorInvalidValue;
+  const size_t smem = (size_t)2 * S * sizeof(float);
+  if (dtype == DT_BF16)
+    span_head_fwd_kernel<bf16><<<B, 256, smem, st>>>(y, Wh, bh, labels, B, S, H, row_loss, logits_out, dlogits, err);
+  else
+    span_head_fwd_kernel<float><<<B, 256, smem, st>>>(y, Wh, bh, labels, B, S, H, row_loss, logits_out, dlogits, err);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  mean_kernel<<<1, 256, 0, st>>>(row_loss, B, loss);
+  note_launch(2);
+  return cudaGetLastError();
+}
+
+cudaError_t span_head_bwd(const void* y, int dtype, const float* Wh, const float* dlogits, int B,
+                          int S, int H, float* dWh, float* dbh, float* dy, float* part,
+                          cudaStream_t st) {
+  if (H % 4) return cudaErrorInvalidValue;
+  const int T = B * S;
+  span_head_dy_kernel<<<blocks_for((int64_t)T, 8), 256, 0, st>>>(Wh, dlogits, T, H, dy);
+  note_launch(1);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || (!dWh && !dbh)) return e;
+  const int chunk = (T + SPAN_CHUNKS - 1) / SPAN_CHUNKS;
+  float* part_b = part + (size_t)SPAN_CHUNKS * 2 * H;
+  dim3 grid(blocks_for(H, 128), SPAN_CHUNKS);
+  if (dtype == DT_BF16)
+    span_head_dw_kernel<bf16><<<grid, 128, 0, st>>>(y, dlogits, T, H, chunk, part, part_b);
+  else
+    span_head_dw_kernel<float><<<grid, 128, 0, st>>>(y, dlogits, T, H, chunk, part, part_b);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  span_head_dw_reduce_kernel<<<blocks_for((int64_t)2 * H, 256), 256, 0, st>>>(part, part_b, SPAN_CHUNKS, H, dWh, dbh);
+  note_launch(2);
   return cudaGetLastError();
 }
 

@@ -196,6 +196,21 @@ cudaError_t encoder_head_fwd(const void* y, int dtype, const float* Wh, const fl
 cudaError_t encoder_head_bwd(const void* y, int dtype, const float* Wh, const float* dlogits,
                              int B, int S, int H, int C, float* dWh, float* dbh, float* dy,
                              cudaStream_t st);
+// Span head of extractive QA (start and end logits at every token, Wh [2, H], bh [2]):
+// logits_out (optional) [B*S, 2]; dlogits [B*S, 2] = (softmax over the sequence - onehot) /
+// (2 B) per column; row_loss [B] = (CE_start + CE_end) / 2; loss = their mean (fixed order).
+// labels [B, 2] = (start, end); labels outside [0, S) set RA_DEVERR_BOUNDS and are read as 0.
+constexpr int SPAN_MAX_SEQ = 4096;
+cudaError_t span_head_fwd(const void* y, int dtype, const float* Wh, const float* bh,
+                          const int32_t* labels, int B, int S, int H, float* row_loss, float* loss,
+                          float* logits_out, float* dlogits, unsigned* err, cudaStream_t st);
+// Its backward: dy [B*S, H] (every row written), and, when dWh / dbh are not null, the head
+// gradients through span_head_chunks() token chunks summed in a fixed order; part holds
+// span_head_chunks() * (2 H + 2) floats.
+int span_head_chunks();
+cudaError_t span_head_bwd(const void* y, int dtype, const float* Wh, const float* dlogits, int B,
+                          int S, int H, float* dWh, float* dbh, float* dy, float* part,
+                          cudaStream_t st);
 // Decoder cross-entropy over T rows of V logits (act), in place: logits <- dLoss/dlogits
 // (mean over T).  Per-row losses in row_loss, then loss = mean (fixed order).
 // Labels outside [0, V) set RA_DEVERR_BOUNDS in *err and are read as 0.

@@ -59,6 +59,7 @@ struct ra_ctx {
   int L = 0, H = 0, F = 0, nh = 0, dh = 0, C = 0, Tmax = 0, max_depth = 0;
   int act = DT_F32;
   bool dec = false;
+  bool span = false;   // encoder with the span (start/end) head over every token
   std::string err;
 
   // region sizes and layouts
@@ -79,6 +80,7 @@ struct ra_ctx {
   size_t b_dY[2]{}, b_ds2 = 0, b_df = 0, b_du = 0, b_dy1 = 0, b_ds1 = 0, b_da = 0, b_dO = 0,
          b_dqkv = 0, b_dz = 0, b_part = 0, b_D = 0;
   size_t h_dlogits = 0, h_logits = 0, h_rowloss = 0, h_xL = 0, h_nf = 0, h_rstdf = 0;
+  size_t h_part = 0;   // span head: token-chunk partials of dWh and dbh
 
   // bound memory
   char* W = nullptr;
@@ -311,8 +313,9 @@ void plan(ra_ctx* c) {
   c->b_part = ws.take(adapter_bwd_partials_floats(c->Tmax, c->H, c->m) * 4 + 4096);
   c->b_D = ws.take(Bh * 4);
   // head
-  c->h_dlogits = ws.take((size_t)c->cfg.max_batch * c->C * 4);
+  c->h_dlogits = ws.take((c->span ? T : (size_t)c->cfg.max_batch) * c->C * 4);
   c->h_rowloss = ws.take(T * 4);
+  if (c->span) c->h_part = ws.take((size_t)span_head_chunks() * (2 * H + 2) * 4);
   if (c->dec) {
     c->h_logits = ws.take(T * (size_t)c->C * es);
     c->h_xL = ws.take(T * H * 4);
@@ -335,7 +338,8 @@ ra_status ra_create(const ra_model_cfg* cfg, int32_t adapter_dim, ra_ctx** out) 
   if (!cfg || !out) return RA_ERR_ARG;
   *out = nullptr;
   const ra_model_cfg& g = *cfg;
-  if (g.arch != RA_ENCODER_POSTLN && g.arch != RA_DECODER_PRENORM) return RA_ERR_ARG;
+  if (g.arch != RA_ENCODER_POSTLN && g.arch != RA_DECODER_PRENORM && g.arch != RA_ENCODER_POSTLN_SPAN)
+    return RA_ERR_ARG;
   if (g.dtype != RA_F32 && g.dtype != RA_BF16) return RA_ERR_ARG;
   if (g.n_layers < 1 || g.hidden < 64 || g.n_heads < 1 || g.ffn < 1 || g.n_out < 1 ||
       g.max_batch < 1 || g.max_seq < 1)
@@ -346,6 +350,7 @@ ra_status ra_create(const ra_model_cfg* cfg, int32_t adapter_dim, ra_ctx** out) 
   int dh = g.hidden / g.n_heads;
   if (dh % 32 || dh > 128) return RA_ERR_SHAPE;
   if (g.arch == RA_ENCODER_POSTLN && (g.n_out > 32 || g.max_batch > 256)) return RA_ERR_SHAPE;
+  if (g.arch == RA_ENCODER_POSTLN_SPAN && (g.n_out != 2 || g.max_seq > SPAN_MAX_SEQ)) return RA_ERR_SHAPE;
   if (g.arch == RA_DECODER_PRENORM && ((g.dtype == RA_BF16 && g.n_out % 8) || g.head_trainable))
     return RA_ERR_SHAPE;
   ra_ctx* c = new ra_ctx;
@@ -361,6 +366,7 @@ ra_status ra_create(const ra_model_cfg* cfg, int32_t adapter_dim, ra_ctx** out) 
   c->max_depth = g.max_depth ? g.max_depth : g.n_layers;
   c->act = g.dtype == RA_BF16 ? DT_BF16 : DT_F32;
   c->dec = g.arch == RA_DECODER_PRENORM;
+  c->span = g.arch == RA_ENCODER_POSTLN_SPAN;
   c->depth = c->max_depth;
   c->set_mask.assign((size_t)(c->L + 1) * RA_P_COUNT, 0);
   plan(c);
@@ -654,8 +660,17 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     ctx->top_out = out_idx;
     out_idx ^= 1;
   }
-  // head: CLS token of the last block's output
   float* Ph = ctx->P() + (size_t)L * 4 * H * m;
+  if (ctx->span) {
+    // span head: start and end logits at every token of the last block's output
+    CU(prof(ctx, RA_PROF_HEAD, 4.0 * T * H, (double)T * H * dtype_size(act), st, [&] {
+      return span_head_fwd(xin, act, Ph, Ph + (size_t)2 * H, labels, B, S, H,
+                           ctx->ws<float>(ctx->h_rowloss), loss, logits, ctx->ws<float>(ctx->h_dlogits),
+                           ctx->ws<unsigned>(ctx->ws_err), st);
+    }));
+    return RA_OK;
+  }
+  // head: CLS token of the last block's output
   CU(prof(ctx, RA_PROF_HEAD, 2.0 * B * H * ctx->C, (double)B * H * dtype_size(act), st, [&] {
     return encoder_head_fwd(xin, act, Ph, Ph + (size_t)ctx->C * H, labels, B, S, H, ctx->C, loss,
                             logits, ctx->ws<float>(ctx->h_dlogits), ctx->ws<unsigned>(ctx->ws_err), st);
@@ -802,7 +817,18 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
   float* dY = ctx->ws<float>(ctx->b_dY[0]);
   int dyi = 0;
   // head
-  if (!ctx->dec) {
+  if (ctx->span) {
+    // every token receives a gradient: the span head writes all of dY
+    float* Ph = ctx->P() + (size_t)L * 4 * H * m;
+    float* Gh = ctx->G() + (size_t)L * 4 * H * m;
+    const void* yL = ctx->ws(ctx->s_X[ctx->top_out]);
+    CU(prof(ctx, RA_PROF_HEAD, 8.0 * T * H, (double)T * H * (dtype_size(act) + 4), st, [&] {
+      return span_head_bwd(yL, act, Ph, ctx->ws<float>(ctx->h_dlogits), B, S, H,
+                           ctx->cfg.head_trainable ? Gh : nullptr,
+                           ctx->cfg.head_trainable ? Gh + (size_t)2 * H : nullptr, dY,
+                           ctx->ws<float>(ctx->h_part), st);
+    }));
+  } else if (!ctx->dec) {
     float* Ph = ctx->P() + (size_t)L * 4 * H * m;
     float* Gh = ctx->G() + (size_t)L * 4 * H * m;
     CU(cudaMemsetAsync(dY, 0, (size_t)T * H * 4, st));

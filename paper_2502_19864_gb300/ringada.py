@@ -21,7 +21,7 @@ RA_OK, RA_ERR_ARG, RA_ERR_STATE, RA_ERR_NOT_SAVED, RA_ERR_SHAPE, RA_ERR_NOMEM, R
 STATUS_NAMES = {0: "RA_OK", 1: "RA_ERR_ARG", 2: "RA_ERR_STATE", 3: "RA_ERR_NOT_SAVED",
                 4: "RA_ERR_SHAPE", 5: "RA_ERR_NOMEM", 6: "RA_ERR_CUDA", 7: "RA_ERR_TIMEOUT",
                 8: "RA_ERR_UNSUPPORTED"}
-RA_ENCODER_POSTLN, RA_DECODER_PRENORM = 0, 1
+RA_ENCODER_POSTLN, RA_DECODER_PRENORM, RA_ENCODER_POSTLN_SPAN = 0, 1, 2
 RA_F32, RA_BF16 = 0, 1
 
 # ra_param ids (same order as the header's enum)

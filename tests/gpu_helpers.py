@@ -12,8 +12,14 @@ BF16_LOSS_TOL = 2e-2    # relative, loss; normwise, logits (bf16 models)
 BF16_GRAD_TOL = 5e-2    # normwise, per adapter/head gradient tensor (bf16 models)
 
 
+def ra_arch(cfg):
+    if cfg.arch == "decoder":
+        return R.RA_DECODER_PRENORM
+    return R.RA_ENCODER_POSTLN_SPAN if cfg.head == "span" else R.RA_ENCODER_POSTLN
+
+
 def ra_cfg(cfg, max_depth=0, max_batch=None, max_seq=None):
-    arch = R.RA_ENCODER_POSTLN if cfg.arch == "encoder" else R.RA_DECODER_PRENORM
+    arch = ra_arch(cfg)
     dt = R.RA_BF16 if cfg.dtype == "bf16" else R.RA_F32
     return R.make_cfg(arch, cfg.n_layers, cfg.hidden, cfg.n_heads, cfg.ffn, cfg.n_out,
                       max_batch or cfg.batch, max_seq or cfg.seq, dt, int(cfg.head_trainable),
@@ -35,7 +41,7 @@ class GpuRun:
         self.x = torch.tensor(w["x"], dtype=torch.float32).to(dt).cuda()
         self.labels = torch.tensor(w["labels"], dtype=torch.int32).cuda()
         self.loss = torch.zeros(1, dtype=torch.float32, device="cuda")
-        rows = cfg.batch if cfg.arch == "encoder" else cfg.tokens
+        rows = cfg.batch if (cfg.arch == "encoder" and cfg.head == "cls") else cfg.tokens
         self.logits = torch.zeros(rows, cfg.n_out, dtype=torch.float32, device="cuda") if want_logits else None
 
     @property
@@ -91,9 +97,19 @@ def rel_norm(a, b):
     return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
 
 
+# The span head's bias gets no gradient (a common shift of a sequence's start or end logits
+# leaves its softmax unchanged): the GPU's fp32 sum of dlogits must be zero up to rounding.
+SPAN_BIAS_GRAD_ABS = 1e-5
+
+
 def check_step(cfg, gpu_loss, gpu_logits, gpu_grads, gpu_head, ref, k):
     """Asserts the parity bar; returns the worst errors for reporting."""
     report = {}
+    if getattr(cfg, "head", "cls") == "span" and "bh" in gpu_head:
+        gpu_head = dict(gpu_head)
+        report["head_bh_abs"] = float(np.abs(gpu_head.pop("bh")).max())
+        assert report["head_bh_abs"] <= SPAN_BIAS_GRAD_ABS, report
+        assert np.abs(ref["head_grads"]["bh"]).max() <= 1e-14
     if cfg.dtype == "f32":
         report["loss"] = abs(gpu_loss - ref["loss"]) / abs(ref["loss"])
         assert report["loss"] <= F32_TOL, report

@@ -45,6 +45,12 @@ def test_create_validates_shapes(lib):
     assert e.value.status == R.RA_ERR_ARG
     with pytest.raises(R.RingAdaError):   # decoder head must be frozen
         R.ra_create(enc_cfg(arch=R.RA_DECODER_PRENORM, n_out=64, head_trainable=1), 16)
+    # the span head has exactly two outputs (start, end) and sequences of at most 4096
+    for bad in (dict(n_out=3), dict(n_out=2, max_seq=4097)):
+        with pytest.raises(R.RingAdaError) as e:
+            R.ra_create(enc_cfg(arch=R.RA_ENCODER_POSTLN_SPAN, **bad), 16)
+        assert e.value.status == R.RA_ERR_SHAPE
+    R.ra_destroy(R.ra_create(enc_cfg(arch=R.RA_ENCODER_POSTLN_SPAN, n_out=2), 16))
     ctx = R.ra_create(enc_cfg(), 16)
     R.ra_destroy(ctx)
 

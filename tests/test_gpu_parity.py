@@ -35,12 +35,12 @@ def _parity_all_depths(name, depths=None, seed=0):
     return reports
 
 
-@pytest.mark.parametrize("name", ["tiny", "mid_enc_f32", "tiny_dec"])
+@pytest.mark.parametrize("name", ["tiny", "mid_enc_f32", "tiny_dec", "tiny_span"])
 def test_fp32_parity_every_depth(name):
     _parity_all_depths(name)
 
 
-@pytest.mark.parametrize("name", ["small_enc_bf16", "small_dec_bf16"])
+@pytest.mark.parametrize("name", ["small_enc_bf16", "small_dec_bf16", "small_span_bf16"])
 def test_bf16_parity_every_depth(name):
     _parity_all_depths(name)
 
