@@ -360,7 +360,7 @@ def gpu_main(args):
     for d in SWEEP:
         if d != HEADLINE_D:
             sweep[d] = run.time_steps(d, steps, warmup)
-    # headline: timed region with the clock sampler running and the profiled graph
+    # headline: the plain graph timed with the clock sampler running
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
