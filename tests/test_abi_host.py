@@ -132,3 +132,39 @@ def test_schedule_depth_follows_the_unfreezing_rule():
     # Algorithm 1 / the sched workload: d = min(1 + floor(s / 50), 12)
     assert [R.schedule_depth(s) for s in (0, 49, 50, 99, 100, 549, 550, 599)] == \
         [1, 1, 2, 2, 3, 11, 12, 12]
+
+
+def _mb_set(sizes):
+    # every buffer of the plan starts on a 256-byte boundary
+    return sum((s + 255) // 256 * 256 for s in sizes)
+
+
+@pytest.mark.parametrize("arch", ["encoder", "decoder"])
+def test_saved_set_per_layer_is_the_backward_inputs(lib, arch):
+    """The activation arena holds, per unfrozen layer, exactly what the backward reads: the
+    lowest layer k keeps the adapter and norm inputs of its FFN half and the A adapter's
+    inputs (no attention backward runs there); every layer above also keeps q|k|v, the
+    attention output and the row log-sum-exp (and, decoder, its fp32 input and RMS scale).
+    Capacity = max_depth x the full set."""
+    B, S, H, heads, F, m = 4, 64, 256, 4, 1024, 32
+    T = B * S
+    es = 2  # bf16
+    if arch == "encoder":
+        cfg = dict(arch=R.RA_ENCODER_POSTLN, n_out=2)
+        lowest = [T * H * es, T * m * 4, T * H * es, T * 4, T * F * es, T * H * es, T * m * 4,
+                  T * H * es, T * 4]          # a, zA, xhat1, rstd1, GELU'(u), f, zF, xhat2, rstd2
+        full_only = [T * 3 * H * es, T * H * es, B * heads * S * 4]   # qkv, O, lse
+    else:
+        cfg = dict(arch=R.RA_DECODER_PRENORM, n_out=64, head_trainable=0)
+        lowest = [T * H * es, T * m * 4, T * H * 4, T * 4, T * 2 * F * es, T * H * es, T * m * 4]
+        #         a, zA, x1 (f32), rstd2, gate|up, f, zF
+        full_only = [T * H * 4, T * 4, T * 3 * H * es, T * H * es, B * heads * S * 4]
+        #            x_in (f32), rstd1, qkv, O, lse
+    full = _mb_set(lowest) + _mb_set(full_only)
+    caps = []
+    for md in (1, 3):
+        ctx = R.ra_create(enc_cfg(n_layers=3, hidden=H, n_heads=heads, ffn=F, max_batch=B,
+                                  max_seq=S, dtype=R.RA_BF16, max_depth=md, **cfg), m)
+        caps.append(R.ra_get_stats(ctx)["saved_bytes_capacity"])
+        R.ra_destroy(ctx)
+    assert caps == [full, 3 * full]
