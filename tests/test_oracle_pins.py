@@ -629,3 +629,22 @@ def test_planted_mistakes_are_caught(monkeypatch):
     monkeypatch.setattr(O, "layer_norm", unbiased_var)
     with pytest.raises(AssertionError):
         test_encoder_without_adapters_matches_torch_layer_bitwise_identity_invariant()
+
+    # span head: start and end labels swapped, or the two cross-entropies summed instead of
+    # averaged; the torch comparison and the finite differences must both notice
+    good_span = O.encoder_span_head
+    monkeypatch.setattr(O, "encoder_span_head",
+                        lambda y, head, labels, cfg: good_span(y, head, np.asarray(labels)[:, ::-1], cfg))
+    with pytest.raises(AssertionError):
+        test_span_head_matches_torch_autograd()
+
+    def summed(y, head, labels, cfg):
+        loss, logits, dy, g = good_span(y, head, labels, cfg)
+        return 2 * loss, logits, dy, g
+    monkeypatch.setattr(O, "encoder_span_head", summed)
+    with pytest.raises(AssertionError):
+        test_span_head_matches_torch_autograd()
+    with pytest.raises(AssertionError):
+        cfg = synth.CONFIGS["tiny_span"]
+        _fd_check(cfg, synth.make_workload(cfg, 0), d=1, n_coords=4, zero_keys=("bh",))
+    monkeypatch.setattr(O, "encoder_span_head", good_span)
