@@ -208,7 +208,9 @@ def cross_entropy(logits, labels):
 # ----------------------------------------------------------------------------------------
 
 def encoder_layer_forward(x, P, cfg, adapters=True):
-    """Post-LN encoder block; adapters on the attention-output and FFN-output branches."""
+    """Post-LN encoder block; adapters on the attention-output and FFN-output branches
+    (Houlsby placement), or, with ``cfg.adapters == "paper"``, the single adapter of Fig. 1
+    after the FFN add & LayerNorm: out = y2 + sigma(y2 W_down) W_up (Eq. 1 on y2)."""
     B, S, H, nh = cfg.batch, cfg.seq, cfg.hidden, cfg.n_heads
     qkv = x @ P["Wqkv"].T + P["bqkv"]
     q = split_heads(qkv[:, :H], B, S, nh)
@@ -216,6 +218,17 @@ def encoder_layer_forward(x, P, cfg, adapters=True):
     v = split_heads(qkv[:, 2 * H:], B, S, nh)
     O, p = attention(q, k, v, causal=False)
     a = merge_heads(O) @ P["Wo"].T + P["bo"]
+    if getattr(cfg, "adapters", "houlsby") == "paper":
+        y1, ln1 = layer_norm(x + a, P["ln1_g"], P["ln1_b"], cfg.norm_eps)
+        u = y1 @ P["W1"].T + P["b1"]
+        f = gelu(u) @ P["W2"].T + P["b2"]
+        y2, ln2 = layer_norm(y1 + f, P["ln2_g"], P["ln2_b"], cfg.norm_eps)
+        if adapters:
+            out, zF = adapter_forward(y2, P["WdF"], P["WuF"])
+        else:
+            out, zF = y2, None
+        cache = dict(q=q, k=k, v=v, p=p, ln1=ln1, u=u, y2=y2, zF=zF, ln2=ln2)
+        return out, cache
     if adapters:
         a2, zA = adapter_forward(a, P["WdA"], P["WuA"])
     else:
@@ -234,8 +247,22 @@ def encoder_layer_forward(x, P, cfg, adapters=True):
 
 def encoder_layer_backward(dy, P, c, cfg, lowest):
     """Reverse mode through one encoder block.  At the lowest unfrozen layer it stops after
-    the attention-branch adapter's weight gradients (no gradient into the block input)."""
+    the attention-branch adapter's weight gradients (no gradient into the block input); with
+    the paper's single adapter it stops right after that adapter's weight gradients."""
     grads = {}
+    if getattr(cfg, "adapters", "houlsby") == "paper":
+        dy2, grads["WdF"], grads["WuF"] = adapter_backward(dy, c["y2"], c["zF"], P["WdF"], P["WuF"],
+                                                           need_dh=not lowest)
+        if lowest:
+            return None, grads
+        ds2 = layer_norm_backward(dy2, P["ln2_g"], c["ln2"])
+        du = (ds2 @ P["W2"]) * gelu_grad(c["u"])
+        dy1 = ds2 + du @ P["W1"]
+        ds1 = layer_norm_backward(dy1, P["ln1_g"], c["ln1"])
+        dO = split_heads(ds1 @ P["Wo"], cfg.batch, cfg.seq, cfg.n_heads)
+        dq, dk, dv = attention_backward(dO, c["q"], c["k"], c["v"], c["p"])
+        dqkv = np.concatenate([merge_heads(dq), merge_heads(dk), merge_heads(dv)], axis=1)
+        return ds1 + dqkv @ P["Wqkv"], grads
     ds2 = layer_norm_backward(dy, P["ln2_g"], c["ln2"])
     df, grads["WdF"], grads["WuF"] = adapter_backward(ds2, c["f"], c["zF"], P["WdF"], P["WuF"])
     du = (df @ P["W2"]) * gelu_grad(c["u"])

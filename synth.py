@@ -45,6 +45,8 @@ class ModelCfg:
     rope_theta: float = 10000.0
     head: str = "cls"    # encoder head: "cls" (position 0, n_out classes) | "span" (start/end
                          # logits at every position, n_out = 2)
+    adapters: str = "houlsby"  # encoder: "houlsby" (attention- and FFN-branch adapters) |
+                               # "paper" (one adapter after the FFN add & LayerNorm, Fig. 1)
 
     @property
     def head_dim(self) -> int:
@@ -61,6 +63,10 @@ def _enc(L, H, h, F, m, B, S, dtype, C=2):
 
 def _span(L, H, h, F, m, B, S, dtype):
     return ModelCfg("encoder", L, H, h, F, m, 2, B, S, dtype, True, 1e-12, head="span")
+
+
+def _paper(L, H, h, F, m, B, S, dtype):
+    return ModelCfg("encoder", L, H, h, F, m, 2, B, S, dtype, True, 1e-12, adapters="paper")
 
 
 def _dec(L, H, h, F, m, V, B, S, dtype):
@@ -81,6 +87,8 @@ CONFIGS: Dict[str, ModelCfg] = {
     # span (start/end) head over every token, the shape of extractive question answering
     "tiny_span": _span(2, 128, 2, 512, 16, 4, 32, "f32"),
     "small_span_bf16": _span(3, 256, 4, 1024, 32, 3, 100, "bf16"),
+    # the paper's placement: one adapter per block, after the FFN add & LayerNorm
+    "tiny_paper": _paper(2, 128, 2, 512, 16, 4, 32, "f32"),
 }
 
 
@@ -92,7 +100,14 @@ ADAPTER_KEYS = ["WdA", "WuA", "WdF", "WuF"]
 
 
 def layer_keys(cfg: ModelCfg) -> List[str]:
+    if cfg.arch == "encoder" and cfg.adapters == "paper":
+        return [k for k in ENCODER_LAYER_KEYS if k not in ("WdA", "WuA")]
     return ENCODER_LAYER_KEYS if cfg.arch == "encoder" else DECODER_LAYER_KEYS
+
+
+def adapter_keys(cfg: ModelCfg) -> List[str]:
+    """The trainable adapter matrices of one block."""
+    return ["WdF", "WuF"] if cfg.arch == "encoder" and cfg.adapters == "paper" else ADAPTER_KEYS
 
 
 def head_keys(cfg: ModelCfg) -> List[str]:

@@ -281,7 +281,8 @@ def _stress_workload(cfg, seed=0, up_std=0.05):
     r = rng(100 + seed)
     for p in w["layers"]:
         for key in ("WuA", "WuF"):
-            p[key] = r.normal(size=p[key].shape) * up_std
+            if key in p:
+                p[key] = r.normal(size=p[key].shape) * up_std
     return w
 
 
@@ -312,6 +313,48 @@ def test_encoder_stack_matches_torch_layers_with_autograd():
             g = par.grad.numpy()
             err = np.linalg.norm(res["grads"][l][key] - g) / np.linalg.norm(g)
             assert err < 1e-10, (l, key, err)
+
+
+def test_paper_placement_matches_torch_layers_with_autograd():
+    """The paper's single adapter per block (Fig. 1, after the FFN add & LayerNorm): torch's
+    TransformerEncoderLayer without adapters, followed by Eq. 1 on its output, under
+    autograd; and the early-stopped backward equals the full one above k, bitwise."""
+    import dataclasses
+    cfg = dataclasses.replace(_small_enc_cfg(), adapters="paper")
+    w = _stress_workload(cfg)
+    layers, head = O.to_f64_params(w["layers"], w["head"])
+    res = O.step(cfg, layers, head, w["x"], w["labels"], cfg.n_layers)
+    mods = [_torch_encoder_layer(cfg, P, adapters=False) for P in layers]
+    ad = [(T(P["WdF"], True), T(P["WuF"], True)) for P in layers]
+    Wh, bh = T(head["Wh"], True), T(head["bh"], True)
+    h = T(w["x"])
+    for m, (Wd, Wu) in zip(mods, ad):
+        y = m(h)
+        h = y + Fnn.gelu(y @ Wd) @ Wu
+    logits = h[:, 0, :] @ Wh.T + bh
+    loss = Fnn.cross_entropy(logits, torch.tensor(w["labels"]).long())
+    loss.backward()
+    assert res["loss"] == pytest.approx(loss.item(), rel=1e-12)
+    np.testing.assert_allclose(res["logits"], logits.detach().numpy(), rtol=1e-11, atol=1e-13)
+    np.testing.assert_allclose(res["head_grads"]["Wh"], Wh.grad.numpy(), rtol=1e-9, atol=1e-14)
+    for l, (Wd, Wu) in enumerate(ad):
+        assert sorted(res["grads"][l]) == ["WdF", "WuF"]
+        for key, par in (("WdF", Wd), ("WuF", Wu)):
+            g = par.grad.numpy()
+            err = np.linalg.norm(res["grads"][l][key] - g) / np.linalg.norm(g)
+            assert err < 1e-10, (l, key, err)
+    for d in range(1, cfg.n_layers):
+        r = O.step(cfg, layers, head, w["x"], w["labels"], d)
+        assert sorted(r["grads"]) == list(range(cfg.n_layers - d, cfg.n_layers))
+        for l in r["grads"]:
+            for key in ("WdF", "WuF"):
+                np.testing.assert_array_equal(r["grads"][l][key], res["grads"][l][key])
+
+
+def test_fd_tiny_paper_placement():
+    cfg = synth.CONFIGS["tiny_paper"]
+    _fd_check(cfg, synth.make_workload(cfg, 0), d=1, n_coords=24)
+    _fd_check(cfg, _stress_workload(cfg, 3), d=cfg.n_layers, n_coords=12)
 
 
 def test_encoder_without_adapters_matches_torch_layer_bitwise_identity_invariant():
@@ -394,7 +437,7 @@ def _fd_check(cfg, w, d, n_coords=48, eps=1e-2, tol=1e-6, seed=0, zero_keys=()):
         return O.forward(cfg, layers, head, None, w["labels"], d, start_layer=k, h0=h_k)["loss"]
 
     r = rng(seed)
-    targets = [(l, key) for l in range(k, cfg.n_layers) for key in synth.ADAPTER_KEYS]
+    targets = [(l, key) for l in range(k, cfg.n_layers) for key in synth.adapter_keys(cfg)]
     if cfg.head_trainable:
         targets += [("head", key) for key in ("Wh", "bh")]
     for l, key in targets:
