@@ -421,6 +421,105 @@ def test_decoder_branch_wiring_special_cases():
 
 
 # ----------------------------------------------------------------------------------------
+# decoder block wiring: closed forms and properties a wrong wiring breaks
+# ----------------------------------------------------------------------------------------
+
+def _dec_block(seed=3, up_std=0.3):
+    cfg = synth.CONFIGS["tiny_dec"]
+    w = _stress_workload(cfg, seed, up_std=up_std)
+    P = O.to_f64_params(w["layers"], w["head"])[0][0]
+    cs = O.rope_tables(cfg.seq, cfg.head_dim, cfg.rope_theta)
+    x = O.f64(w["x"]).reshape(cfg.tokens, cfg.hidden)
+    return cfg, P, cs, x
+
+
+def _dec_out(x, P, cfg, cs):
+    # through the module attribute, so that a planted replacement is what runs
+    return O.decoder_layer_forward(x, P, cfg, cs)[0]
+
+
+def test_decoder_norm_gains_zero_close_each_branch():
+    """Pre-norm wiring: every projection of a branch reads that branch's RMSNorm output.
+    With the first gain zero, q = k = v = 0, so the attention branch and its adapter give
+    exactly zero and the block (with the down projection zero too) is the identity; with
+    the second gain zero, gate = up = 0 and the block output is x1, the same as with the
+    down projection zero."""
+    cfg, P, cs, x = _dec_block()
+    Q = {k: v.copy() for k, v in P.items()}
+    Q["rms1_g"][:] = 0.0
+    Q["Wd"][:] = 0.0
+    np.testing.assert_array_equal(_dec_out(x, Q, cfg, cs), x)
+    Q = {k: v.copy() for k, v in P.items()}
+    Q["rms2_g"][:] = 0.0
+    R = {k: v.copy() for k, v in P.items()}
+    R["Wd"][:] = 0.0
+    y_gain0, y_down0 = _dec_out(x, Q, cfg, cs), _dec_out(x, R, cfg, cs)
+    np.testing.assert_array_equal(y_gain0, y_down0)
+    assert np.abs(y_gain0 - x).max() > 1e-3       # the attention branch is live
+
+
+def test_decoder_uniform_causal_attention_closed_form():
+    """With Wq = Wk = 0 every score is zero, so causal attention averages the values of
+    positions 0..t.  With Wo = I, no attention-branch adapter and Wd = 0 the block output
+    minus its input is that running mean of RMSNorm(x) Wv^T (torch's rms_norm)."""
+    cfg, P, cs, x = _dec_block()
+    H, B, S = cfg.hidden, cfg.batch, cfg.seq
+    P["Wq"][:] = 0.0
+    P["Wk"][:] = 0.0
+    P["Wo"][:] = np.eye(H)
+    P["WuA"][:] = 0.0
+    P["Wd"][:] = 0.0
+    n1 = Fnn.rms_norm(T(x), (H,), T(P["rms1_g"]), eps=cfg.norm_eps).numpy()
+    v = (n1 @ P["Wv"].T).reshape(B, S, H)
+    mean = np.cumsum(v, axis=1) / np.arange(1, S + 1)[None, :, None]
+    np.testing.assert_allclose(_dec_out(x, P, cfg, cs) - x, mean.reshape(B * S, H),
+                               rtol=1e-10, atol=1e-12)
+
+
+def test_decoder_block_is_causal():
+    """Changing the inputs at positions > t leaves every output at positions <= t
+    unchanged (the mask hides the future), while the later outputs do change."""
+    cfg, P, cs, x = _dec_block()
+    B, S, H = cfg.batch, cfg.seq, cfg.hidden
+    y = _dec_out(x, P, cfg, cs).reshape(B, S, H)
+    t = S // 3
+    x2 = x.reshape(B, S, H).copy()
+    x2[:, t + 1:, :] += rng(9).normal(size=x2[:, t + 1:, :].shape)
+    y2 = _dec_out(x2.reshape(B * S, H), P, cfg, cs).reshape(B, S, H)
+    np.testing.assert_allclose(y2[:, :t + 1], y[:, :t + 1], rtol=1e-12, atol=1e-13)
+    assert np.abs(y2[:, t + 1:] - y[:, t + 1:]).max() > 1e-2
+
+
+def test_decoder_branches_are_scale_invariant():
+    """RMSNorm(c x) = RMSNorm(x) for c > 0 (up to eps, 1e-6 against a mean square near 1),
+    so a branch whose projections all read its norm output adds the same increment for x
+    and for 3x: with Wd = 0 the attention branch, with Wo = 0 the FFN branch."""
+    cfg, P, cs, x = _dec_block()
+    for zero in ("Wd", "Wo"):
+        Q = {k: v.copy() for k, v in P.items()}
+        Q[zero][:] = 0.0
+        inc1 = _dec_out(x, Q, cfg, cs) - x
+        inc3 = _dec_out(3.0 * x, Q, cfg, cs) - 3.0 * x
+        assert np.abs(inc1).max() > 1e-3
+        np.testing.assert_allclose(inc3, inc1, rtol=1e-5, atol=1e-5 * np.abs(inc1).max())
+
+
+def test_decoder_heads_are_separable():
+    """Multi-head attention: head h's output depends only on head h's rows of Wq, Wk and
+    Wv (RoPE rotates pairs inside one head).  With Wo reading head 0 only and Wd = 0,
+    redrawing the other heads' projection rows leaves the block output unchanged."""
+    cfg, P, cs, x = _dec_block()
+    dh = cfg.head_dim
+    P["Wo"][:, dh:] = 0.0
+    P["Wd"][:] = 0.0
+    y = _dec_out(x, P, cfg, cs)
+    r = rng(11)
+    for key in ("Wq", "Wk", "Wv"):
+        P[key][dh:, :] = r.normal(size=P[key][dh:, :].shape) * 0.2
+    np.testing.assert_allclose(_dec_out(x, P, cfg, cs), y, rtol=1e-12, atol=1e-13)
+
+
+# ----------------------------------------------------------------------------------------
 # finite differences (brute force) on the tiny configs
 # ----------------------------------------------------------------------------------------
 
@@ -691,3 +790,70 @@ def test_planted_mistakes_are_caught(monkeypatch):
         cfg = synth.CONFIGS["tiny_span"]
         _fd_check(cfg, synth.make_workload(cfg, 0), d=1, n_coords=4, zero_keys=("bh",))
     monkeypatch.setattr(O, "encoder_span_head", good_span)
+
+    # decoder block wiring: q or v projected from x instead of RMSNorm(x), gate/up fed by
+    # x1 instead of RMSNorm(x1), the causal mask reversed, RoPE applied across the merged
+    # heads; each fails one of the wiring pins
+    good_dec = O.decoder_layer_forward
+    x_case = _dec_block()
+    np.testing.assert_array_equal(_decoder_variant(None)(*_dec_args(x_case))[0],
+                                  good_dec(*_dec_args(x_case))[0])
+    wiring_pins = (test_decoder_norm_gains_zero_close_each_branch,
+                   test_decoder_uniform_causal_attention_closed_form,
+                   test_decoder_block_is_causal,
+                   test_decoder_branches_are_scale_invariant,
+                   test_decoder_heads_are_separable)
+    for mistake in ("q_from_x", "v_from_x", "gate_up_from_x1", "mask_reversed", "rope_merged"):
+        monkeypatch.setattr(O, "decoder_layer_forward", _decoder_variant(mistake))
+        failed = 0
+        for pin in wiring_pins:
+            try:
+                pin()
+            except AssertionError:
+                failed += 1
+        assert failed >= 1, mistake
+        monkeypatch.setattr(O, "decoder_layer_forward", good_dec)
+
+
+def _dec_args(case):
+    cfg, P, cs, x = case
+    return x, P, cfg, cs
+
+
+def _decoder_variant(mistake):
+    """The oracle's decoder block forward restated with one wiring mistake planted (None:
+    no mistake, which must equal the oracle bitwise)."""
+    def fwd(x, P, cfg, rope_cs, adapters=True):
+        B, S, nh, H = cfg.batch, cfg.seq, cfg.n_heads, cfg.hidden
+        cos, sin = rope_cs
+        n1, rms1 = O.rms_norm(x, P["rms1_g"], cfg.norm_eps)
+        qin = x if mistake == "q_from_x" else n1
+        vin = x if mistake == "v_from_x" else n1
+        if mistake == "rope_merged":
+            # rotate-half pairs (i, i + H/2) across the whole row, before the head split
+            ang_q = O.rope(np.stack([qin @ P["Wq"].T]), *O.rope_tables(B * S, H, cfg.rope_theta))[0]
+            ang_k = O.rope(np.stack([n1 @ P["Wk"].T]), *O.rope_tables(B * S, H, cfg.rope_theta))[0]
+            q = O.split_heads(ang_q, B, S, nh)
+            k = O.split_heads(ang_k, B, S, nh)
+        else:
+            q = O.rope(O.split_heads(qin @ P["Wq"].T, B, S, nh), cos, sin)
+            k = O.rope(O.split_heads(n1 @ P["Wk"].T, B, S, nh), cos, sin)
+        v = O.split_heads(vin @ P["Wv"].T, B, S, nh)
+        if mistake == "mask_reversed":
+            Of, p = O.attention(q[:, :, ::-1], k[:, :, ::-1], v[:, :, ::-1], causal=True)
+            Oo, p = Of[:, :, ::-1], p[:, :, ::-1, ::-1]
+        else:
+            Oo, p = O.attention(q, k, v, causal=True)
+        a = O.merge_heads(Oo) @ P["Wo"].T
+        a2, zA = O.adapter_forward(a, P["WdA"], P["WuA"]) if adapters else (a, None)
+        x1 = x + a2
+        n2, rms2 = O.rms_norm(x1, P["rms2_g"], cfg.norm_eps)
+        fin = x1 if mistake == "gate_up_from_x1" else n2
+        gate = fin @ P["Wg"].T
+        up = fin @ P["Wu"].T
+        f = (O.silu(gate) * up) @ P["Wd"].T
+        f2, zF = O.adapter_forward(f, P["WdF"], P["WuF"]) if adapters else (f, None)
+        cache = dict(rms1=rms1, q=q, k=k, v=v, p=p, a=a, zA=zA, rms2=rms2, gate=gate, up=up,
+                     f=f, zF=zF)
+        return x1 + f2, cache
+    return fwd
