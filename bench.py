@@ -1,12 +1,14 @@
 #!/usr/bin/env python
 """Throughput of the adapter fine-tuning step (forward, loss, early-stopped backward, Adam)
-on the BERT-base-shaped workload, versus the unfreezing depth d (k = L - d).
+on the BERT-large-shaped workload, versus the unfreezing depth d (k = L - d).
 
 One "step" is ra_forward + ra_backward_truncated(k) + ra_adapter_update over one batch of
-32 x 128 synthetic tokens, replayed from a CUDA graph; inputs are resident in HBM when the
-timed region starts.  The headline is samples/s at d = 6 (a frozen prefix of 6 blocks plus
-a 6-block backward); the sweep over d = 1, 3, 6, 12 is in "sweep".  The step streams more
-than 1 GB per call, far above the 129 MB L2, so no flush is needed between steps.
+32 x 256 synthetic tokens (24 layers, H 1024, 16 heads, FFN 4096, adapters m 64), replayed
+from a CUDA graph; inputs are resident in HBM when the timed region starts.  The headline
+is samples/s at d = 12 (a frozen prefix of 12 blocks plus a 12-block backward); the sweep
+over d = 1, 6, 12, 24 is in "sweep", and the BERT-base-shaped sweep (d = 1, 3, 6, 12) in
+"base".  A step streams several GB, far above the 129 MB L2, so no flush is needed
+between steps.
 
   python bench.py [--gpus N --steps K --warmup W]      # the CUDA path (one JSON line)
   python bench.py --impl reference ...                 # the fp64 oracle on the host cores
@@ -30,12 +32,14 @@ sys.path.insert(0, ROOT)
 
 METRIC = "fine-tune samples/sec vs unfrozen depth k"
 UNIT = "samples/s"
-HEADLINE_D = 6
-SWEEP = [1, 3, 6, 12]
-# other workloads (--config): depth sweep and headline depth of each
+DEFAULT_CONFIG = "large"
+# workloads (--config): depth sweep and headline depth of each
 SWEEPS = {"base": ([1, 3, 6, 12], 6), "large": ([1, 6, 12, 24], 12), "llama": ([4], 4),
           "tiny": ([1, 2], 1)}
-CPU_SAMPLE_BATCH = 2      # sequences of 128 tokens per oracle step (bounded CPU sample)
+HEADLINE_D = 12
+SWEEP = [1, 6, 12, 24]
+# sequences per oracle step in the bounded CPU sample of each workload
+CPU_SAMPLE_BATCH = {"base": 2, "large": 1, "llama": 1, "tiny": 4}
 
 
 def parse():
@@ -44,8 +48,8 @@ def parse():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", default="base")
-    ap.add_argument("--no-large", action="store_true", help="skip the BERT-large GEMM check")
+    ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--no-extra", action="store_true", help="skip the BERT-base sweep")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--schedule", action="store_true",
                     help="run the 600-step top-down unfreezing schedule on the BERT-base workload")
@@ -97,18 +101,33 @@ def run_cpu_baseline(cfg_name, depth, batch, seconds):
     res = json.loads(r.stdout.strip().splitlines()[-1])
     return {"value": res["rate"], "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": "%d oracle steps (fp64 numpy, BLAS on %d threads) of %s at d=%d on %d of "
-                      "the 32 sequences, %.1f s" % (res["steps"], cores, cfg_name, depth, batch,
-                                                   res["seconds"])}
+                      "the batch's sequences, %.1f s" % (res["steps"], cores, cfg_name, depth, batch,
+                                                        res["seconds"])}
+
+
+def workload_config(name, depth, world=1):
+    """The `config` object of the JSON line: the same for the CUDA arm and the reference arm."""
+    import synth
+    cfg = synth.CONFIGS[name]
+    return {"workload": "%s-shaped adapter step (%d layers, H %d, %d heads, FFN %d, adapters "
+                        "m %d, batch %d x %d), d=%d" % (name, cfg.n_layers, cfg.hidden, cfg.n_heads,
+                                                         cfg.ffn, cfg.adapter_dim, cfg.batch,
+                                                         cfg.seq, depth),
+            "global_batch": cfg.batch * world, "seq_len": cfg.seq, "depth": depth,
+            "parallelism": "replicas" if world > 1 else "single",
+            "l2": "inputs larger than L2 (several GB streamed per step)"}
 
 
 def reference_main(args):
     _, rank, _ = rank_env()
     if rank != 0:
         return 0
+    global SWEEP, HEADLINE_D
+    SWEEP, HEADLINE_D = SWEEPS[args.config]
     import synth
     cfg = synth.CONFIGS[args.config]
     cores = os.cpu_count() or 1
-    # warm-up and timed oracle steps, each a bounded sample (CPU_SAMPLE_BATCH sequences)
+    # warm-up and timed oracle steps, each a bounded sample (one sequence of the batch)
     oracle_sample_rate(args.config, HEADLINE_D, 1, 0, steps=max(1, min(args.warmup, 2)))
     rate, n, el = oracle_sample_rate(args.config, HEADLINE_D, 1, 0, steps=args.steps)
     line = {
@@ -116,11 +135,10 @@ def reference_main(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * el / n,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": "bert-base-shaped adapter step, d=%d (one of 32 sequences per "
-                               "oracle step)" % HEADLINE_D, "batch": 1, "seq_len": cfg.seq,
-                   "layers": cfg.n_layers, "hidden": cfg.hidden},
+        "config": workload_config(args.config, HEADLINE_D, args.gpus),
         "cpu_baseline": {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
-                         "sample": "%d fp64 oracle steps on 1 sequence of 128 tokens" % n},
+                         "sample": "%d fp64 oracle steps, each on 1 of the %d sequences of %d "
+                                   "tokens (samples/s = sequences per second)" % (n, cfg.batch, cfg.seq)},
         "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
@@ -131,14 +149,18 @@ def reference_main(args):
 # GPU leg
 # ---------------------------------------------------------------------------------------
 
+CLOCK_FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
 def start_clock_sampler(index):
+    """nvidia-smi sampling every 50 ms for the whole GPU-timed part of the run; the samples
+    carry timestamps so each timed region gets its own record (clock_record)."""
     path = tempfile.mktemp(prefix="clocks_", suffix=".csv")
-    q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
-         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
     try:
         f = open(path, "w")
-        p = subprocess.Popen(["nvidia-smi", "-i", str(index), "--query-gpu=" + q,
+        p = subprocess.Popen(["nvidia-smi", "-i", str(index), "--query-gpu=" + CLOCK_FIELDS,
                               "--format=csv,noheader,nounits", "-lms", "50"], stdout=f,
                              stderr=subprocess.DEVNULL)
         return p, f, path
@@ -147,29 +169,47 @@ def start_clock_sampler(index):
 
 
 def stop_clock_sampler(h):
+    """Stops the sampler; returns the samples as (unix time, sm MHz, max MHz, reasons)."""
+    import datetime
     p, f, path = h
     if p is None:
-        return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        return None
     p.terminate()
     p.wait(timeout=10)
     f.close()
-    sm, smax, reasons = [], None, set()
     names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    out = []
     for line in open(path):
         parts = [x.strip() for x in line.split(",")]
-        if len(parts) < 9:
+        if len(parts) < 10:
             continue
         try:
-            sm.append(float(parts[1]))
-            smax = float(parts[2])
+            ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+            sm, smax = float(parts[2]), float(parts[3])
         except ValueError:
             continue
-        for nm, v in zip(names, parts[5:9]):
-            if v.lower() == "active":
-                reasons.add(nm)
+        out.append((ts, sm, smax, {nm for nm, v in zip(names, parts[6:10]) if v.lower() == "active"}))
     os.unlink(path)
-    return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
-            "reasons": sorted(reasons), "samples": len(sm)}
+    return out
+
+
+def clock_record(samples, t0=None, t1=None):
+    """Median SM clock, max clock and active throttle reasons of the samples in [t0, t1]
+    (all samples without a window; the nearest sample when a region is shorter than the
+    sampling period)."""
+    if samples is None:
+        return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+    sel = [s for s in samples if (t0 is None or s[0] >= t0) and (t1 is None or s[0] <= t1)]
+    if not sel and samples and t0 is not None:
+        mid = 0.5 * (t0 + t1)
+        sel = [min(samples, key=lambda s: abs(s[0] - mid))]
+    if not sel:
+        return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+    reasons = set()
+    for s in sel:
+        reasons |= s[3]
+    return {"sm_mhz": statistics.median(s[1] for s in sel), "sm_max_mhz": max(s[2] for s in sel),
+            "reasons": sorted(reasons), "samples": len(sel)}
 
 
 def measured_peaks():
@@ -323,6 +363,17 @@ def job_value(world, batch, ms):
     return world * batch / (ms / 1000.0)
 
 
+def gemm_rate(prof, peaks):
+    """GEMM throughput of one step from the profiled pass, against the measured peaks."""
+    g = prof.get("gemm")
+    if not g or g["ms"] <= 0:
+        return None
+    tf = g["flops"] / (g["ms"] / 1000.0) / 1e12
+    return {"tflops": tf, "frac_burst": tf / peaks["bf16_tflops"],
+            "frac_sustained": tf / peaks["bf16_tflops_sustained"], "calls": g["calls"],
+            "flops": g["flops"], "ms": g["ms"]}
+
+
 def gpu_main(args):
     import torch
     import synth
@@ -349,32 +400,42 @@ def gpu_main(args):
     # CPU baseline first (its own process, before the GPU work starts)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = run_cpu_baseline(args.config, HEADLINE_D, 1 if cfg.batch < CPU_SAMPLE_BATCH else CPU_SAMPLE_BATCH, 12.0)
+        cpu = run_cpu_baseline(args.config, HEADLINE_D,
+                               min(cfg.batch, CPU_SAMPLE_BATCH.get(args.config, 1)), 12.0)
 
     run = Runner(cfg, max(SWEEP), device)
     sweep = {}
     for d in SWEEP:
         run.capture(d)
     run.capture(HEADLINE_D, profile=True)
+    # the clock sampler runs through every timed region; each region keeps its window
+    clk = start_clock_sampler(torch.cuda.current_device())
+    windows = {}
     # sweep points (not the headline)
     for d in SWEEP:
         if d != HEADLINE_D:
+            t0 = time.time()
             sweep[d] = run.time_steps(d, steps, warmup)
-    # headline: the plain graph timed with the clock sampler running
+            windows["d=%d" % d] = (t0, time.time())
+    # headline: the plain graph
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
-    clk = start_clock_sampler(torch.cuda.current_device())
+    t0 = time.time()
     ms = run.time_steps(HEADLINE_D, steps, warmup)
-    clocks = stop_clock_sampler(clk)
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
+    windows["headline"] = (t0, time.time())
     sweep[HEADLINE_D] = ms
+    t0 = time.time()
     e2e_ms, h2d, d2h = run.time_e2e(HEADLINE_D, steps)
-    # per-kernel device times: a second timed region, the same step with an event around
+    windows["e2e"] = (t0, time.time())
+    # per-kernel device times: a further timed region, the same step with an event around
     # every kernel (replays of the profiled graph)
+    t0 = time.time()
     prof = run.kernel_times(HEADLINE_D, min(steps, 50))
+    windows["kernel_times"] = (t0, time.time())
     launches_headline = run.launches[HEADLINE_D]
     saved_by_d = dict(run.saved)
     R.ra_set_unfrozen_depth(run.model.ctx, HEADLINE_D)
@@ -387,32 +448,43 @@ def gpu_main(args):
 
     B = cfg.batch
     value = job_value(world, B, ms)
-    g = prof["gemm"]
-    gemm_tflops = g["flops"] / (g["ms"] / 1000.0) / 1e12 if g["ms"] > 0 else None
+    gr = gemm_rate(prof, peaks)
     traffic_per_flop, traffic_note = gemm_traffic()
+    g = prof["gemm"]
     launches_per_gemm = max(1, g["calls"])
     roof = {
         "kernel": "frozen-weight and dX GEMMs (tcgen05, bf16 in, fp32 accumulate), all launches of one step",
         "bound": "tensor", "unit": "TFLOP/s",
-        "achieved": gemm_tflops,
-        "peak": peaks["bf16_tflops_sustained"],
-        "peak_kind": "%s bf16 sustained (kernel timed inside a long step)" % peak_kind,
-        "frac": (gemm_tflops / peaks["bf16_tflops_sustained"]) if gemm_tflops else None,
+        "achieved": gr["tflops"] if gr else None,
+        "peak": peaks["bf16_tflops"],
+        "peak_kind": "%s dense bf16 burst (cuBLAS GEMM timed alone; the SM clock stays at its maximum "
+                     "through this step)" % peak_kind,
+        "frac": gr["frac_burst"] if gr else None,
+        "frac_of_sustained": gr["frac_sustained"] if gr else None,
+        "peak_sustained": peaks["bf16_tflops_sustained"],
         "launches": g["calls"],
         "flops_per_launch": g["flops"] / launches_per_gemm,
         "traffic": (traffic_per_flop * g["flops"] / launches_per_gemm) if traffic_per_flop else None,
         "traffic_note": traffic_note,
+        "timing": "each GEMM launch between its own pair of CUDA events (profiled replay of the step graph)",
     }
     phases = {k: {"ms": v["ms"], "calls": v["calls"],
                   "tflops": (v["flops"] / v["ms"] / 1e9) if v["ms"] > 0 and v["flops"] else None,
                   "gbs": (v["bytes"] / v["ms"] / 1e6) if v["ms"] > 0 and v["bytes"] else None}
               for k, v in prof.items()}
+    phases_sum = sum(v["ms"] for v in prof.values())
 
-    large = None
-    if rank == 0 and not args.no_large and args.config == "base":
+    extra = None
+    if rank == 0 and not args.no_extra and args.config == "large":
         del run
         torch.cuda.empty_cache()
-        large = large_gemm_check(torch, R, synth, device, peaks)
+        extra = base_sweep(torch, R, synth, device, peaks, steps, warmup, windows)
+    samples = stop_clock_sampler(clk)
+    clocks = clock_record(samples, *windows["headline"])
+    clocks["whole_run"] = clock_record(samples, min(w[0] for w in windows.values()),
+                                       max(w[1] for w in windows.values()))
+    clocks["by_region"] = {k: clock_record(samples, *w) for k, w in windows.items()
+                           if k != "headline"}
 
     if rank != 0:
         if dist:
@@ -422,14 +494,7 @@ def gpu_main(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
         "warmup": warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
-        "config": {"workload": "%s-shaped adapter step (%d layers, H %d, %d heads, FFN %d, adapters "
-                               "m %d, batch %d x %d), d=%d" % (args.config, cfg.n_layers, cfg.hidden,
-                                                                cfg.n_heads, cfg.ffn, cfg.adapter_dim,
-                                                                cfg.batch, cfg.seq, HEADLINE_D),
-                   "global_batch": B * world, "seq_len": cfg.seq, "depth": HEADLINE_D,
-                   "parallelism": "replicas" if world > 1 else "single",
-                   "l2": "inputs larger than L2 (>1 GB streamed per step)",
-                   "cuda_graph": True},
+        "config": dict(workload_config(args.config, HEADLINE_D, world), cuda_graph=True),
         "sweep": {"d=%d" % d: {"samples_per_s": job_value(world, B, sweep[d]),
                                "ms_per_step": sweep[d], "k": cfg.n_layers - d,
                                "saved_activation_bytes": saved_by_d[d]}
@@ -438,13 +503,16 @@ def gpu_main(args):
         "saved_bytes_at_headline": saved_by_d[HEADLINE_D],
         "roofline": roof,
         "phases_ms": phases,
+        "phases_note": "per-kernel times from the profiled replay (an event pair around every "
+                       "kernel removes the launch overlap); their sum is %.3f ms, %.2fx the plain "
+                       "step" % (phases_sum, phases_sum / ms if ms else 0.0),
         "clocks": clocks,
         "e2e": {"value": job_value(world, B, e2e_ms), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
         "gpu_launches": launches_headline * steps,
         "gpu_launches_per_step": launches_headline,
         "cpu_baseline": cpu,
-        "large": large,
+        "base": extra,
     }
     print(json.dumps(line))
     if dist:
@@ -452,24 +520,25 @@ def gpu_main(args):
     return 0
 
 
-def large_gemm_check(torch, R, synth, device, peaks):
-    """BERT-large-shaped step at d = 24 and d = 1: samples/s and the GEMMs' tensor throughput
-    (the target for these GEMMs is >= 60 % of the dense bf16 peak)."""
-    cfg = synth.CONFIGS["large"]
-    run = Runner(cfg, cfg.n_layers, device)
+def base_sweep(torch, R, synth, device, peaks, steps, warmup, windows):
+    """The BERT-base-shaped step over d = 1, 3, 6, 12: samples/s and, at d = 6, the GEMMs'
+    throughput from a profiled replay."""
+    cfg = synth.CONFIGS["base"]
+    ds, hd = SWEEPS["base"]
+    run = Runner(cfg, max(ds), device)
     out = {}
-    for d in (24, 1):
+    for d in ds:
         run.capture(d)
-        run.capture(d, profile=True)
-        ms = run.time_steps(d, 10, 3)
-        prof = run.kernel_times(d, 10)
-        g = prof["gemm"]
-        tf = g["flops"] / (g["ms"] / 1000.0) / 1e12 if g["ms"] > 0 else None
+    run.capture(hd, profile=True)
+    t0 = time.time()
+    for d in ds:
+        ms = run.time_steps(d, steps, warmup)
         out["d=%d" % d] = {"samples_per_s": cfg.batch / (ms / 1000.0), "ms_per_step": ms,
-                           "gemm_tflops": tf,
-                           "gemm_frac_sustained": tf / peaks["bf16_tflops_sustained"] if tf else None,
-                           "gemm_frac_burst": tf / peaks["bf16_tflops"] if tf else None,
-                           "gemm_share_of_step": g["ms"] / ms if ms else None}
+                           "saved_activation_bytes": run.saved[d]}
+    prof = run.kernel_times(hd, min(steps, 50))
+    windows["base"] = (t0, time.time())
+    out["gemm_at_d=%d" % hd] = gemm_rate(prof, peaks)
+    out["phases_ms_at_d=%d" % hd] = {k: round(v["ms"], 4) for k, v in prof.items()}
     return out
 
 

@@ -296,7 +296,10 @@ size_t ra_adapter_backward_scratch_bytes(int32_t T, int32_t H, int32_t m);
  * the call allocates nothing and frees nothing.  Sizes whose scratch need
  * (ra_adapter_backward_scratch_bytes) exceeds the array are rejected with RA_ERR_NOMEM.
  * The first call on a device looks up the array's device address (cudaGetSymbolAddress);
- * make that first call before any stream capture.  All calls share the one array: calls
+ * make that first call before any stream capture.  The address is kept per device together
+ * with the CUDA context it belongs to; a call made after that context was destroyed and
+ * re-created (e.g. by cudaDeviceReset) looks it up again, so it too should come before any
+ * capture.  All calls share the one array: calls
  * that can overlap on the GPU (different streams without ordering) race on it and must be
  * serialised by the caller.  Nothing in the array needs to start at zero: every element a
  * call reads was written earlier in the same call. */

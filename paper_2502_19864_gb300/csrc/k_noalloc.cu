@@ -5,6 +5,7 @@
 // slots of serving runtimes) have no allocator to call, and loops that forbid allocation
 // once running cannot afford cudaMalloc, which can block, synchronise the device or fail
 // at any time.  This variant keeps its scratch in a fixed device array instead.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -21,18 +22,47 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratch
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
+// per device: the array's address and the CUDA context it was looked up in.  A module
+// variable's address belongs to the context; after a device reset (or any other teardown
+// and re-creation of the primary context) the cached address would point into a dead
+// context, so the lookup is redone whenever the current context differs.
 void* g_scratch_ptr[kMaxDevices] = {};
+CUcontext g_scratch_ctx[kMaxDevices] = {};
+
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+CtxGetCurrentFn ctx_get_current() {
+  static CtxGetCurrentFn fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<CtxGetCurrentFn>(p);
+  }
+  return fn;
+}
 
 // Device address of the array on the current device (host code cannot use the array's
-// name as an address: it names a host-side stand-in).  Looked up once per device.
+// name as an address: it names a host-side stand-in).  Looked up once per device and
+// context.
 ra_status scratch_on_current_device(void** out) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return RA_ERR_CUDA;
+  CtxGetCurrentFn get = ctx_get_current();
+  if (!get) return RA_ERR_CUDA;
+  CUcontext cur = nullptr;
+  if (get(&cur) != CUDA_SUCCESS) return RA_ERR_CUDA;
   std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_scratch_ptr[dev]) {
+  if (!cur || !g_scratch_ptr[dev] || g_scratch_ctx[dev] != cur) {
+    // the lookup also makes the device's primary context current if none was
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return RA_ERR_CUDA;
+    if (get(&cur) != CUDA_SUCCESS || !cur) return RA_ERR_CUDA;
     g_scratch_ptr[dev] = p;
+    g_scratch_ctx[dev] = cur;
   }
   *out = g_scratch_ptr[dev];
   return RA_OK;

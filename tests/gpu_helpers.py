@@ -8,6 +8,11 @@ from paper_2502_19864_gb300 import ringada as R
 
 # tolerances of the parity bar
 F32_TOL = 1e-4          # max |gpu - oracle| / max |oracle|, per tensor (fp32 models)
+# element-wise relative error of fp32 models, max_i |gpu_i - oracle_i| / max(|oracle_i|,
+# floor): relative error is undefined at zeros, so elements below the floor (a stated
+# fraction of the tensor's largest magnitude) are measured against the floor instead
+F32_ELEM_FLOOR = 1e-2   # floor = F32_ELEM_FLOOR * max |oracle|
+F32_ELEM_TOL = 1e-3
 BF16_LOSS_TOL = 2e-2    # relative, loss; normwise, logits (bf16 models)
 BF16_GRAD_TOL = 5e-2    # normwise, per adapter/head gradient tensor (bf16 models)
 
@@ -93,6 +98,11 @@ def rel_max(a, b):
     return float(np.abs(a - b).max() / max(np.abs(b).max(), 1e-30))
 
 
+def rel_elem(a, b, floor_frac=F32_ELEM_FLOOR):
+    floor = floor_frac * max(float(np.abs(b).max()), 1e-30)
+    return float((np.abs(a - b) / np.maximum(np.abs(b), floor)).max())
+
+
 def rel_norm(a, b):
     return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
 
@@ -116,15 +126,23 @@ def check_step(cfg, gpu_loss, gpu_logits, gpu_grads, gpu_head, ref, k):
         if gpu_logits is not None:
             report["logits"] = rel_max(gpu_logits, ref["logits"])
             assert report["logits"] <= F32_TOL, report
+            report["logits_elem"] = rel_elem(gpu_logits, ref["logits"])
+            assert report["logits_elem"] <= F32_ELEM_TOL, report
         for l in range(k, cfg.n_layers):
             for key in synth.ADAPTER_KEYS:
                 e = rel_max(gpu_grads[l][key], ref["grads"][l][key])
                 report["g%d%s" % (l, key)] = e
                 assert e <= F32_TOL, (l, key, e)
+                e = rel_elem(gpu_grads[l][key], ref["grads"][l][key])
+                report["g%d%s_elem" % (l, key)] = e
+                assert e <= F32_ELEM_TOL, (l, key, "elementwise", e)
         for key, g in gpu_head.items():
             e = rel_max(g, ref["head_grads"][key])
             report["head" + key] = e
             assert e <= F32_TOL, (key, e)
+            e = rel_elem(g, ref["head_grads"][key])
+            report["head%s_elem" % key] = e
+            assert e <= F32_ELEM_TOL, (key, "elementwise", e)
     else:
         report["loss"] = abs(gpu_loss - ref["loss"]) / abs(ref["loss"])
         assert report["loss"] <= BF16_LOSS_TOL, report

@@ -2,10 +2,12 @@
 cannot allocate device memory: plug-in hosts that hand over only inputs and outputs, and
 loops that forbid allocation once running.  Checked through the C ABI against the existing
 ra_adapter_backward on two calls in a row with different inputs, since the fixed scratch
-array is shared by every call and keeps the previous call's contents.  Named to run last."""
+array is shared by every call and keeps the previous call's contents, and on both calls
+against the fp64 oracle's adapter backward (Eq. 1 differentiated).  Named to run last."""
 import numpy as np
 import pytest
 
+from oracle import ringada_oracle as O
 from paper_2502_19864_gb300 import ringada as R
 
 pytestmark = pytest.mark.gpu
@@ -65,6 +67,12 @@ def test_no_alloc_matches_the_scratch_entry_point_on_consecutive_calls():
         for a, b in zip(got, ref):
             a, b = a.double().cpu().numpy(), b.double().cpu().numpy()
             assert np.abs(a - b).max() <= 1e-5 * np.abs(b).max()
+        # the oracle on the same fp32 inputs: dh, dW_down, dW_up within the fp32 parity bar
+        host = {k: v.double().cpu().numpy() for k, v in x.items()}
+        dh, dWd, dWu = O.adapter_backward(host["g"], host["h"], host["z"], host["Wd"], host["Wu"])
+        for a, b in zip(got, (dWd, dWu, dh)):
+            a = a.double().cpu().numpy()
+            assert np.abs(a - b).max() <= 1e-4 * np.abs(b).max()
 
 
 def test_no_alloc_rejects_sizes_beyond_its_array():
