@@ -60,6 +60,18 @@ typedef enum {
 
 enum { RA_ENCODER_POSTLN = 0, RA_DECODER_PRENORM = 1, RA_ENCODER_POSTLN_SPAN = 2 };
 enum { RA_F32 = 0, RA_BF16 = 1 };
+/* Adapter placement (ra_model_cfg.adapter_placement).
+ *   RA_ADAPTERS_HOULSBY   two adapters per block, on the attention-output and FFN-output
+ *                         branches before their residual add (both archs; parameters
+ *                         RA_P_WDA/WUA and RA_P_WDF/WUF);
+ *   RA_ADAPTERS_POST_FFN  the placement of the paper's Fig. 1 (Section II-A): one adapter
+ *                         per block after the FFN's add & LayerNorm, out = y2 +
+ *                         sigma(y2 W_down) W_up (Eq. 1 on the block's LayerNorm output),
+ *                         nothing after it; encoders only; its matrices are RA_P_WDF/WUF
+ *                         (RA_P_WDA/WUA are not part of such a model).  At the lowest
+ *                         unfrozen layer the backward stops right after this adapter's
+ *                         weight gradients. */
+enum { RA_ADAPTERS_HOULSBY = 0, RA_ADAPTERS_POST_FFN = 1 };
 
 /* Model shape.  Encoder: post-LN blocks (LayerNorm, biased linears, exact-GELU FFN), a
  * trainable n_out-class linear head on the token at position 0.  Span encoder
@@ -83,6 +95,7 @@ typedef struct {
                               saved-activation arena: memory falls as this falls */
   float norm_eps;          /* LayerNorm / RMSNorm epsilon */
   float rope_theta;        /* RoPE base (decoder) */
+  int32_t adapter_placement; /* RA_ADAPTERS_HOULSBY (0) | RA_ADAPTERS_POST_FFN (encoders) */
 } ra_model_cfg;
 
 typedef struct {
@@ -146,6 +159,12 @@ ra_status ra_bind_memory(ra_ctx* ctx, void* weights_dev, size_t weights_bytes,
  * model must have been set once before the first ra_forward.  Builds the transposed
  * copies the backward reads.  Enqueued on stream. */
 ra_status ra_set_weights(ra_ctx* ctx, const ra_tensor_desc* list, int32_t n, ra_stream_t stream);
+
+/* Top-down unfreezing schedule (Algorithm 1: every `interval` rounds the depth grows by
+ * one adapter layer, d <- d + 1, from the top down; Section IV unfreezes one more every 40
+ * steps): the depth of 0-based step `step` is min(d0 + floor(step / interval), d_max).
+ * Host-only, pure.  Returns -1 for step < 0, interval < 1, d0 < 1 or d_max < d0. */
+int32_t ra_schedule_depth(int32_t step, int32_t interval, int32_t d0, int32_t d_max);
 
 /* Unfreezing depth d (1..max_depth): the next forward saves activations for layers
  * k = L - d .. L-1 only (Section III-A: below the depth only the forward runs). */

@@ -237,8 +237,14 @@ __device__ __forceinline__ void store_block(bf16* dst, int H, const bf16* src, i
   }
 }
 
-template <int MB, bool DEC, int SZ>
+// MODE: FWD_LN (post-LN encoder: residual add, LayerNorm), FWD_RMS (pre-norm decoder: f32
+// residual stream, RMSNorm of it), FWD_NONE (the paper's post-FFN placement: y = a +
+// GELU(a W_down) W_up, no residual operand, no norm)
+enum : int { FWD_LN = 0, FWD_RMS = 1, FWD_NONE = 2 };
+
+template <int MB, int MODE, int SZ>
 __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
+  constexpr bool DEC = MODE == FWD_RMS;
   extern __shared__ __align__(16) uint8_t sm[];
   pdl_wait();
   pdl_trigger();
@@ -279,12 +285,27 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_fwd_mma_kernel(FwdArgs p) {
   __syncthreads();
   // encoder: the residual rows of this warp's columns land in the (now free) partial buffer
   // while phase 2 runs
-  if (!DEC) load_block_async(Rs, lda, reinterpret_cast<const bf16*>(p.resid), t0, p.T, H, nbase, lane);
+  if (MODE == FWD_LN) load_block_async(Rs, lda, reinterpret_cast<const bf16*>(p.resid), t0, p.T, H, nbase, lane);
   float v[8][4];
   phase2<MB>(v, Ss, lds, p.WuT, MB, nbase, lane);
-  if (!DEC) {
+  if (MODE == FWD_LN) {
     cp_async_wait_all();
     __syncwarp();
+  }
+  if (MODE == FWD_NONE) {
+    // y = a + GELU(z) W_up, through this warp's columns of the a rows
+    const int rl0 = g, rl1 = g + 8;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      const int c = nbase + nt * 8 + 2 * t;
+      const float2 a0 = unpack2(*reinterpret_cast<const uint32_t*>(As + (size_t)rl0 * lda + c));
+      const float2 a1 = unpack2(*reinterpret_cast<const uint32_t*>(As + (size_t)rl1 * lda + c));
+      *reinterpret_cast<uint32_t*>(As + (size_t)rl0 * lda + c) = pack2(v[nt][0] + a0.x, v[nt][1] + a0.y);
+      *reinterpret_cast<uint32_t*>(As + (size_t)rl1 * lda + c) = pack2(v[nt][2] + a1.x, v[nt][3] + a1.y);
+    }
+    __syncwarp();
+    store_block(p.y, H, As, lda, t0, p.T, nbase, lane);
+    return;
   }
   const int rl0 = g, rl1 = g + 8;  // local rows of c0/c1 and c2/c3
   const int r0 = t0 + rl0, r1 = t0 + rl1;
@@ -416,10 +437,10 @@ struct BwdArgs {
   const bf16* Wu;     // [m, H]
   const bf16* Wd;     // [H, m]
   float* dz;          // [T, m]
-  bf16* dh;           // [T, H] or null
+  void* dh;           // [T, H] or null: bf16, or f32 when DH_F32
 };
 
-template <int MB, int SZ>
+template <int MB, int SZ, bool DH_F32>
 __global__ void RA_ROWS_BOUNDS(SZ) adapter_bwd_rows_mma_kernel(BwdArgs p) {
   extern __shared__ __align__(16) uint8_t sm[];
   pdl_wait();
@@ -455,6 +476,23 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_bwd_rows_mma_kernel(BwdArgs p) {
   float v[8][4];
   phase2<MB>(v, Ds, lds, p.Wd, MB, nbase, lane);
   const int r0 = t0 + g, r1 = r0 + 8;
+  if (DH_F32) {
+    // fp32 dh (the gradient feeding a LayerNorm backward), written from registers
+    float* dh = reinterpret_cast<float*>(p.dh);
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      const int c = nbase + nt * 8 + 2 * t;
+      if (r0 < p.T) {
+        const float2 q0 = *reinterpret_cast<const float2*>(p.g + (size_t)r0 * H + c);
+        *reinterpret_cast<float2*>(dh + (size_t)r0 * H + c) = make_float2(v[nt][0] + q0.x, v[nt][1] + q0.y);
+      }
+      if (r1 < p.T) {
+        const float2 q1 = *reinterpret_cast<const float2*>(p.g + (size_t)r1 * H + c);
+        *reinterpret_cast<float2*>(dh + (size_t)r1 * H + c) = make_float2(v[nt][2] + q1.x, v[nt][3] + q1.y);
+      }
+    }
+    return;
+  }
   // dh goes through this warp's columns of the staged g rows, then out in whole row segments
 #pragma unroll
   for (int nt = 0; nt < 8; ++nt) {
@@ -466,7 +504,7 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_bwd_rows_mma_kernel(BwdArgs p) {
     *reinterpret_cast<uint32_t*>(Gs + (size_t)(g + 8) * ldg + c) = pack2(v[nt][2] + q1.x, v[nt][3] + q1.y);
   }
   __syncwarp();
-  store_block(p.dh, H, Gs, ldg, t0, p.T, nbase, lane);
+  store_block(reinterpret_cast<bf16*>(p.dh), H, Gs, ldg, t0, p.T, nbase, lane);
 }
 
 // ---------------------------------------------------------------------------------------
@@ -612,19 +650,21 @@ int smem_per_sm() {
   return v;
 }
 
-template <int MB, bool DEC>
+template <int MB, int MODE>
 cudaError_t launch_fwd(FwdArgs p, cudaStream_t st) {
+  constexpr bool DEC = MODE == FWD_RMS;
   // gamma (and beta) go to shared memory when that keeps the CTAs per SM (1 KB reserved each)
-  const int gbf = (DEC ? 1 : 2) * p.H;
+  const int gbf = MODE == FWD_NONE ? 0 : (DEC ? 1 : 2) * p.H;
   const size_t s0 = fwd_layout(p.H, MB, 0).bytes, s1 = fwd_layout(p.H, MB, gbf).bytes;
   const int per_sm = smem_per_sm();
-  const bool aligned = ((uintptr_t)p.gamma & 15) == 0 && (DEC || ((uintptr_t)p.beta & 15) == 0);
+  const bool aligned = MODE != FWD_NONE && ((uintptr_t)p.gamma & 15) == 0 &&
+                       (DEC || ((uintptr_t)p.beta & 15) == 0);
   p.stage_gb = aligned && s1 <= 220 * 1024 && per_sm > 0 &&
                per_sm / (int)(s1 + 1024) == per_sm / (int)(s0 + 1024);
   const size_t smem = p.stage_gb ? s1 : s0;
   const int sz = size_class(p.H);
-  auto k = sz == 0 ? adapter_fwd_mma_kernel<MB, DEC, 0>
-         : sz == 1 ? adapter_fwd_mma_kernel<MB, DEC, 1> : adapter_fwd_mma_kernel<MB, DEC, 2>;
+  auto k = sz == 0 ? adapter_fwd_mma_kernel<MB, MODE, 0>
+         : sz == 1 ? adapter_fwd_mma_kernel<MB, MODE, 1> : adapter_fwd_mma_kernel<MB, MODE, 2>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k, dim3((p.T + R - 1) / R), dim3((p.H / COLS_PER_WARP) * 32), smem, st, p);
@@ -632,12 +672,12 @@ cudaError_t launch_fwd(FwdArgs p, cudaStream_t st) {
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-template <int MB>
+template <int MB, bool DH_F32>
 cudaError_t launch_bwd(const BwdArgs& p, cudaStream_t st) {
   const size_t smem = rows_smem(p.H, MB);
   const int sz = size_class(p.H);
-  auto k = sz == 0 ? adapter_bwd_rows_mma_kernel<MB, 0>
-         : sz == 1 ? adapter_bwd_rows_mma_kernel<MB, 1> : adapter_bwd_rows_mma_kernel<MB, 2>;
+  auto k = sz == 0 ? adapter_bwd_rows_mma_kernel<MB, 0, DH_F32>
+         : sz == 1 ? adapter_bwd_rows_mma_kernel<MB, 1, DH_F32> : adapter_bwd_rows_mma_kernel<MB, 2, DH_F32>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k, dim3((p.T + R - 1) / R), dim3((p.H / COLS_PER_WARP) * 32), smem, st, p);
@@ -663,27 +703,33 @@ cudaError_t adapter_fwd_mma(const AdapterFwdArgs& a, const void* WdT_b, const vo
   p.z = a.z; p.resid = a.resid; p.gamma = a.gamma; p.beta = a.beta; p.eps = a.eps;
   p.y = reinterpret_cast<bf16*>(a.y); p.x_out = a.x_out;
   p.xhat = reinterpret_cast<bf16*>(a.xhat); p.rstd = a.rstd;
+  if (a.no_norm && (a.decoder || a.resid)) return cudaErrorNotSupported;
+  const int mode = a.no_norm ? FWD_NONE : a.decoder ? FWD_RMS : FWD_LN;
+#define RA_FWD_MODES(MB)                                                          \
+  return mode == FWD_NONE ? launch_fwd<MB, FWD_NONE>(p, st)                       \
+       : mode == FWD_RMS  ? launch_fwd<MB, FWD_RMS>(p, st) : launch_fwd<MB, FWD_LN>(p, st)
   switch (a.m) {
-    case 32: return a.decoder ? launch_fwd<32, true>(p, st) : launch_fwd<32, false>(p, st);
-    case 64: return a.decoder ? launch_fwd<64, true>(p, st) : launch_fwd<64, false>(p, st);
-    case 128: return a.decoder ? launch_fwd<128, true>(p, st) : launch_fwd<128, false>(p, st);
+    case 32: RA_FWD_MODES(32);
+    case 64: RA_FWD_MODES(64);
+    case 128: RA_FWD_MODES(128);
   }
+#undef RA_FWD_MODES
   return cudaErrorNotSupported;
 }
 
 cudaError_t adapter_bwd_mma(const AdapterBwdArgs& a, const void* Wu_b, const void* Wd_b,
                             cudaStream_t st) {
   if (a.dtype != DT_BF16 || !adapter_mma_ok(a.H, a.m)) return cudaErrorNotSupported;
-  if (a.dh && a.dh_dtype != DT_BF16) return cudaErrorNotSupported;
   BwdArgs p;
   p.T = a.T; p.H = a.H; p.m = a.m; p.g = a.g; p.z = a.z;
   p.Wu = reinterpret_cast<const bf16*>(Wu_b);
   p.Wd = reinterpret_cast<const bf16*>(Wd_b);
-  p.dz = a.dz; p.dh = reinterpret_cast<bf16*>(a.dh);
+  p.dz = a.dz; p.dh = a.dh;
+  const bool f32 = a.dh && a.dh_dtype == DT_F32;
   cudaError_t e = cudaErrorNotSupported;
-  if (a.m == 32) e = launch_bwd<32>(p, st);
-  else if (a.m == 64) e = launch_bwd<64>(p, st);
-  else if (a.m == 128) e = launch_bwd<128>(p, st);
+  if (a.m == 32) e = f32 ? launch_bwd<32, true>(p, st) : launch_bwd<32, false>(p, st);
+  else if (a.m == 64) e = f32 ? launch_bwd<64, true>(p, st) : launch_bwd<64, false>(p, st);
+  else if (a.m == 128) e = f32 ? launch_bwd<128, true>(p, st) : launch_bwd<128, false>(p, st);
   if (e != cudaSuccess) return e;
   // weight-gradient partials on the tensor cores, then the fixed-order sum
   DwArgs d;

@@ -103,7 +103,7 @@ __global__ void __launch_bounds__(WARPS * 32) adapter_fwd_kernel(AdapterFwdArgs 
         int i = i0 + lane + 32 * cc;
         if (i < H) {
           float res = 0.f;
-          if (t < a.T)
+          if (t < a.T && a.resid)
             res = a.decoder ? reinterpret_cast<const float*>(a.resid)[(int64_t)t * H + i]
                             : ldf<T>(a.resid, (int64_t)t * H + i);
           rows[r * H + i] = res + rows[r * H + i] + acc[r][cc];
@@ -117,7 +117,9 @@ __global__ void __launch_bounds__(WARPS * 32) adapter_fwd_kernel(AdapterFwdArgs 
     int t = t0 + r;
     if (t >= a.T) break;
     float* v = rows + r * H;
-    if (!a.decoder) {
+    if (a.no_norm) {
+      for (int i = lane; i < H; i += 32) stf<T>(a.y, (int64_t)t * H + i, v[i]);
+    } else if (!a.decoder) {
       float s = 0.f;
       for (int i = lane; i < H; i += 32) s += v[i];
       float mu = warp_sum(s) / H;
@@ -329,7 +331,7 @@ int dw_chunks(int T, int H) {
 // ---------------------------------------------------------------------------------------
 template <typename T>
 __global__ void layernorm_bwd_kernel(const float* dy, const float* dy2, const void* xhat, const float* rstd,
-                                     const float* gamma, float* ds, int Tn, int H) {
+                                     const float* gamma, float* ds, void* ds_act, int Tn, int H) {
   int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (t >= Tn) return;
   float s1 = 0.f, s2 = 0.f;
@@ -345,8 +347,36 @@ __global__ void layernorm_bwd_kernel(const float* dy, const float* dy2, const vo
   for (int i = lane; i < H; i += 32) {
     float gy = (dy[(int64_t)t * H + i] + (dy2 ? dy2[(int64_t)t * H + i] : 0.f)) * gamma[i];
     float xh = ldf<T>(xhat, (int64_t)t * H + i);
-    ds[(int64_t)t * H + i] = r * (gy - s1 - xh * s2);
+    const float d = r * (gy - s1 - xh * s2);
+    ds[(int64_t)t * H + i] = d;
+    if (ds_act) stf<T>(ds_act, (int64_t)t * H + i, d);
   }
+}
+
+// LayerNorm of a residual sum: y = LN(x + a) * gamma + beta; xhat and rstd saved when given.
+// One warp per row (any H); x, a, y and xhat in the activation type.
+template <typename T>
+__global__ void add_layernorm_fwd_kernel(const void* x, const void* a, const float* gamma,
+                                         const float* beta, float eps, void* y, void* xhat,
+                                         float* rstd_out, int Tn, int H) {
+  int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (t >= Tn) return;
+  const int64_t base = (int64_t)t * H;
+  float s = 0.f;
+  for (int i = lane; i < H; i += 32) s += ldf<T>(x, base + i) + ldf<T>(a, base + i);
+  const float mu = warp_sum(s) / H;
+  float q = 0.f;
+  for (int i = lane; i < H; i += 32) {
+    const float d = ldf<T>(x, base + i) + ldf<T>(a, base + i) - mu;
+    q += d * d;
+  }
+  const float r = rsqrtf(warp_sum(q) / H + eps);
+  for (int i = lane; i < H; i += 32) {
+    const float xh = (ldf<T>(x, base + i) + ldf<T>(a, base + i) - mu) * r;
+    stf<T>(y, base + i, xh * gamma[i] + beta[i]);
+    if (xhat) stf<T>(xhat, base + i, xh);
+  }
+  if (rstd_out && lane == 0) rstd_out[t] = r;
 }
 
 template <typename TX, typename TN>
@@ -410,7 +440,7 @@ template <> __device__ __forceinline__ void st4<bf16>(void* p, int64_t i, float4
 
 template <typename TX, int V>
 __global__ void __launch_bounds__(256) layernorm_bwd_vec_kernel(const float* dy, const float* dy2,
-    const void* xhat, const float* rstd, const float* gamma, float* ds, int Tn, int H) {
+    const void* xhat, const float* rstd, const float* gamma, float* ds, void* ds_act, int Tn, int H) {
   pdl_wait();
   pdl_trigger();
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
@@ -438,9 +468,50 @@ __global__ void __launch_bounds__(256) layernorm_bwd_vec_kernel(const float* dy,
 #pragma unroll
   for (int v = 0; v < V; ++v) {
     const int c = (v * 32 + lane) * 4;
-    st4<float>(ds, base + c, make_float4(r * (g[v].x - s1 - x[v].x * s2), r * (g[v].y - s1 - x[v].y * s2),
-                                         r * (g[v].z - s1 - x[v].z * s2), r * (g[v].w - s1 - x[v].w * s2)));
+    const float4 d = make_float4(r * (g[v].x - s1 - x[v].x * s2), r * (g[v].y - s1 - x[v].y * s2),
+                                 r * (g[v].z - s1 - x[v].z * s2), r * (g[v].w - s1 - x[v].w * s2));
+    st4<float>(ds, base + c, d);
+    if (ds_act) st4<TX>(ds_act, base + c, d);
   }
+}
+
+// Vector form of add_layernorm_fwd_kernel (H a multiple of 128): a warp holds its row in
+// registers, V float4 per lane, 16- or 8-byte accesses.
+template <typename T, int V>
+__global__ void __launch_bounds__(256) add_layernorm_fwd_vec_kernel(const void* x, const void* a,
+    const float* gamma, const float* beta, float eps, void* y, void* xhat, float* rstd_out, int Tn,
+    int H) {
+  pdl_wait();
+  pdl_trigger();
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= Tn) return;
+  const int64_t base = (int64_t)row * H;
+  float4 v[V];
+  float s = 0.f;
+#pragma unroll
+  for (int k = 0; k < V; ++k) {
+    const int c = (k * 32 + lane) * 4;
+    const float4 xa = ld4<T>(x, base + c), aa = ld4<T>(a, base + c);
+    v[k] = make_float4(xa.x + aa.x, xa.y + aa.y, xa.z + aa.z, xa.w + aa.w);
+    s += v[k].x + v[k].y + v[k].z + v[k].w;
+  }
+  const float mu = warp_sum(s) / H;
+  float q = 0.f;
+#pragma unroll
+  for (int k = 0; k < V; ++k) {
+    const float d0 = v[k].x - mu, d1 = v[k].y - mu, d2 = v[k].z - mu, d3 = v[k].w - mu;
+    q += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
+  }
+  const float r = rsqrtf(warp_sum(q) / H + eps);
+#pragma unroll
+  for (int k = 0; k < V; ++k) {
+    const int c = (k * 32 + lane) * 4;
+    const float4 gm = ld4<float>(gamma, c), bt = ld4<float>(beta, c);
+    const float4 xh = make_float4((v[k].x - mu) * r, (v[k].y - mu) * r, (v[k].z - mu) * r, (v[k].w - mu) * r);
+    st4<T>(y, base + c, make_float4(xh.x * gm.x + bt.x, xh.y * gm.y + bt.y, xh.z * gm.z + bt.z, xh.w * gm.w + bt.w));
+    if (xhat) st4<T>(xhat, base + c, xh);
+  }
+  if (rstd_out && lane == 0) rstd_out[row] = r;
 }
 
 template <typename TX, typename TN, int V>
@@ -951,8 +1022,9 @@ cudaError_t adapter_dw_reduce(const float* partials, int nchunk, int H, int m, f
 
 cudaError_t adapter_bwd(const AdapterBwdArgs& a, cudaStream_t st) {
   if (a.m > MAXM || a.m <= 0) return cudaErrorInvalidValue;
-  if (a.dtype == DT_BF16 && a.Wu_b && a.Wd_b && adapter_mma_ok(a.H, a.m) &&
-      (!a.dh || a.dh_dtype == DT_BF16))
+  // the tensor-core kernels write dh as bf16 or f32, so whether (and how) dh is wanted
+  // never changes which kernels compute dz and dW
+  if (a.dtype == DT_BF16 && a.Wu_b && a.Wd_b && adapter_mma_ok(a.H, a.m))
     return adapter_bwd_mma(a, a.Wu_b, a.Wd_b, st);
   size_t smem = ((size_t)ROWS * a.H + ROWS * MAXM) * sizeof(float);
   unsigned grid = blocks_for(a.T, ROWS);
@@ -980,15 +1052,31 @@ cudaError_t adapter_bwd(const AdapterBwdArgs& a, cudaStream_t st) {
 
 cudaError_t layernorm_bwd(const float* dy, const float* dy2, const void* xhat, const float* rstd,
                           const float* gamma, float* ds, int T, int H, int dtype,
-                          cudaStream_t st) {
+                          cudaStream_t st, void* ds_act) {
   unsigned grid = blocks_for((int64_t)T * 32, 256);
   if (const int V = row_vec(H)) {
-    if (dtype == DT_BF16) RA_VEC_SWITCH(V, ((void)launch_pdl(layernorm_bwd_vec_kernel<bf16, VV>, dim3(grid), dim3(256), (size_t)0, st, dy, dy2, xhat, rstd, gamma, ds, T, H)))
-    else RA_VEC_SWITCH(V, ((void)launch_pdl(layernorm_bwd_vec_kernel<float, VV>, dim3(grid), dim3(256), (size_t)0, st, dy, dy2, xhat, rstd, gamma, ds, T, H)))
+    if (dtype == DT_BF16) RA_VEC_SWITCH(V, ((void)launch_pdl(layernorm_bwd_vec_kernel<bf16, VV>, dim3(grid), dim3(256), (size_t)0, st, dy, dy2, xhat, rstd, gamma, ds, ds_act, T, H)))
+    else RA_VEC_SWITCH(V, ((void)launch_pdl(layernorm_bwd_vec_kernel<float, VV>, dim3(grid), dim3(256), (size_t)0, st, dy, dy2, xhat, rstd, gamma, ds, ds_act, T, H)))
   } else if (dtype == DT_BF16) {
-    layernorm_bwd_kernel<bf16><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, T, H);
+    layernorm_bwd_kernel<bf16><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, ds_act, T, H);
   } else {
-    layernorm_bwd_kernel<float><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, T, H);
+    layernorm_bwd_kernel<float><<<grid, 256, 0, st>>>(dy, dy2, xhat, rstd, gamma, ds, ds_act, T, H);
+  }
+  note_launch(1);
+  return cudaGetLastError();
+}
+
+cudaError_t add_layernorm_fwd(const void* x, const void* a, const float* gamma, const float* beta,
+                              float eps, void* y, void* xhat, float* rstd, int T, int H, int dtype,
+                              cudaStream_t st) {
+  unsigned grid = blocks_for((int64_t)T * 32, 256);
+  if (const int V = row_vec(H)) {
+    if (dtype == DT_BF16) RA_VEC_SWITCH(V, ((void)launch_pdl(add_layernorm_fwd_vec_kernel<bf16, VV>, dim3(grid), dim3(256), (size_t)0, st, x, a, gamma, beta, eps, y, xhat, rstd, T, H)))
+    else RA_VEC_SWITCH(V, ((void)launch_pdl(add_layernorm_fwd_vec_kernel<float, VV>, dim3(grid), dim3(256), (size_t)0, st, x, a, gamma, beta, eps, y, xhat, rstd, T, H)))
+  } else if (dtype == DT_BF16) {
+    add_layernorm_fwd_kernel<bf16><<<grid, 256, 0, st>>>(x, a, gamma, beta, eps, y, xhat, rstd, T, H);
+  } else {
+    add_layernorm_fwd_kernel<float><<<grid, 256, 0, st>>>(x, a, gamma, beta, eps, y, xhat, rstd, T, H);
   }
   note_launch(1);
   return cudaGetLastError();

@@ -119,9 +119,12 @@ cudaError_t attention_fwd_tc(const AttnArgs& a, cudaStream_t st);
 //   out_pre = a + GELU(a Wd) Wu, z = a Wd (saved if z != null)
 //   encoder: y = LN(resid + out_pre) * g + b ; xhat, rstd saved (if non-null)
 //   decoder: x_out(f32) = resid(f32) + out_pre ; n = RMSNorm(x_out) * g (act), rstd
+//   no_norm (the paper's post-FFN placement): y = out_pre (act), no residual operand (the
+//            residual of Eq. 1 is the adapter input a itself), no norm
 struct AdapterFwdArgs {
   int T = 0, H = 0, m = 0, dtype = DT_F32;
   bool decoder = false;
+  bool no_norm = false;
   const void* a = nullptr;      // [T, H] act
   const float* Wd = nullptr;    // [H, m]
   const float* Wu = nullptr;    // [m, H]
@@ -175,9 +178,16 @@ cudaError_t adapter_dw_reduce(const float* partials, int nchunk, int H, int m, f
 // LayerNorm backward with frozen gamma: ds = rstd * (gy - mean(gy) - xhat mean(gy xhat)),
 // gy = (dy + dy2) * gamma.  dy, dy2 (nullable: 0) f32, xhat act, ds f32.  The second input
 // lets a residual-stream gradient join here instead of in the producing GEMM's epilogue.
+// ds_act (nullable): a copy of ds in the activation type, for a GEMM that reads it.
 cudaError_t layernorm_bwd(const float* dy, const float* dy2, const void* xhat, const float* rstd,
                           const float* gamma, float* ds, int T, int H, int dtype,
-                          cudaStream_t st);
+                          cudaStream_t st, void* ds_act = nullptr);
+// LayerNorm of a residual sum (the add & norm sublayer): y = LN(x + a) * gamma + beta with
+// biased variance; xhat = the normalised sum and rstd = 1 / sqrt(var + eps) saved when
+// non-null.  x, a, y, xhat in dtype; statistics in fp32.
+cudaError_t add_layernorm_fwd(const void* x, const void* a, const float* gamma, const float* beta,
+                              float eps, void* y, void* xhat, float* rstd, int T, int H, int dtype,
+                              cudaStream_t st);
 // RMSNorm forward: n = x * rstd * gamma; x given as act (x_act) or f32 (x_f32);
 // optionally copies x into x_f32_out (f32 residual stream).
 cudaError_t rmsnorm_fwd(const void* x, int x_dtype, const float* gamma, float eps, void* n,

@@ -48,6 +48,7 @@ struct SlotOff {  // offsets of one saved-activation slot, relative to the slot 
   // encoder (gp: GELU'(u) of the FFN pre-activation u, saved for the backward)
   size_t qkv, O, lse, a, zA, xhat1, rstd1, gp, f, zF, xhat2, rstd2;
   size_t x_in, x1, gu;                                               // decoder extras
+  size_t y2;                                                         // post-FFN adapter input
   size_t full_bytes, lowest_bytes, slot_bytes;
 };
 
@@ -60,6 +61,7 @@ struct ra_ctx {
   int act = DT_F32;
   bool dec = false;
   bool span = false;   // encoder with the span (start/end) head over every token
+  bool post_ffn = false;  // the paper's placement: one adapter per block after the FFN's add & LN
   std::string err;
 
   // region sizes and layouts
@@ -173,8 +175,10 @@ int64_t param_numel(const ra_ctx* c, int layer, int p) {
     return -1;
   }
   switch (p) {
-    case RA_P_WDA: case RA_P_WDF: return H * m;
-    case RA_P_WUA: case RA_P_WUF: return m * H;
+    case RA_P_WDA: return c->post_ffn ? -1 : H * m;
+    case RA_P_WUA: return c->post_ffn ? -1 : m * H;
+    case RA_P_WDF: return H * m;
+    case RA_P_WUF: return m * H;
     default: break;
   }
   if (!c->dec) {
@@ -256,6 +260,17 @@ void plan(ra_ctx* c) {
   s.O = sl.take(T * H * es);
   s.lse = sl.take(Bh * 4);
   size_t full_only = sl.off;
+  if (c->post_ffn) {
+    // layers > k: the attention and FFN backward's inputs; layer k: the adapter's alone
+    s.xhat1 = sl.take(T * H * es);
+    s.rstd1 = sl.take(T * 4);
+    s.gp = sl.take(T * F * es);
+    s.xhat2 = sl.take(T * H * es);
+    s.rstd2 = sl.take(T * 4);
+    full_only = sl.off;
+    s.y2 = sl.take(T * H * es);
+    s.zF = sl.take(T * m * 4);
+  } else {
   s.a = sl.take(T * H * es);
   s.zA = sl.take(T * m * 4);
   if (!c->dec) {
@@ -272,6 +287,7 @@ void plan(ra_ctx* c) {
     s.gu = sl.take(T * 2 * F * es);
     s.f = sl.take(T * H * es);
     s.zF = sl.take(T * m * 4);
+  }
   }
   s.slot_bytes = sl.off;
   s.full_bytes = sl.off;
@@ -353,6 +369,9 @@ ra_status ra_create(const ra_model_cfg* cfg, int32_t adapter_dim, ra_ctx** out) 
   if (g.arch == RA_ENCODER_POSTLN_SPAN && (g.n_out != 2 || g.max_seq > SPAN_MAX_SEQ)) return RA_ERR_SHAPE;
   if (g.arch == RA_DECODER_PRENORM && ((g.dtype == RA_BF16 && g.n_out % 8) || g.head_trainable))
     return RA_ERR_SHAPE;
+  if (g.adapter_placement != RA_ADAPTERS_HOULSBY && g.adapter_placement != RA_ADAPTERS_POST_FFN)
+    return RA_ERR_ARG;
+  if (g.adapter_placement == RA_ADAPTERS_POST_FFN && g.arch == RA_DECODER_PRENORM) return RA_ERR_SHAPE;
   ra_ctx* c = new ra_ctx;
   c->cfg = g;
   c->m = adapter_dim;
@@ -367,6 +386,7 @@ ra_status ra_create(const ra_model_cfg* cfg, int32_t adapter_dim, ra_ctx** out) 
   c->act = g.dtype == RA_BF16 ? DT_BF16 : DT_F32;
   c->dec = g.arch == RA_DECODER_PRENORM;
   c->span = g.arch == RA_ENCODER_POSTLN_SPAN;
+  c->post_ffn = g.adapter_placement == RA_ADAPTERS_POST_FFN;
   c->depth = c->max_depth;
   c->set_mask.assign((size_t)(c->L + 1) * RA_P_COUNT, 0);
   plan(c);
@@ -507,6 +527,12 @@ ra_status ra_set_weights(ra_ctx* ctx, const ra_tensor_desc* list, int32_t n, ra_
   return RA_OK;
 }
 
+int32_t ra_schedule_depth(int32_t step, int32_t interval, int32_t d0, int32_t d_max) {
+  if (step < 0 || interval < 1 || d0 < 1 || d_max < d0) return -1;
+  const int64_t d = (int64_t)d0 + step / interval;
+  return (int32_t)(d < d_max ? d : d_max);
+}
+
 ra_status ra_set_unfrozen_depth(ra_ctx* ctx, int32_t d) {
   if (!ctx) return RA_ERR_ARG;
   if (d < 1 || d > ctx->max_depth)
@@ -632,6 +658,43 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     at.err = ctx->ws<unsigned>(ctx->ws_err);
     if (!lse) at.lse = nullptr;
     CU(P_attn_fwd(ctx, at, st));
+    if (ctx->post_ffn) {
+      // Fig. 1 placement: y1 = LN1(x + a); y2 = LN2(y1 + f); out = y2 + GELU(y2 Wd) Wu
+      void* a_s = ctx->ws<char>(ctx->s_a);
+      g = gemm_args(ctx, O, H, ctx->w(o.Wo), H, T, H, H);
+      g.C = a_s; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.bo);
+      CU(P_gemm(ctx, g, st));
+      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * ((full ? 4 : 3) * dtype_size(act)), st, [&] {
+        return add_layernorm_fwd(xin, a_s, ctx->w<float>(o.g1), ctx->w<float>(o.be1), ctx->cfg.norm_eps,
+                                 y1, full ? xhat1 : nullptr, full ? rstd1 : nullptr, T, H, act, st);
+      }));
+      g = gemm_args(ctx, y1, H, ctx->w(o.W1), H, T, F, H);
+      // layers above k keep GELU'(u) for the FFN backward; layer k stops at its adapter
+      g.epi = full ? EPI_BIAS_GELU_G : EPI_BIAS_GELU;
+      g.C = full ? gp : nullptr; g.ldc = F; g.c_dtype = act; g.bias = ctx->w<float>(o.b1);
+      g.C2 = hbuf; g.ldc2 = F; g.c2_dtype = act;
+      CU(P_gemm(ctx, g, st));
+      void* f_s = ctx->ws<char>(ctx->s_f);
+      g = gemm_args(ctx, hbuf, F, ctx->w(o.W2), F, T, H, F);
+      g.C = f_s; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.b2);
+      CU(P_gemm(ctx, g, st));
+      // the adapter's input: saved for layers >= k, else scratch (a is consumed by now)
+      void* y2 = saved ? sb + so.y2 : a_s;
+      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * ((full ? 4 : 3) * dtype_size(act)), st, [&] {
+        return add_layernorm_fwd(y1, f_s, ctx->w<float>(o.g2), ctx->w<float>(o.be2), ctx->cfg.norm_eps,
+                                 y2, full ? xhat2 : nullptr, full ? rstd2 : nullptr, T, H, act, st);
+      }));
+      AdapterFwdArgs ad;
+      ad.T = T; ad.H = H; ad.m = m; ad.dtype = act; ad.no_norm = true;
+      ad.a = y2; ad.Wd = Pl + (size_t)2 * H * m; ad.Wu = Pl + (size_t)3 * H * m; ad.z = zF;
+      ad.WdT_b = ctx->shadowT(l, 2); ad.WuT_b = ctx->shadowT(l, 3);
+      ad.y = xout;
+      CU(P_adapter_fwd(ctx, ad, st));
+      xin = xout;
+      ctx->top_out = out_idx;
+      out_idx ^= 1;
+      continue;
+    }
     g = gemm_args(ctx, O, H, ctx->w(o.Wo), H, T, H, H);
     g.C = a; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.bo);
     CU(P_gemm(ctx, g, st));
@@ -862,7 +925,53 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
     AdapterBwdArgs ab;
     ab.T = T; ab.H = H; ab.m = m; ab.dtype = act; ab.dz = ctx->ws<float>(ctx->b_dz);
     ab.partials = ctx->ws<float>(ctx->b_part);
-    if (!ctx->dec) {
+    if (ctx->post_ffn) {
+      // Fig. 1 placement: the adapter sits on top of the block, so its backward comes first
+      // (g = dY, input y2); at layer k the traversal ends right after its weight gradients
+      float* dy2 = ctx->ws<float>(ctx->b_ds1);
+      ab.g = dY; ab.h = sb + so.y2; ab.z = (float*)(sb + so.zF);
+      ab.WuT = PTl + (size_t)3 * H * m; ab.WdT = PTl + (size_t)2 * H * m;
+      ab.Wu_b = ctx->shadow(l, 3); ab.Wd_b = ctx->shadow(l, 2);
+      ab.dh = lowest ? nullptr : dy2; ab.dh_dtype = DT_F32;
+      ab.dWd = Gl + (size_t)2 * H * m; ab.dWu = Gl + (size_t)3 * H * m;
+      CU(P_adapter_bwd(ctx, ab, st));
+      if (lowest) break;
+      // ds2 = LN2'(dy2), kept in f32 for the residual path and in the activation type for
+      // the GEMM
+      float* ds2 = ctx->ws<float>(ctx->b_ds2);
+      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * (8 + 2 * dtype_size(act)), st, [&] {
+        return layernorm_bwd(dy2, nullptr, sb + so.xhat2, (float*)(sb + so.rstd2), ctx->w<float>(o.g2), ds2,
+                             T, H, act, st, ctx->ws(ctx->b_df));
+      }));
+      GemmArgs g = gemm_args(ctx, ctx->ws(ctx->b_df), H, ctx->w(o.W2T), H, T, F, H);
+      g.epi = EPI_MUL; g.C = ctx->ws(ctx->b_du); g.ldc = F; g.c_dtype = act;
+      g.aux = sb + so.gp; g.ldaux = F; g.aux_dtype = act;
+      CU(P_gemm(ctx, g, st));
+      float* dy1 = ctx->ws<float>(ctx->b_dy1);
+      g = gemm_args(ctx, ctx->ws(ctx->b_du), F, ctx->w(o.W1T), F, T, H, F);
+      g.C = dy1; g.ldc = H; g.c_dtype = DT_F32;
+      CU(P_gemm(ctx, g, st));
+      float* ds1 = ctx->ws<float>(ctx->b_ds1);
+      CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * (12 + 2 * dtype_size(act)), st, [&] {
+        return layernorm_bwd(dy1, ds2, sb + so.xhat1, (float*)(sb + so.rstd1), ctx->w<float>(o.g1), ds1,
+                             T, H, act, st, ctx->ws(ctx->b_da));
+      }));
+      g = gemm_args(ctx, ctx->ws(ctx->b_da), H, ctx->w(o.WoT), H, T, H, H);
+      g.C = ctx->ws(ctx->b_dO); g.ldc = H; g.c_dtype = act;
+      CU(P_gemm(ctx, g, st));
+      AttnArgs at;
+      at.qkv = sb + so.qkv; at.B = B; at.S = S; at.n_heads = ctx->nh; at.head_dim = ctx->dh;
+      at.dtype = act; at.scale = 1.f / sqrtf((float)ctx->dh); at.O = sb + so.O;
+      at.lse = (float*)(sb + so.lse); at.dO = ctx->ws(ctx->b_dO); at.Dscratch = ctx->ws<float>(ctx->b_D);
+      at.dqkv = ctx->ws(ctx->b_dqkv); at.err = ctx->ws<unsigned>(ctx->ws_err);
+      CU(P_attn_bwd(ctx, at, st));
+      // dX = ds1 + dqkv Wqkv, the residual joined in the GEMM's epilogue (the next layer's
+      // adapter backward reads dX whole)
+      g = gemm_args(ctx, ctx->ws(ctx->b_dqkv), 3 * H, ctx->w(o.WqkvT), 3 * H, T, H, 3 * H);
+      g.epi = EPI_RESID; g.C = dX; g.ldc = H; g.c_dtype = DT_F32;
+      g.aux = ds1; g.ldaux = H; g.aux_dtype = DT_F32;
+      CU(P_gemm(ctx, g, st));
+    } else if (!ctx->dec) {
       float* ds2 = ctx->ws<float>(ctx->b_ds2);
       CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * (8 + dtype_size(act) + (dY2 ? 4 : 0)), st,
               [&] { return layernorm_bwd(dY, dY2, sb + so.xhat2, (float*)(sb + so.rstd2), ctx->w<float>(o.g2), ds2, T, H, act, st); }));
@@ -1004,7 +1113,8 @@ ra_status locate(ra_ctx* ctx, int32_t layer, int32_t which, float* base, const f
                  int64_t* n) {
   if (!ctx->Tr) return fail(ctx, RA_ERR_STATE, "ra_bind_memory first");
   const size_t H = ctx->H, m = ctx->m;
-  if (layer >= 0 && layer < ctx->L && which >= RA_P_WDA && which <= RA_P_WUF) {
+  if (layer >= 0 && layer < ctx->L && which >= RA_P_WDA && which <= RA_P_WUF &&
+      !(ctx->post_ffn && (which == RA_P_WDA || which == RA_P_WUA))) {
     *p = base + (size_t)layer * 4 * H * m + (size_t)(which - RA_P_WDA) * H * m;
     *n = (int64_t)(H * m);
     return RA_OK;

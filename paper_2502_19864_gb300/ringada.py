@@ -23,6 +23,7 @@ STATUS_NAMES = {0: "RA_OK", 1: "RA_ERR_ARG", 2: "RA_ERR_STATE", 3: "RA_ERR_NOT_S
                 8: "RA_ERR_UNSUPPORTED"}
 RA_ENCODER_POSTLN, RA_DECODER_PRENORM, RA_ENCODER_POSTLN_SPAN = 0, 1, 2
 RA_F32, RA_BF16 = 0, 1
+RA_ADAPTERS_HOULSBY, RA_ADAPTERS_POST_FFN = 0, 1
 
 # ra_param ids (same order as the header's enum)
 PARAMS = ["RA_P_WQKV", "RA_P_BQKV", "RA_P_WO", "RA_P_BO", "RA_P_LN1_G", "RA_P_LN1_B",
@@ -48,7 +49,8 @@ class ra_model_cfg(C.Structure):
                 ("n_heads", C.c_int32), ("ffn", C.c_int32), ("n_out", C.c_int32),
                 ("max_batch", C.c_int32), ("max_seq", C.c_int32), ("dtype", C.c_int32),
                 ("head_trainable", C.c_int32), ("max_depth", C.c_int32),
-                ("norm_eps", C.c_float), ("rope_theta", C.c_float)]
+                ("norm_eps", C.c_float), ("rope_theta", C.c_float),
+                ("adapter_placement", C.c_int32)]
 
 
 class ra_adam_cfg(C.Structure):
@@ -96,6 +98,7 @@ _SIGS = {
                                  C.c_void_p, C.c_size_t]),
     "ra_set_weights": (C.c_int, [C.c_void_p, C.POINTER(ra_tensor_desc), C.c_int32, C.c_void_p]),
     "ra_set_unfrozen_depth": (C.c_int, [C.c_void_p, C.c_int32]),
+    "ra_schedule_depth": (C.c_int32, [C.c_int32, C.c_int32, C.c_int32, C.c_int32]),
     "ra_forward": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32,
                              C.c_void_p, C.c_void_p, C.c_void_p]),
     "ra_backward_truncated": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p]),
@@ -312,13 +315,17 @@ def ra_kernel_launches() -> int:
 
 def schedule_depth(step_index: int, interval: int = 50, d0: int = 1, d_max: int = 12) -> int:
     """Top-down unfreezing (Algorithm 1: d <- d + 1 every interval), per 0-based step."""
-    return min(d0 + step_index // interval, d_max)
+    d = lib().ra_schedule_depth(step_index, interval, d0, d_max)
+    if d < 0:
+        raise RingAdaError(RA_ERR_ARG, "ra_schedule_depth: invalid arguments")
+    return d
 
 
 def make_cfg(arch, n_layers, hidden, n_heads, ffn, n_out, max_batch, max_seq, dtype,
-             head_trainable, max_depth=0, norm_eps=1e-12, rope_theta=10000.0):
+             head_trainable, max_depth=0, norm_eps=1e-12, rope_theta=10000.0,
+             adapter_placement=0):
     return ra_model_cfg(arch, n_layers, hidden, n_heads, ffn, n_out, max_batch, max_seq, dtype,
-                        head_trainable, max_depth, norm_eps, rope_theta)
+                        head_trainable, max_depth, norm_eps, rope_theta, adapter_placement)
 
 
 class Model:

@@ -89,6 +89,7 @@ CONFIGS: Dict[str, ModelCfg] = {
     "small_span_bf16": _span(3, 256, 4, 1024, 32, 3, 100, "bf16"),
     # the paper's placement: one adapter per block, after the FFN add & LayerNorm
     "tiny_paper": _paper(2, 128, 2, 512, 16, 4, 32, "f32"),
+    "small_paper_bf16": _paper(3, 256, 4, 1024, 32, 3, 100, "bf16"),
 }
 
 

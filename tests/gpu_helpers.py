@@ -26,9 +26,10 @@ def ra_arch(cfg):
 def ra_cfg(cfg, max_depth=0, max_batch=None, max_seq=None):
     arch = ra_arch(cfg)
     dt = R.RA_BF16 if cfg.dtype == "bf16" else R.RA_F32
+    placement = R.RA_ADAPTERS_POST_FFN if cfg.adapters == "paper" else R.RA_ADAPTERS_HOULSBY
     return R.make_cfg(arch, cfg.n_layers, cfg.hidden, cfg.n_heads, cfg.ffn, cfg.n_out,
                       max_batch or cfg.batch, max_seq or cfg.seq, dt, int(cfg.head_trainable),
-                      max_depth, cfg.norm_eps, cfg.rope_theta)
+                      max_depth, cfg.norm_eps, cfg.rope_theta, placement)
 
 
 class GpuRun:
@@ -75,7 +76,7 @@ class GpuRun:
         out = {}
         for l in range(k, self.cfg.n_layers):
             out[l] = {key: self.model.grad(l, key).double().cpu().numpy().reshape(
-                synth.param_shape(self.cfg, key)) for key in synth.ADAPTER_KEYS}
+                synth.param_shape(self.cfg, key)) for key in synth.adapter_keys(self.cfg)}
         return out
 
     def head_grads(self):
@@ -129,7 +130,7 @@ def check_step(cfg, gpu_loss, gpu_logits, gpu_grads, gpu_head, ref, k):
             report["logits_elem"] = rel_elem(gpu_logits, ref["logits"])
             assert report["logits_elem"] <= F32_ELEM_TOL, report
         for l in range(k, cfg.n_layers):
-            for key in synth.ADAPTER_KEYS:
+            for key in synth.adapter_keys(cfg):
                 e = rel_max(gpu_grads[l][key], ref["grads"][l][key])
                 report["g%d%s" % (l, key)] = e
                 assert e <= F32_TOL, (l, key, e)
@@ -150,7 +151,7 @@ def check_step(cfg, gpu_loss, gpu_logits, gpu_grads, gpu_head, ref, k):
             report["logits"] = rel_norm(gpu_logits, ref["logits"])
             assert report["logits"] <= BF16_LOSS_TOL, report
         for l in range(k, cfg.n_layers):
-            for key in synth.ADAPTER_KEYS:
+            for key in synth.adapter_keys(cfg):
                 e = rel_norm(gpu_grads[l][key], ref["grads"][l][key])
                 report["g%d%s" % (l, key)] = e
                 assert e <= BF16_GRAD_TOL, (l, key, e)

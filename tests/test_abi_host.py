@@ -51,6 +51,16 @@ def test_create_validates_shapes(lib):
             R.ra_create(enc_cfg(arch=R.RA_ENCODER_POSTLN_SPAN, **bad), 16)
         assert e.value.status == R.RA_ERR_SHAPE
     R.ra_destroy(R.ra_create(enc_cfg(arch=R.RA_ENCODER_POSTLN_SPAN, n_out=2), 16))
+    # adapter placement: Houlsby or the paper's post-FFN adapter (encoders only)
+    with pytest.raises(R.RingAdaError) as e:
+        R.ra_create(enc_cfg(adapter_placement=5), 16)
+    assert e.value.status == R.RA_ERR_ARG
+    with pytest.raises(R.RingAdaError) as e:
+        R.ra_create(enc_cfg(arch=R.RA_DECODER_PRENORM, n_out=64, head_trainable=0,
+                            adapter_placement=R.RA_ADAPTERS_POST_FFN), 16)
+    assert e.value.status == R.RA_ERR_SHAPE
+    for arch in (R.RA_ENCODER_POSTLN, R.RA_ENCODER_POSTLN_SPAN):
+        R.ra_destroy(R.ra_create(enc_cfg(arch=arch, adapter_placement=R.RA_ADAPTERS_POST_FFN), 16))
     ctx = R.ra_create(enc_cfg(), 16)
     R.ra_destroy(ctx)
 
@@ -128,10 +138,15 @@ def test_null_arguments_are_rejected(lib):
     assert lib.ra_gemm_bf16(16, 16, 16, 1, 8, 12, None, None, None) == R.RA_ERR_SHAPE
 
 
-def test_schedule_depth_follows_the_unfreezing_rule():
-    # Algorithm 1 / the sched workload: d = min(1 + floor(s / 50), 12)
+def test_schedule_depth_follows_the_unfreezing_rule(lib):
+    # Algorithm 1 / the sched workload: d = min(1 + floor(s / 50), 12), evaluated in the
+    # library (ra_schedule_depth)
     assert [R.schedule_depth(s) for s in (0, 49, 50, 99, 100, 549, 550, 599)] == \
         [1, 1, 2, 2, 3, 11, 12, 12]
+    assert R.schedule_depth(7, interval=3, d0=2, d_max=4) == 4
+    assert R.schedule_depth(0, interval=40, d0=1, d_max=24) == 1
+    assert lib.ra_schedule_depth(-1, 50, 1, 12) == -1      # invalid arguments
+    assert lib.ra_schedule_depth(5, 0, 1, 12) == -1
 
 
 def _mb_set(sizes):
@@ -139,13 +154,15 @@ def _mb_set(sizes):
     return sum((s + 255) // 256 * 256 for s in sizes)
 
 
-@pytest.mark.parametrize("arch", ["encoder", "decoder"])
+@pytest.mark.parametrize("arch", ["encoder", "decoder", "post_ffn"])
 def test_saved_set_per_layer_is_the_backward_inputs(lib, arch):
     """The activation arena holds, per unfrozen layer, exactly what the backward reads: the
     lowest layer k keeps the adapter and norm inputs of its FFN half and the A adapter's
     inputs (no attention backward runs there); every layer above also keeps q|k|v, the
     attention output and the row log-sum-exp (and, decoder, its fp32 input and RMS scale).
-    Capacity = max_depth x the full set."""
+    With the paper's single post-FFN adapter the lowest layer keeps only that adapter's
+    input and bottleneck pre-activation, and the layers above add both norms' xhat and
+    rstd and GELU'(u).  Capacity = max_depth x the full set."""
     B, S, H, heads, F, m = 4, 64, 256, 4, 1024, 32
     T = B * S
     es = 2  # bf16
@@ -154,6 +171,12 @@ def test_saved_set_per_layer_is_the_backward_inputs(lib, arch):
         lowest = [T * H * es, T * m * 4, T * H * es, T * 4, T * F * es, T * H * es, T * m * 4,
                   T * H * es, T * 4]          # a, zA, xhat1, rstd1, GELU'(u), f, zF, xhat2, rstd2
         full_only = [T * 3 * H * es, T * H * es, B * heads * S * 4]   # qkv, O, lse
+    elif arch == "post_ffn":
+        cfg = dict(arch=R.RA_ENCODER_POSTLN, n_out=2, adapter_placement=R.RA_ADAPTERS_POST_FFN)
+        lowest = [T * H * es, T * m * 4]     # y2 (the adapter input), zF
+        full_only = [T * 3 * H * es, T * H * es, B * heads * S * 4, T * H * es, T * 4,
+                     T * F * es, T * H * es, T * 4]
+        #            qkv, O, lse, xhat1, rstd1, GELU'(u), xhat2, rstd2
     else:
         cfg = dict(arch=R.RA_DECODER_PRENORM, n_out=64, head_trainable=0)
         lowest = [T * H * es, T * m * 4, T * H * 4, T * 4, T * 2 * F * es, T * H * es, T * m * 4]

@@ -35,19 +35,21 @@ def _parity_all_depths(name, depths=None, seed=0):
     return reports
 
 
-@pytest.mark.parametrize("name", ["tiny", "mid_enc_f32", "tiny_dec", "tiny_span"])
+@pytest.mark.parametrize("name", ["tiny", "mid_enc_f32", "tiny_dec", "tiny_span", "tiny_paper"])
 def test_fp32_parity_every_depth(name):
     _parity_all_depths(name)
 
 
-@pytest.mark.parametrize("name", ["small_enc_bf16", "small_dec_bf16", "small_span_bf16"])
+@pytest.mark.parametrize("name", ["small_enc_bf16", "small_dec_bf16", "small_span_bf16",
+                                  "small_paper_bf16"])
 def test_bf16_parity_every_depth(name):
     _parity_all_depths(name)
 
 
-def test_truncated_equals_full_and_nothing_below_k():
+@pytest.mark.parametrize("name", ["mid_enc_f32", "tiny_paper", "small_enc_bf16", "small_paper_bf16"])
+def test_truncated_equals_full_and_nothing_below_k(name):
     import torch
-    cfg = synth.CONFIGS["mid_enc_f32"]
+    cfg = synth.CONFIGS[name]
     w = synth.make_workload(cfg, 3)
     run = GpuRun(cfg, w)
     try:
@@ -57,7 +59,7 @@ def test_truncated_equals_full_and_nothing_below_k():
             k = cfg.n_layers - d
             # sentinel in every gradient buffer below k
             for l in range(k):
-                for key in synth.ADAPTER_KEYS:
+                for key in synth.adapter_keys(cfg):
                     ptr, n = R.ra_get_grad(run.ctx, l, R.P[R.KEY_TO_PARAM[key]])
                     base = run.model.buffers[1]
                     off = ptr - base.data_ptr()
@@ -65,11 +67,11 @@ def test_truncated_equals_full_and_nothing_below_k():
             run.step(d)
             g = run.grads(k)
             for l in range(k, cfg.n_layers):
-                for key in synth.ADAPTER_KEYS:
+                for key in synth.adapter_keys(cfg):
                     np.testing.assert_array_equal(g[l][key], full[l][key])
             below = run.grads(0)
             for l in range(k):
-                for key in synth.ADAPTER_KEYS:
+                for key in synth.adapter_keys(cfg):
                     assert np.isnan(below[l][key]).all(), (d, l, key)
     finally:
         run.close()
