@@ -238,7 +238,7 @@ def gemm_traffic():
 class Runner:
     """A model context plus CUDA graphs of one step per depth."""
 
-    def __init__(self, cfg, max_depth, device):
+    def __init__(self, cfg, max_depth, device, prefix_buffers=0):
         import torch
         import synth
         from paper_2502_19864_gb300 import ringada as R
@@ -249,7 +249,10 @@ class Runner:
                                         cfg.n_out, cfg.batch, cfg.seq,
                                         R.RA_BF16 if cfg.dtype == "bf16" else R.RA_F32,
                                         int(cfg.head_trainable), max_depth, cfg.norm_eps,
-                                        cfg.rope_theta), cfg.adapter_dim, device=device)
+                                        cfg.rope_theta,
+                                        R.RA_ADAPTERS_POST_FFN if cfg.adapters == "paper"
+                                        else R.RA_ADAPTERS_HOULSBY, prefix_buffers),
+                             cfg.adapter_dim, device=device)
         self.model.set_weights(w["layers"], w["head"])
         dt = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
         self.x = torch.tensor(w["x"], dtype=torch.float32).to(dt).to(device)
@@ -259,6 +262,7 @@ class Runner:
         self.labels_host = torch.tensor(w["labels"], dtype=torch.int32).pin_memory()
         self.loss_host = torch.zeros(1, dtype=torch.float32).pin_memory()
         self.graphs = {}       # plain graphs of one step per depth (what is timed)
+        self.ograph = {}       # per depth: two graphs of the overlapped step (prefix buffers)
         self.pgraphs = {}      # the same step with a CUDA event around every kernel
         self.launches = {}
         self.saved = {}
@@ -288,6 +292,55 @@ class Runner:
         torch.cuda.synchronize()
         (self.pgraphs if profile else self.graphs)[d] = g
         return g
+
+    def capture_overlap(self, d):
+        """Two graphs of the step with the next batch's frozen prefix overlapped: graph b runs
+        the suffix (blocks k..L-1, head), backward and update of the batch whose prefix is
+        in buffer b on the capture stream, and the prefix of the next batch into buffer 1 - b
+        on a second stream (forked and joined inside the graph).  Replaying 0, 1, 0, ...
+        processes one batch per replay."""
+        torch, R, c, cfg = self.torch, self.R, self.model.ctx, self.cfg
+        R.ra_set_unfrozen_depth(c, d)
+        side = torch.cuda.Stream()
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            R.ra_forward_prefix(c, self.x.data_ptr(), cfg.batch, cfg.seq, 0, stream=s.cuda_stream)
+        torch.cuda.synchronize()
+        graphs = []
+        for b in (0, 1):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s, capture_error_mode="relaxed"):
+                cur = torch.cuda.current_stream()
+                side.wait_stream(cur)
+                R.ra_forward_prefix(c, self.x.data_ptr(), cfg.batch, cfg.seq, 1 - b,
+                                    stream=side.cuda_stream)
+                R.ra_forward_suffix(c, b, self.labels.data_ptr(), self.loss.data_ptr(), None,
+                                    stream=cur.cuda_stream)
+                R.ra_backward_truncated(c, cfg.n_layers - d, stream=cur.cuda_stream)
+                R.ra_adapter_update(c, stream=cur.cuda_stream)
+                cur.wait_stream(side)
+            graphs.append(g)
+        torch.cuda.synchronize()
+        # buffer 0 holds a prefix for the first replay of graph 0 (graph 1 refills it)
+        with torch.cuda.stream(s):
+            R.ra_forward_prefix(c, self.x.data_ptr(), cfg.batch, cfg.seq, 0, stream=s.cuda_stream)
+        torch.cuda.synchronize()
+        self.ograph[d] = graphs
+
+    def time_overlap(self, d, steps, warmup):
+        torch = self.torch
+        g = self.ograph[d]
+        for i in range(2 * ((warmup + 1) // 2)):
+            g[i % 2].replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for i in range(steps):
+            g[i % 2].replay()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / steps
 
     def kernel_times(self, d, reps):
         """Per-kernel device times of the step at depth d: the profiled graph (an event
@@ -403,7 +456,7 @@ def gpu_main(args):
         cpu = run_cpu_baseline(args.config, HEADLINE_D,
                                min(cfg.batch, CPU_SAMPLE_BATCH.get(args.config, 1)), 12.0)
 
-    run = Runner(cfg, max(SWEEP), device)
+    run = Runner(cfg, max(SWEEP), device, prefix_buffers=int(cfg.arch == "encoder"))
     sweep = {}
     for d in SWEEP:
         run.capture(d)
@@ -438,6 +491,19 @@ def gpu_main(args):
     windows["kernel_times"] = (t0, time.time())
     launches_headline = run.launches[HEADLINE_D]
     saved_by_d = dict(run.saved)
+    # the next batch's frozen prefix on a second stream, overlapping this batch's suffix,
+    # backward and update (same work per step; timed the same way)
+    overlap = None
+    if cfg.arch == "encoder":
+        overlap = {}
+        t0 = time.time()
+        for d in SWEEP:
+            run.capture_overlap(d)
+            o_ms = run.time_overlap(d, steps, warmup)
+            overlap["d=%d" % d] = {"ms_per_step": o_ms, "samples_per_s": job_value(world, cfg.batch, o_ms),
+                                   "sequential_ms_per_step": sweep[d],
+                                   "speedup": sweep[d] / o_ms}
+        windows["overlap"] = (t0, time.time())
     R.ra_set_unfrozen_depth(run.model.ctx, HEADLINE_D)
 
     # the slowest rank's times (headline, end to end and every sweep point)
@@ -512,6 +578,7 @@ def gpu_main(args):
         "gpu_launches": launches_headline * steps,
         "gpu_launches_per_step": launches_headline,
         "cpu_baseline": cpu,
+        "prefix_overlap": overlap,
         "base": extra,
     }
     print(json.dumps(line))
@@ -525,16 +592,20 @@ def base_sweep(torch, R, synth, device, peaks, steps, warmup, windows):
     throughput from a profiled replay."""
     cfg = synth.CONFIGS["base"]
     ds, hd = SWEEPS["base"]
-    run = Runner(cfg, max(ds), device)
+    run = Runner(cfg, max(ds), device, prefix_buffers=1)
     out = {}
     for d in ds:
         run.capture(d)
+        run.capture_overlap(d)
     run.capture(hd, profile=True)
     t0 = time.time()
     for d in ds:
         ms = run.time_steps(d, steps, warmup)
+        o_ms = run.time_overlap(d, steps, warmup)
         out["d=%d" % d] = {"samples_per_s": cfg.batch / (ms / 1000.0), "ms_per_step": ms,
-                           "saved_activation_bytes": run.saved[d]}
+                           "saved_activation_bytes": run.saved[d],
+                           "prefix_overlap": {"samples_per_s": cfg.batch / (o_ms / 1000.0),
+                                              "ms_per_step": o_ms, "speedup": ms / o_ms}}
     prof = run.kernel_times(hd, min(steps, 50))
     windows["base"] = (t0, time.time())
     out["gemm_at_d=%d" % hd] = gemm_rate(prof, peaks)

@@ -96,6 +96,8 @@ typedef struct {
   float norm_eps;          /* LayerNorm / RMSNorm epsilon */
   float rope_theta;        /* RoPE base (decoder) */
   int32_t adapter_placement; /* RA_ADAPTERS_HOULSBY (0) | RA_ADAPTERS_POST_FFN (encoders) */
+  int32_t prefix_buffers;  /* encoders: 1 reserves the second set of forward scratch buffers
+                              and the two prefix outputs of ra_forward_prefix/suffix */
 } ra_model_cfg;
 
 typedef struct {
@@ -178,6 +180,29 @@ ra_status ra_set_unfrozen_depth(ra_ctx* ctx, int32_t d);
  * are read as 0 and reported by ra_sync_status. */
 ra_status ra_forward(ra_ctx* ctx, const void* x_dev, const int32_t* labels_dev, int32_t B,
                      int32_t S, float* loss_dev, float* logits_dev, ra_stream_t stream);
+
+/* The same forward split in two, so that the next batch's frozen prefix can run while the
+ * current batch is still in its backward and update (Section III-A: the forward below the
+ * unfreezing depth is independent of the training above it and can run at the same time;
+ * Section III-B.2).  Encoders only; the context needs cfg.prefix_buffers = 1.
+ *
+ * ra_forward_prefix runs blocks 0 .. k-1 (k = L - d for the depth set now) on x_dev
+ * [B, S, H] and leaves the input of block k in prefix buffer `buf` (0 or 1); with k = 0 it
+ * copies x_dev there.  It saves nothing and reads only the frozen weights and the adapters
+ * of blocks below k, which no update at this or a larger depth writes, and it uses its own
+ * scratch buffers: it may run on another stream concurrently with ra_forward_suffix of the
+ * other buffer, ra_backward_truncated and ra_adapter_update.  The caller orders it after
+ * the ra_forward_suffix that last read the same buffer.
+ *
+ * ra_forward_suffix runs blocks k .. L-1, the head and the loss from prefix buffer `buf`,
+ * with the same arguments and results as ra_forward, and enables the backward as
+ * ra_forward does.  The caller orders it after the prefix that filled `buf`.  Returns
+ * RA_ERR_STATE if no prefix filled `buf` or the depth changed since, RA_ERR_UNSUPPORTED
+ * without prefix buffers (or for a decoder). */
+ra_status ra_forward_prefix(ra_ctx* ctx, const void* x_dev, int32_t B, int32_t S, int32_t buf,
+                            ra_stream_t stream);
+ra_status ra_forward_suffix(ra_ctx* ctx, int32_t buf, const int32_t* labels_dev,
+                            float* loss_dev, float* logits_dev, ra_stream_t stream);
 
 /* Backward ending at layer k (0-based; Algorithm 1 "Bw propagation ending at the
  * (L - d + 1)-th adapter" is k = L - d).  Requires a preceding forward; k must satisfy

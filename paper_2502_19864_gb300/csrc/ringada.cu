@@ -100,7 +100,16 @@ struct ra_ctx {
   bool bwd_since_update = false;
   int n_updates = 0;
   int last_xL_slot = 0;
-  int top_out = 0;  // index of the ping-pong buffer holding the last layer's output (encoder)
+  const void* yL = nullptr;  // the last block's output of the latest forward (encoder head input)
+  // next-batch prefix (ra_forward_prefix / ra_forward_suffix, encoders): a second set of
+  // forward scratch buffers, so that the prefix of one batch can run on another stream while
+  // the previous batch's suffix, backward and update run, and two buffers for its output
+  struct FwdScratch { size_t X[2], qkv, O, a, y1, h, f; };
+  FwdScratch fs[2]{};
+  bool prefix_bufs = false;
+  size_t pbuf[2]{};
+  struct PrefixState { bool valid; int k, B, S; };
+  PrefixState pf[2]{};
 
   // profiling: event pairs around kernel calls
   bool profiling = false;
@@ -314,6 +323,21 @@ void plan(ra_ctx* c) {
   c->s_f = ws.take(T * H * es);
   c->s_u = c->dec ? 0 : ws.take(T * F * es);
   c->s_gu = c->dec ? ws.take(T * 2 * F * es) : 0;
+  c->fs[0] = {{c->s_X[0], c->s_X[1]}, c->s_qkv, c->s_O, c->s_a, c->s_y1, c->s_h, c->s_f};
+  c->prefix_bufs = !c->dec && c->cfg.prefix_buffers != 0;
+  if (c->prefix_bufs) {
+    ra_ctx::FwdScratch& f1 = c->fs[1];
+    f1.X[0] = ws.take(T * H * es);
+    f1.X[1] = ws.take(T * H * es);
+    f1.qkv = ws.take(T * 3 * H * es);
+    f1.O = ws.take(T * H * es);
+    f1.a = ws.take(T * H * es);
+    f1.y1 = ws.take(T * H * es);
+    f1.h = ws.take(T * F * es);
+    f1.f = ws.take(T * H * es);
+    c->pbuf[0] = ws.take(T * H * es);
+    c->pbuf[1] = ws.take(T * H * es);
+  }
   // backward
   c->b_dY[0] = ws.take(T * H * 4);
   c->b_dY[1] = ws.take(T * H * 4);
@@ -621,32 +645,36 @@ GemmArgs gemm_args(const ra_ctx* c, const void* A, int lda, const void* B, int l
   return g;
 }
 
-ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss, float* logits,
-                          const int32_t* labels, cudaStream_t st) {
-  const int L = ctx->L, H = ctx->H, F = ctx->F, m = ctx->m, T = B * S, act = ctx->act;
-  const int k = ctx->L - ctx->depth;
+// Encoder blocks [l0, l1) on input x with the lowest unfrozen layer k (layers >= k write
+// their saved set, layers < k keep nothing).  Scratch comes from the set fs; the block
+// outputs ping-pong through fs.X, except that the last block writes last_out when given.
+// *y_out receives the last block's output.
+ra_status encoder_blocks(ra_ctx* ctx, const void* x, int B, int S, int l0, int l1, int k,
+                         const ra_ctx::FwdScratch& fs, void* last_out, const void** y_out,
+                         cudaStream_t st) {
+  const int H = ctx->H, F = ctx->F, m = ctx->m, T = B * S, act = ctx->act;
   const void* xin = x;
   int out_idx = 0;
-  for (int l = 0; l < L; ++l) {
+  for (int l = l0; l < l1; ++l) {
     const LayerWOff& o = ctx->lw[l];
     const bool saved = l >= k, full = l > k;
     char* sb = saved ? ctx->slot(l) : nullptr;
     const SlotOff& so = ctx->so;
-    void* qkv = full ? sb + so.qkv : ctx->ws<char>(ctx->s_qkv);
-    void* O = full ? sb + so.O : ctx->ws<char>(ctx->s_O);
+    void* qkv = full ? sb + so.qkv : ctx->ws<char>(fs.qkv);
+    void* O = full ? sb + so.O : ctx->ws<char>(fs.O);
     float* lse = full ? (float*)(sb + so.lse) : nullptr;
-    void* a = saved ? sb + so.a : ctx->ws<char>(ctx->s_a);
+    void* a = saved ? sb + so.a : ctx->ws<char>(fs.a);
     float* zA = saved ? (float*)(sb + so.zA) : nullptr;
     void* xhat1 = saved ? sb + so.xhat1 : nullptr;
     float* rstd1 = saved ? (float*)(sb + so.rstd1) : nullptr;
     void* gp = saved ? sb + so.gp : nullptr;
-    void* f = saved ? sb + so.f : ctx->ws<char>(ctx->s_f);
+    void* f = saved ? sb + so.f : ctx->ws<char>(fs.f);
     float* zF = saved ? (float*)(sb + so.zF) : nullptr;
     void* xhat2 = saved ? sb + so.xhat2 : nullptr;
     float* rstd2 = saved ? (float*)(sb + so.rstd2) : nullptr;
-    void* y1 = ctx->ws<char>(ctx->s_y1);
-    void* hbuf = ctx->ws<char>(ctx->s_h);
-    void* xout = ctx->ws<char>(ctx->s_X[out_idx]);
+    void* y1 = ctx->ws<char>(fs.y1);
+    void* hbuf = ctx->ws<char>(fs.h);
+    void* xout = (last_out && l + 1 == l1) ? last_out : ctx->ws<char>(fs.X[out_idx]);
     const float* Pl = ctx->P() + (size_t)l * 4 * H * m;
 
     GemmArgs g = gemm_args(ctx, xin, H, ctx->w(o.Wqkv), H, T, 3 * H, H);
@@ -660,7 +688,7 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     CU(P_attn_fwd(ctx, at, st));
     if (ctx->post_ffn) {
       // Fig. 1 placement: y1 = LN1(x + a); y2 = LN2(y1 + f); out = y2 + GELU(y2 Wd) Wu
-      void* a_s = ctx->ws<char>(ctx->s_a);
+      void* a_s = ctx->ws<char>(fs.a);
       g = gemm_args(ctx, O, H, ctx->w(o.Wo), H, T, H, H);
       g.C = a_s; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.bo);
       CU(P_gemm(ctx, g, st));
@@ -674,7 +702,7 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
       g.C = full ? gp : nullptr; g.ldc = F; g.c_dtype = act; g.bias = ctx->w<float>(o.b1);
       g.C2 = hbuf; g.ldc2 = F; g.c2_dtype = act;
       CU(P_gemm(ctx, g, st));
-      void* f_s = ctx->ws<char>(ctx->s_f);
+      void* f_s = ctx->ws<char>(fs.f);
       g = gemm_args(ctx, hbuf, F, ctx->w(o.W2), F, T, H, F);
       g.C = f_s; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.b2);
       CU(P_gemm(ctx, g, st));
@@ -691,7 +719,6 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
       ad.y = xout;
       CU(P_adapter_fwd(ctx, ad, st));
       xin = xout;
-      ctx->top_out = out_idx;
       out_idx ^= 1;
       continue;
     }
@@ -720,9 +747,17 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
     ad.y = xout; ad.xhat = xhat2; ad.rstd = rstd2;
     CU(P_adapter_fwd(ctx, ad, st));
     xin = xout;
-    ctx->top_out = out_idx;
     out_idx ^= 1;
   }
+  *y_out = xin;
+  return RA_OK;
+}
+
+// Encoder head and loss on the last block's output y.
+ra_status encoder_head_forward(ra_ctx* ctx, const void* xin, int B, int S, float* loss,
+                               float* logits, const int32_t* labels, cudaStream_t st) {
+  const int L = ctx->L, H = ctx->H, m = ctx->m, T = B * S, act = ctx->act;
+  ctx->yL = xin;
   float* Ph = ctx->P() + (size_t)L * 4 * H * m;
   if (ctx->span) {
     // span head: start and end logits at every token of the last block's output
@@ -739,6 +774,14 @@ ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss,
                             logits, ctx->ws<float>(ctx->h_dlogits), ctx->ws<unsigned>(ctx->ws_err), st);
   }));
   return RA_OK;
+}
+
+ra_status encoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss, float* logits,
+                          const int32_t* labels, cudaStream_t st) {
+  const void* y = nullptr;
+  ra_status r = encoder_blocks(ctx, x, B, S, 0, ctx->L, ctx->L - ctx->depth, ctx->fs[0], nullptr, &y, st);
+  if (r != RA_OK) return r;
+  return encoder_head_forward(ctx, y, B, S, loss, logits, labels, st);
 }
 
 ra_status decoder_forward(ra_ctx* ctx, const void* x, int B, int S, float* loss, float* logits,
@@ -864,6 +907,64 @@ ra_status ra_forward(ra_ctx* ctx, const void* x_dev, const int32_t* labels_dev, 
   return RA_OK;
 }
 
+ra_status ra_forward_prefix(ra_ctx* ctx, const void* x_dev, int32_t B, int32_t S, int32_t buf,
+                            ra_stream_t stream) {
+  if (!ctx) return RA_ERR_ARG;
+  if (!ctx->prefix_bufs)
+    return fail(ctx, RA_ERR_UNSUPPORTED, "no prefix buffers (encoder with cfg.prefix_buffers = 1)");
+  if (!ctx->W) return fail(ctx, RA_ERR_STATE, "ra_bind_memory first");
+  if (!ctx->weights_ready) return fail(ctx, RA_ERR_STATE, "not every parameter was set");
+  if (!x_dev) return fail(ctx, RA_ERR_ARG, "null input");
+  if (buf < 0 || buf > 1) return fail(ctx, RA_ERR_ARG, "buf %d not 0 or 1", buf);
+  if (B < 1 || S < 1) return fail(ctx, RA_ERR_ARG, "empty batch");
+  if (B > ctx->cfg.max_batch || S > ctx->cfg.max_seq)
+    return fail(ctx, RA_ERR_SHAPE, "B=%d S=%d beyond capacity %d x %d", B, S,
+                ctx->cfg.max_batch, ctx->cfg.max_seq);
+  CU(cudaSetDevice(ctx->device));
+  cudaStream_t st = (cudaStream_t)stream;
+  const int k = ctx->L - ctx->depth;
+  void* out = ctx->ws<char>(ctx->pbuf[buf]);
+  ctx->pf[buf].valid = false;
+  if (k == 0) {
+    CU(cudaMemcpyAsync(out, x_dev, (size_t)B * S * ctx->H * dtype_size(ctx->act),
+                       cudaMemcpyDeviceToDevice, st));
+  } else {
+    const void* y = nullptr;
+    ra_status r = encoder_blocks(ctx, x_dev, B, S, 0, k, k, ctx->fs[1], out, &y, st);
+    if (r != RA_OK) return r;
+  }
+  ctx->pf[buf] = {true, k, B, S};
+  return RA_OK;
+}
+
+ra_status ra_forward_suffix(ra_ctx* ctx, int32_t buf, const int32_t* labels_dev, float* loss_dev,
+                            float* logits_dev, ra_stream_t stream) {
+  if (!ctx) return RA_ERR_ARG;
+  if (!ctx->prefix_bufs)
+    return fail(ctx, RA_ERR_UNSUPPORTED, "no prefix buffers (encoder with cfg.prefix_buffers = 1)");
+  if (buf < 0 || buf > 1) return fail(ctx, RA_ERR_ARG, "buf %d not 0 or 1", buf);
+  if (!labels_dev || !loss_dev) return fail(ctx, RA_ERR_ARG, "null input");
+  const int k = ctx->L - ctx->depth;
+  const ra_ctx::PrefixState p = ctx->pf[buf];
+  if (!p.valid) return fail(ctx, RA_ERR_STATE, "no ra_forward_prefix filled buffer %d", buf);
+  if (p.k != k)
+    return fail(ctx, RA_ERR_STATE, "the prefix in buffer %d stops at layer %d, the depth now needs %d",
+                buf, p.k, k);
+  CU(cudaSetDevice(ctx->device));
+  cudaStream_t st = (cudaStream_t)stream;
+  const void* y = nullptr;
+  ra_status r = encoder_blocks(ctx, ctx->ws<char>(ctx->pbuf[buf]), p.B, p.S, k, ctx->L, k, ctx->fs[0],
+                               nullptr, &y, st);
+  if (r == RA_OK) r = encoder_head_forward(ctx, y, p.B, p.S, loss_dev, logits_dev, labels_dev, st);
+  if (r != RA_OK) return r;
+  ctx->k_fwd = k;
+  ctx->fB = p.B;
+  ctx->fS = p.S;
+  ctx->labels = labels_dev;
+  ctx->k_bwd = -1;
+  return RA_OK;
+}
+
 // ---- backward ----------------------------------------------------------------------------
 ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
   if (!ctx) return RA_ERR_ARG;
@@ -884,7 +985,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
     // every token receives a gradient: the span head writes all of dY
     float* Ph = ctx->P() + (size_t)L * 4 * H * m;
     float* Gh = ctx->G() + (size_t)L * 4 * H * m;
-    const void* yL = ctx->ws(ctx->s_X[ctx->top_out]);
+    const void* yL = ctx->yL;
     CU(prof(ctx, RA_PROF_HEAD, 8.0 * T * H, (double)T * H * (dtype_size(act) + 4), st, [&] {
       return span_head_bwd(yL, act, Ph, ctx->ws<float>(ctx->h_dlogits), B, S, H,
                            ctx->cfg.head_trainable ? Gh : nullptr,
@@ -895,7 +996,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
     float* Ph = ctx->P() + (size_t)L * 4 * H * m;
     float* Gh = ctx->G() + (size_t)L * 4 * H * m;
     CU(cudaMemsetAsync(dY, 0, (size_t)T * H * 4, st));
-    const void* yL = ctx->ws(ctx->s_X[ctx->top_out]);
+    const void* yL = ctx->yL;
     CU(prof(ctx, RA_PROF_HEAD, 4.0 * B * H * ctx->C, (double)B * H * (dtype_size(act) + 4), st, [&] {
       return encoder_head_bwd(yL, act, Ph, ctx->ws<float>(ctx->h_dlogits), B, S, H, ctx->C,
                               ctx->cfg.head_trainable ? Gh : nullptr,

@@ -50,7 +50,7 @@ class ra_model_cfg(C.Structure):
                 ("max_batch", C.c_int32), ("max_seq", C.c_int32), ("dtype", C.c_int32),
                 ("head_trainable", C.c_int32), ("max_depth", C.c_int32),
                 ("norm_eps", C.c_float), ("rope_theta", C.c_float),
-                ("adapter_placement", C.c_int32)]
+                ("adapter_placement", C.c_int32), ("prefix_buffers", C.c_int32)]
 
 
 class ra_adam_cfg(C.Structure):
@@ -101,6 +101,10 @@ _SIGS = {
     "ra_schedule_depth": (C.c_int32, [C.c_int32, C.c_int32, C.c_int32, C.c_int32]),
     "ra_forward": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32,
                              C.c_void_p, C.c_void_p, C.c_void_p]),
+    "ra_forward_prefix": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
+                                    C.c_void_p]),
+    "ra_forward_suffix": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
+                                    C.c_void_p]),
     "ra_backward_truncated": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p]),
     "ra_adapter_update": (C.c_int, [C.c_void_p, C.POINTER(ra_adam_cfg), C.c_void_p]),
     "ra_get_grad": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.POINTER(C.c_void_p),
@@ -197,6 +201,15 @@ def ra_set_unfrozen_depth(ctx, d: int):
 def ra_forward(ctx, x_ptr, labels_ptr, B, S, loss_ptr, logits_ptr=None, stream=None):
     _check(lib().ra_forward(ctx, x_ptr, labels_ptr, B, S, loss_ptr, logits_ptr,
                             _stream_ptr(stream)), ctx)
+
+
+def ra_forward_prefix(ctx, x_ptr, B, S, buf, stream=None):
+    _check(lib().ra_forward_prefix(ctx, x_ptr, B, S, buf, _stream_ptr(stream)), ctx)
+
+
+def ra_forward_suffix(ctx, buf, labels_ptr, loss_ptr, logits_ptr=None, stream=None):
+    _check(lib().ra_forward_suffix(ctx, buf, labels_ptr, loss_ptr, logits_ptr,
+                                   _stream_ptr(stream)), ctx)
 
 
 def ra_backward_truncated(ctx, k: int, stream=None):
@@ -323,9 +336,10 @@ def schedule_depth(step_index: int, interval: int = 50, d0: int = 1, d_max: int 
 
 def make_cfg(arch, n_layers, hidden, n_heads, ffn, n_out, max_batch, max_seq, dtype,
              head_trainable, max_depth=0, norm_eps=1e-12, rope_theta=10000.0,
-             adapter_placement=0):
+             adapter_placement=0, prefix_buffers=0):
     return ra_model_cfg(arch, n_layers, hidden, n_heads, ffn, n_out, max_batch, max_seq, dtype,
-                        head_trainable, max_depth, norm_eps, rope_theta, adapter_placement)
+                        head_trainable, max_depth, norm_eps, rope_theta, adapter_placement,
+                        prefix_buffers)
 
 
 class Model:
