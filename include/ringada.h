@@ -317,6 +317,23 @@ int64_t ra_kernel_launches(void);
 ra_status ra_gemm_bf16(const void* A_dev, const void* B_dev, void* C_dev, int32_t M, int32_t N,
                        int32_t K, const float* bias_dev, void* gelu_out_dev, ra_stream_t stream);
 
+/* The same tensor-core GEMM with one of the step's fused epilogues, for tests and kernel
+ * measurements (no counterpart in the paper: these are the step's dense contractions).
+ * C = A[M, K] B[N, K]^T accumulated in fp32 (A, B bf16, K-major: lda = ldb = K), then
+ *   RA_EPI_STORE       C = acc (+ bias)                  (C bf16 or f32: c_dtype)
+ *   RA_EPI_BIAS_GELU   u = acc + bias: C = u (nullable), C2 = GELU(u)     (bf16)
+ *   RA_EPI_BIAS_GELU_G u = acc + bias: C = GELU'(u) (nullable), C2 = GELU(u) (bf16)
+ *   RA_EPI_MUL         C = acc * aux                     (aux bf16 [M, N], C c_dtype)
+ *   RA_EPI_RESID       C = acc + aux                     (aux f32 [M, N], C f32)
+ * Outputs are [M, N] row-major with leading dimension N.  bias: nullable f32 [N].  Device
+ * pointers, 16-byte aligned; N and K multiples of 8.  Enqueued on stream.  RA_ERR_SHAPE
+ * for a combination the kernel does not take, RA_ERR_UNSUPPORTED without sm_103. */
+enum { RA_EPI_STORE = 0, RA_EPI_BIAS_GELU = 1, RA_EPI_MUL = 2, RA_EPI_RESID = 3,
+       RA_EPI_BIAS_GELU_G = 6 };
+ra_status ra_gemm_bf16_epi(const void* A_dev, const void* B_dev, int32_t M, int32_t N, int32_t K,
+                           int32_t epi, const float* bias_dev, const void* aux_dev, void* C_dev,
+                           int32_t c_dtype, void* C2_dev, ra_stream_t stream);
+
 /* Adapter backward of Eq. 1 for T rows (the in-kernel weight-gradient reduction of the
  * step), float32 throughout.  g_dev [T, H] = dLoss/d(adapter output); h_dev [T, H] the
  * adapter input; z_dev [T, m] = h W_down saved by the forward; W_down [H, m], W_up [m, H].

@@ -632,8 +632,10 @@ cudaError_t attention_fwd_mma(const AttnArgs& a, cudaStream_t st) {
   return a.head_dim == 64 ? fwd<64>(a, st) : fwd<128>(a, st);
 }
 
-// expects D = rowsum(dO * O) already in a.Dscratch
+// expects D = rowsum(dO * O) already in a.Dscratch; the encoders' short sequences take the
+// tcgen05 kernel
 cudaError_t attention_bwd_mma(const AttnArgs& a, cudaStream_t st) {
+  if (attention_tc_ok(a) && a.lse) return attention_bwd_tc(a, st);
   return a.head_dim == 64 ? bwd<64>(a, st) : bwd<128>(a, st);
 }
 

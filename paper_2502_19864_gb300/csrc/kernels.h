@@ -111,6 +111,8 @@ cudaError_t attention_bwd_mma(const AttnArgs& a, cudaStream_t st);
 // tcgen05 forward (bf16, head_dim 64, no mask or RoPE, S <= 256)
 bool attention_tc_ok(const AttnArgs& a);
 cudaError_t attention_fwd_tc(const AttnArgs& a, cudaStream_t st);
+// tcgen05 backward for the same shapes; expects D = rowsum(dO * O) in a.Dscratch
+cudaError_t attention_bwd_tc(const AttnArgs& a, cudaStream_t st);
 
 // ---------------------------------------------------------------------------------------
 // Row-wise fused kernels

@@ -1415,6 +1415,43 @@ ra_status ra_gemm_bf16(const void* A_dev, const void* B_dev, void* C_dev, int32_
   return e == cudaSuccess ? RA_OK : RA_ERR_CUDA;
 }
 
+ra_status ra_gemm_bf16_epi(const void* A_dev, const void* B_dev, int32_t M, int32_t N, int32_t K,
+                           int32_t epi, const float* bias_dev, const void* aux_dev, void* C_dev,
+                           int32_t c_dtype, void* C2_dev, ra_stream_t stream) {
+  if (!A_dev || !B_dev || M < 0 || N <= 0 || K <= 0) return RA_ERR_ARG;
+  if (c_dtype != RA_F32 && c_dtype != RA_BF16) return RA_ERR_ARG;
+  if (K % 8 || N % 8) return RA_ERR_SHAPE;
+  GemmArgs g;
+  g.A = A_dev; g.lda = K; g.B = B_dev; g.ldb = K; g.M = M; g.N = N; g.K = K;
+  g.in_dtype = DT_BF16;
+  g.C = C_dev; g.ldc = N; g.c_dtype = c_dtype == RA_BF16 ? DT_BF16 : DT_F32;
+  switch (epi) {
+    case RA_EPI_STORE:
+      if (!C_dev) return RA_ERR_ARG;
+      g.epi = EPI_STORE; g.bias = bias_dev;
+      break;
+    case RA_EPI_BIAS_GELU:
+    case RA_EPI_BIAS_GELU_G:
+      if (!C2_dev || c_dtype != RA_BF16) return RA_ERR_ARG;
+      g.epi = epi == RA_EPI_BIAS_GELU ? EPI_BIAS_GELU : EPI_BIAS_GELU_G;
+      g.bias = bias_dev; g.C2 = C2_dev; g.ldc2 = N; g.c2_dtype = DT_BF16;
+      break;
+    case RA_EPI_MUL:
+      if (!C_dev || !aux_dev) return RA_ERR_ARG;
+      g.epi = EPI_MUL; g.aux = aux_dev; g.ldaux = N; g.aux_dtype = DT_BF16;
+      break;
+    case RA_EPI_RESID:
+      if (!C_dev || !aux_dev || c_dtype != RA_F32) return RA_ERR_ARG;
+      g.epi = EPI_RESID; g.aux = aux_dev; g.ldaux = N; g.aux_dtype = DT_F32;
+      break;
+    default: return RA_ERR_ARG;
+  }
+  if (!tc_available()) return RA_ERR_UNSUPPORTED;
+  cudaError_t e = gemm_tc(g, (cudaStream_t)stream);
+  if (e == cudaErrorNotSupported) return RA_ERR_SHAPE;
+  return e == cudaSuccess ? RA_OK : RA_ERR_CUDA;
+}
+
 size_t ra_adapter_backward_scratch_bytes(int32_t T, int32_t H, int32_t m) {
   if (T < 1 || H < 1 || m < 1) return 0;
   return adapter_bwd_partials_floats(T, H, m) * 4 + (size_t)T * m * 4 + 2 * (size_t)H * m * 4 + 3 * kAlign;

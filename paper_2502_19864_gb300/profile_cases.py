@@ -3,8 +3,9 @@
   python -m paper_2502_19864_gb300.profile_cases gemm M N K [--reps R] [--gelu]
       R launches of the tensor-core GEMM C[M,N] = A[M,K] B[N,K]^T (bf16, via ra_gemm_bf16);
       --gelu adds the bias + GELU epilogue (writes C and GELU(C))
-  python -m paper_2502_19864_gb300.profile_cases step CONFIG D [--reps R]
-      R eager steps (forward, early-stopped backward, update) of a synthetic workload
+  python -m paper_2502_19864_gb300.profile_cases step CONFIG D [--reps R] [--layers N]
+      R eager steps (forward, early-stopped backward, update) of a synthetic workload; with
+      --layers, the workload's per-layer shapes on N layers (a smaller device footprint)
 
 Inputs are seeded synthetic data; every call goes through the C ABI.
 """
@@ -33,16 +34,23 @@ def gemm_case(M, N, K, reps, gelu=False):
     print("gemm %dx%dx%d x%d done" % (M, N, K, reps))
 
 
-def step_case(name, d, reps):
+def step_case(name, d, reps, layers=None):
+    import dataclasses
     import torch
     import synth
     from paper_2502_19864_gb300 import ringada as R
     cfg = synth.CONFIGS[name]
+    if layers:
+        cfg = dataclasses.replace(cfg, n_layers=layers)
     w = synth.make_workload(cfg, 0)
-    arch = R.RA_ENCODER_POSTLN if cfg.arch == "encoder" else R.RA_DECODER_PRENORM
+    if cfg.arch == "decoder":
+        arch = R.RA_DECODER_PRENORM
+    else:
+        arch = R.RA_ENCODER_POSTLN_SPAN if cfg.head == "span" else R.RA_ENCODER_POSTLN
+    placement = R.RA_ADAPTERS_POST_FFN if cfg.adapters == "paper" else R.RA_ADAPTERS_HOULSBY
     m = R.Model(R.make_cfg(arch, cfg.n_layers, cfg.hidden, cfg.n_heads, cfg.ffn, cfg.n_out,
                            cfg.batch, cfg.seq, R.RA_BF16 if cfg.dtype == "bf16" else R.RA_F32,
-                           int(cfg.head_trainable), 0, cfg.norm_eps, cfg.rope_theta),
+                           int(cfg.head_trainable), 0, cfg.norm_eps, cfg.rope_theta, placement),
                 cfg.adapter_dim)
     m.set_weights(w["layers"], w["head"])
     dt = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
@@ -65,6 +73,7 @@ def main():
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--gelu", action="store_true")
+    ap.add_argument("--layers", type=int, default=None)
     a = ap.parse_args()
     import __graft_entry__
     __graft_entry__.build()
@@ -72,7 +81,7 @@ def main():
         M, N, K = (int(v) for v in a.args[:3])
         gemm_case(M, N, K, a.reps, a.gelu)
     else:
-        step_case(a.args[0], int(a.args[1]), a.reps)
+        step_case(a.args[0], int(a.args[1]), a.reps, a.layers)
 
 
 if __name__ == "__main__":

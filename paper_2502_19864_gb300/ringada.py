@@ -122,6 +122,9 @@ _SIGS = {
     "ra_destroy": (None, [C.c_void_p]),
     "ra_gemm_bf16": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32,
                                C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "ra_gemm_bf16_epi": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
+                                   C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
+                                   C.c_void_p, C.c_void_p]),
     "ra_adapter_backward": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                       C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
                                       C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]),
@@ -279,6 +282,15 @@ def ra_destroy(ctx):
 
 def ra_gemm_bf16(A_ptr, B_ptr, C_ptr, M, N, K, bias_ptr=None, gelu_ptr=None, stream=None):
     _check(lib().ra_gemm_bf16(A_ptr, B_ptr, C_ptr, M, N, K, bias_ptr, gelu_ptr, _stream_ptr(stream)))
+
+
+RA_EPI_STORE, RA_EPI_BIAS_GELU, RA_EPI_MUL, RA_EPI_RESID, RA_EPI_BIAS_GELU_G = 0, 1, 2, 3, 6
+
+
+def ra_gemm_bf16_epi(A_ptr, B_ptr, M, N, K, epi, bias_ptr=None, aux_ptr=None, C_ptr=None,
+                     c_dtype=RA_BF16, C2_ptr=None, stream=None):
+    _check(lib().ra_gemm_bf16_epi(A_ptr, B_ptr, M, N, K, epi, bias_ptr, aux_ptr, C_ptr, c_dtype,
+                                  C2_ptr, _stream_ptr(stream)))
 
 
 def ra_adapter_backward_scratch_bytes(T, H, m) -> int:

@@ -90,6 +90,11 @@ CONFIGS: Dict[str, ModelCfg] = {
     # the paper's placement: one adapter per block, after the FFN add & LayerNorm
     "tiny_paper": _paper(2, 128, 2, 512, 16, 4, 32, "f32"),
     "small_paper_bf16": _paper(3, 256, 4, 1024, 32, 3, 100, "bf16"),
+    # two 128-row key/query blocks with a ragged second block (S = 250)
+    "small_enc_s250_bf16": _enc(2, 256, 4, 1024, 32, 2, 250, "bf16"),
+    # the bench workloads' shapes with the other heads / placement (per-kernel profiles)
+    "base_span": _span(12, 768, 12, 3072, 64, 32, 128, "bf16"),
+    "large_paper": _paper(24, 1024, 16, 4096, 64, 32, 256, "bf16"),
 }
 
 

@@ -1,6 +1,7 @@
-"""The tcgen05 GEMM through the C ABI (ra_gemm_bf16) against a plain fp32 PyTorch matmul of
-the same bf16 operands: single tile, ragged M/N/K tails, the BERT/LLaMA shapes of the step,
-the bias and bias+GELU epilogues, and bitwise determinism."""
+"""The tcgen05 GEMM through the C ABI (ra_gemm_bf16, ra_gemm_bf16_epi) against a plain fp32
+PyTorch matmul of the same bf16 operands on the CPU: single tile, ragged M/N/K tails, the
+BERT/LLaMA shapes of the step, every fused epilogue of the step (bias, bias+GELU, the saved
+GELU' factor, the multiply by it, the fp32 residual) and bitwise determinism."""
 import numpy as np
 import pytest
 
@@ -26,7 +27,7 @@ def _run(M, N, K, bias=False, gelu=False, seed=0):
     R.ra_gemm_bf16(A.data_ptr(), B.data_ptr(), C.data_ptr(), M, N, K,
                    b.data_ptr() if bias else None, G.data_ptr() if gelu else None)
     torch.cuda.synchronize()
-    ref = A.float() @ B.float().T
+    ref = (A.float().cpu() @ B.float().cpu().T).cuda()
     if bias:
         ref = ref + b
     return C, G, ref
@@ -84,3 +85,76 @@ def test_gemm_is_deterministic():
     C2, _, _ = _run(1024, 768, 768, seed=3)
     assert bool((C1.view(-1).view(dtype=__import__("torch").int16) ==
                  C2.view(-1).view(dtype=__import__("torch").int16)).all())
+
+
+def _operands(M, N, K, seed):
+    import torch
+    g = torch.Generator(device="cpu").manual_seed(seed)
+    A = torch.randn(M, K, generator=g).to(torch.bfloat16)
+    B = (torch.randn(N, K, generator=g) * 0.05).to(torch.bfloat16)
+    acc = A.float() @ B.float().T          # CPU fp32 reference of the product
+    return A.cuda(), B.cuda(), acc, g
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 264, 136), (8192, 4096, 1024)])
+def test_gemm_gelu_factor_epilogue(M, N, K):
+    """u = acc + bias: C2 = GELU(u), C = GELU'(u) (the factor the backward multiplies by)."""
+    import torch
+    A, B, acc, g = _operands(M, N, K, 5)
+    b = torch.randn(N, generator=g) * 0.1
+    C = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda")
+    G = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda")
+    bd = b.cuda()
+    R.ra_gemm_bf16_epi(A.data_ptr(), B.data_ptr(), M, N, K, R.RA_EPI_BIAS_GELU_G, bd.data_ptr(),
+                       None, C.data_ptr(), R.RA_BF16, G.data_ptr())
+    torch.cuda.synchronize()
+    u = (acc + b).double()
+    phi = torch.exp(-0.5 * u * u) / (2 * torch.pi) ** 0.5
+    Phi = 0.5 * (1 + torch.erf(u / 2 ** 0.5))
+    _check(G, (u * Phi).float().cuda(), tol=1e-2)
+    _check(C, (Phi + u * phi).float().cuda(), tol=1e-2)
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 264, 136), (8192, 4096, 1024)])
+def test_gemm_multiply_epilogue(M, N, K):
+    """C = acc * aux with a bf16 aux operand (the backward's dH GEMM)."""
+    import torch
+    A, B, acc, g = _operands(M, N, K, 6)
+    aux = (torch.rand(M, N, generator=g) * 1.2).to(torch.bfloat16)
+    C = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda")
+    auxd = aux.cuda()
+    R.ra_gemm_bf16_epi(A.data_ptr(), B.data_ptr(), M, N, K, R.RA_EPI_MUL, None, auxd.data_ptr(),
+                       C.data_ptr(), R.RA_BF16)
+    torch.cuda.synchronize()
+    _check(C, (acc * aux.float()).cuda())
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 264, 136), (8192, 1024, 3072)])
+def test_gemm_residual_epilogue(M, N, K):
+    """C = acc + aux, fp32 aux and output (the dX GEMM of the post-FFN adapter placement)."""
+    import torch
+    A, B, acc, g = _operands(M, N, K, 7)
+    aux = torch.randn(M, N, generator=g)
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    auxd = aux.cuda()
+    R.ra_gemm_bf16_epi(A.data_ptr(), B.data_ptr(), M, N, K, R.RA_EPI_RESID, None, auxd.data_ptr(),
+                       C.data_ptr(), R.RA_F32)
+    torch.cuda.synchronize()
+    ref = (acc + aux).cuda()
+    assert not bool(C.isnan().any())
+    # fp32 output: only accumulation-order differences remain
+    assert (C - ref).abs().max().item() <= 1e-4 * ref.abs().max().item()
+
+
+def test_gemm_f32_store_epilogue():
+    """C = acc in fp32 (the encoder's dX GEMMs), no bias."""
+    import torch
+    M, N, K = 8192, 1024, 4096
+    A, B, acc, _ = _operands(M, N, K, 8)
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    R.ra_gemm_bf16_epi(A.data_ptr(), B.data_ptr(), M, N, K, R.RA_EPI_STORE, None, None,
+                       C.data_ptr(), R.RA_F32)
+    torch.cuda.synchronize()
+    ref = acc.cuda()
+    assert not bool(C.isnan().any())
+    assert (C - ref).abs().max().item() <= 1e-4 * ref.abs().max().item()

@@ -41,7 +41,7 @@ def test_fp32_parity_every_depth(name):
 
 
 @pytest.mark.parametrize("name", ["small_enc_bf16", "small_dec_bf16", "small_span_bf16",
-                                  "small_paper_bf16"])
+                                  "small_paper_bf16", "small_enc_s250_bf16"])
 def test_bf16_parity_every_depth(name):
     _parity_all_depths(name)
 
