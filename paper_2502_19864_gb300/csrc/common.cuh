@@ -105,6 +105,13 @@ __device__ __forceinline__ float silu_grad_f(float x) {
   return s * (1.0f + x * (1.0f - s));
 }
 
+// ---- RoPE ---------------------------------------------------------------------------------
+// inverse frequency of rotate-half pair i of a head of dh dims: theta^(-2 i / dh); the angle
+// at position s is s times this (every RoPE kernel evaluates it this way)
+__device__ __forceinline__ float rope_freq(int i, int dh, float theta) {
+  return expf(-logf(theta) * (2.0f * (float)i / (float)dh));
+}
+
 // ---- programmatic dependent launch ----------------------------------------------------
 // A kernel started with launch_pdl may begin while the kernel before it in the stream is
 // still finishing.  pdl_wait() blocks until that kernel has completed and its writes are

@@ -627,15 +627,18 @@ cudaError_t rope_qk_inplace(const AttnArgs& a, cudaStream_t st) {
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+// the tcgen05 kernels take every bf16 shape whose q and k are plain or rotated in place:
+// the one-block forward for the encoders' short sequences, the block-looping forward for
+// longer (the decoder's causal) ones; mma.sync stays for RoPE applied while staging
 cudaError_t attention_fwd_mma(const AttnArgs& a, cudaStream_t st) {
   if (attention_tc_ok(a)) return attention_fwd_tc(a, st);
+  if (attention_fwd_blocks_tc_ok(a)) return attention_fwd_blocks_tc(a, st);
   return a.head_dim == 64 ? fwd<64>(a, st) : fwd<128>(a, st);
 }
 
-// expects D = rowsum(dO * O) already in a.Dscratch; the encoders' short sequences take the
-// tcgen05 kernel
+// expects D = rowsum(dO * O) already in a.Dscratch
 cudaError_t attention_bwd_mma(const AttnArgs& a, cudaStream_t st) {
-  if (attention_tc_ok(a) && a.lse) return attention_bwd_tc(a, st);
+  if (attention_bwd_tc_ok(a)) return attention_bwd_tc(a, st);
   return a.head_dim == 64 ? bwd<64>(a, st) : bwd<128>(a, st);
 }
 

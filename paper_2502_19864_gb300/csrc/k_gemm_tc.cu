@@ -215,7 +215,7 @@ struct EpiIn {
 struct F8 {
   float v[8];
 };
-__device__ __noinline__ F8 gelu8(F8 x) {
+__device__ __forceinline__ F8 gelu8(F8 x) {
 #pragma unroll
   for (int i = 0; i < 8; i += 2) {
     const float2 y = gelu2(make_float2(x.v[i], x.v[i + 1]));
@@ -228,7 +228,7 @@ __device__ __noinline__ F8 gelu8(F8 x) {
 struct F8x2 {
   F8 y, d;
 };
-__device__ __noinline__ F8x2 gelu_both8(F8 x) {
+__device__ __forceinline__ F8x2 gelu_both8(F8 x) {
   F8x2 r;
 #pragma unroll
   for (int i = 0; i < 8; i += 2) {

@@ -702,53 +702,78 @@ constexpr int SPAN_CHUNKS = 32;   // token chunks of the deterministic dWh reduc
 // logits at once) into shared memory; warp c then takes the softmax over S of column c and
 // writes dlogits[t, c] = (p_c(s) - [s == label_c]) / (2 B); row_loss[b] = mean of the two
 // cross-entropies.
+// Span head logits: a warp per token, z[t] = (y_t . Wh[0] + bh[0], y_t . Wh[1] + bh[1]) into
+// zout [T][2] (the dlogits buffer, which the softmax kernel then overwrites in place).
+// 16-byte loads of y (8 bf16 or 4 f32 per load, H a multiple of 8).
 template <typename T>
-__global__ void __launch_bounds__(256) span_head_fwd_kernel(const void* y, const float* Wh,
-    const float* bh, const int32_t* labels, int B, int S, int H, float* row_loss,
-    float* logits_out, float* dlogits, unsigned* err) {
-  extern __shared__ float zs[];  // [S][2]
+__global__ void __launch_bounds__(256) span_head_logits_kernel(const void* y, const float* Wh,
+    const float* bh, int Tn, int H, float* zout) {
+  pdl_wait();
+  pdl_trigger();
+  const int64_t t = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (t >= Tn) return;
+  constexpr int V = 16 / sizeof(T);  // elements per 16-byte load
+  const T* row = reinterpret_cast<const T*>(y) + t * H;
+  float a0 = 0.f, a1 = 0.f;
+  for (int i = lane * V; i < H; i += 32 * V) {
+    const uint4 u = *reinterpret_cast<const uint4*>(row + i);
+    float x[V];
+    if (V == 8) {
+      const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+      for (int k = 0; k < V / 2; ++k) {
+        const float2 f = __bfloat1622float2(h2[k]);
+        x[2 * k] = f.x;
+        x[2 * k + 1] = f.y;
+      }
+    } else {
+      const float* f = reinterpret_cast<const float*>(&u);
+#pragma unroll
+      for (int k = 0; k < V; ++k) x[k] = f[k];
+    }
+#pragma unroll
+    for (int k = 0; k < V; ++k) {
+      a0 = fmaf(x[k], __ldg(Wh + i + k), a0);
+      a1 = fmaf(x[k], __ldg(Wh + H + i + k), a1);
+    }
+  }
+  a0 = warp_sum(a0);
+  a1 = warp_sum(a1);
+  if (lane == 0) *reinterpret_cast<float2*>(zout + 2 * t) = make_float2(a0 + bh[0], a1 + bh[1]);
+}
+
+// Span head softmax and cross-entropy, one CTA per sequence: the start (c = 0) and end (c = 1)
+// columns take a warp each.  z [T][2] arrives in dlogits and is replaced by the gradient.
+__global__ void __launch_bounds__(64) span_head_ce_kernel(const int32_t* labels, int B, int S,
+    float* row_loss, float* logits_out, float* dlogits, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float part[2];
-  const int b = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-  for (int s = warp; s < S; s += nw) {
-    const int64_t row = ((int64_t)b * S + s) * H;
-    float a0 = 0.f, a1 = 0.f;
-#pragma unroll 8
-    for (int i = lane; i < H; i += 32) {
-      const float x = ldf<T>(y, row + i);
-      a0 += x * __ldg(Wh + i);
-      a1 += x * __ldg(Wh + H + i);
-    }
-    a0 = warp_sum(a0);
-    a1 = warp_sum(a1);
-    if (lane == 0) {
-      zs[2 * s] = a0 + bh[0];
-      zs[2 * s + 1] = a1 + bh[1];
-    }
+  const int b = blockIdx.x, c = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float* z = dlogits + (int64_t)b * S * 2;
+  int lab = labels[2 * b + c];
+  if (lab < 0 || lab >= S) {
+    if (lane == 0) set_dev_error(err, RA_DEVERR_BOUNDS);
+    lab = 0;
   }
-  __syncthreads();
-  if (warp < 2) {
-    const int c = warp;
-    int lab = labels[2 * b + c];
-    if (lab < 0 || lab >= S) {
-      if (lane == 0) set_dev_error(err, RA_DEVERR_BOUNDS);
-      lab = 0;
-    }
-    float mx = -INFINITY;
-    for (int s = lane; s < S; s += 32) mx = fmaxf(mx, zs[2 * s + c]);
-    mx = warp_max(mx);
-    float se = 0.f;
-    for (int s = lane; s < S; s += 32) se += expf(zs[2 * s + c] - mx);
-    se = warp_sum(se);
-    const float lse = mx + logf(se);
-    const float inv = 1.f / (2.f * B);
-    for (int s = lane; s < S; s += 32) {
-      const int64_t t = (int64_t)b * S + s;
-      const float z = zs[2 * s + c];
-      if (logits_out) logits_out[2 * t + c] = z;
-      dlogits[2 * t + c] = (expf(z - lse) - (s == lab ? 1.f : 0.f)) * inv;
-    }
-    if (lane == 0) part[c] = lse - zs[2 * lab + c];
+  float mx = -INFINITY;
+  for (int s = lane; s < S; s += 32) mx = fmaxf(mx, z[2 * s + c]);
+  mx = warp_max(mx);
+  float se = 0.f;
+  for (int s = lane; s < S; s += 32) se += expf(z[2 * s + c] - mx);
+  se = warp_sum(se);
+  const float lse = mx + logf(se);
+  const float zlab = z[2 * lab + c];
+  __syncwarp();
+  const float inv = 1.f / (2.f * B);
+  for (int s = lane; s < S; s += 32) {
+    const int64_t t = (int64_t)b * S + s;
+    const float zz = dlogits[2 * t + c];
+    if (logits_out) logits_out[2 * t + c] = zz;
+    dlogits[2 * t + c] = (expf(zz - lse) - (s == lab ? 1.f : 0.f)) * inv;
   }
+  if (lane == 0) part[c] = lse - zlab;
   __syncthreads();
   if (threadIdx.x == 0) row_loss[b] = 0.5f * (part[0] + part[1]);
 }
@@ -1152,16 +1177,16 @@ int span_head_chunks() { return SPAN_CHUNKS; }
 cudaError_t span_head_fwd(const void* y, int dtype, const float* Wh, const float* bh,
                           const int32_t* labels, int B, int S, int H, float* row_loss, float* loss,
                           float* logits_out, float* dlogits, unsigned* err, cudaStream_t st) {
-  if (S < 1 || S > SPAN_MAX_SEQ || B < 1) return cudaErrorInvalidValue;
-  const size_t smem = (size_t)2 * S * sizeof(float);
-  if (dtype == DT_BF16)
-    span_head_fwd_kernel<bf16><<<B, 256, smem, st>>>(y, Wh, bh, labels, B, S, H, row_loss, logits_out, dlogits, err);
-  else
-    span_head_fwd_kernel<float><<<B, 256, smem, st>>>(y, Wh, bh, labels, B, S, H, row_loss, logits_out, dlogits, err);
-  cudaError_t e = cudaGetLastError();
+  if (S < 1 || S > SPAN_MAX_SEQ || B < 1 || H % 8) return cudaErrorInvalidValue;
+  const int T = B * S;
+  cudaError_t e = dtype == DT_BF16
+      ? launch_pdl(span_head_logits_kernel<bf16>, dim3(blocks_for(T, 8)), dim3(256), (size_t)0, st, y, Wh, bh, T, H, dlogits)
+      : launch_pdl(span_head_logits_kernel<float>, dim3(blocks_for(T, 8)), dim3(256), (size_t)0, st, y, Wh, bh, T, H, dlogits);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(span_head_ce_kernel, dim3(B), dim3(64), (size_t)0, st, labels, B, S, row_loss, logits_out, dlogits, err);
   if (e != cudaSuccess) return e;
   mean_kernel<<<1, 256, 0, st>>>(row_loss, B, loss);
-  note_launch(2);
+  note_launch(3);
   return cudaGetLastError();
 }
 

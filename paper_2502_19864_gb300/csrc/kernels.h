@@ -111,8 +111,13 @@ cudaError_t attention_bwd_mma(const AttnArgs& a, cudaStream_t st);
 // tcgen05 forward (bf16, head_dim 64, no mask or RoPE, S <= 256)
 bool attention_tc_ok(const AttnArgs& a);
 cudaError_t attention_fwd_tc(const AttnArgs& a, cudaStream_t st);
-// tcgen05 backward for the same shapes; expects D = rowsum(dO * O) in a.Dscratch
+// tcgen05 kernels over 128-row blocks (bf16, head_dim 64 or 128, causal or not, q and k
+// plain or rotated in place): the backward (expects D = rowsum(dO * O) in a.Dscratch and the
+// forward's lse) and the forward of sequences longer than one block
+bool attention_bwd_tc_ok(const AttnArgs& a);
 cudaError_t attention_bwd_tc(const AttnArgs& a, cudaStream_t st);
+bool attention_fwd_blocks_tc_ok(const AttnArgs& a);
+cudaError_t attention_fwd_blocks_tc(const AttnArgs& a, cudaStream_t st);
 
 // ---------------------------------------------------------------------------------------
 // Row-wise fused kernels

@@ -111,6 +111,9 @@ struct ra_ctx {
   struct PrefixState { bool valid; int k, B, S; };
   PrefixState pf[2]{};
 
+  // measurement: the GEMM launches of a step, recorded to be replayed back to back
+  bool gemm_logging = false;
+  std::vector<GemmArgs> gemm_log;
   // profiling: event pairs around kernel calls
   bool profiling = false;
   struct Rec { int cat; double flops, bytes; cudaEvent_t a, b; };
@@ -594,6 +597,7 @@ cudaError_t P_gemm(ra_ctx* c, const GemmArgs& g, cudaStream_t st) {
   double aux = g.aux ? M * (g.epi == EPI_DSWIGLU ? 2 * N : N) * esz(g.aux_dtype) : 0;
   if (g.epi == EPI_DSWIGLU) out = 2 * M * N * esz(g.c_dtype);
   double bytes = (M * K + N * K) * esz(g.in_dtype) + out + aux;
+  if (c->gemm_logging) c->gemm_log.push_back(g);
   return prof(c, RA_PROF_GEMM, 2 * M * N * K, bytes, st, [&] { return gemm(g, st); });
 }
 
@@ -1398,6 +1402,29 @@ ra_status ra_profile_records(ra_ctx* ctx, ra_profile_record* out, int32_t max, i
 }
 
 int64_t ra_kernel_launches(void) { return (int64_t)launches_so_far(); }
+
+ra_status ra_profile_gemm_log(ra_ctx* ctx, int32_t on) {
+  if (!ctx) return RA_ERR_ARG;
+  ctx->gemm_logging = on != 0;
+  if (on) ctx->gemm_log.clear();
+  return RA_OK;
+}
+
+ra_status ra_profile_gemm_replay(ra_ctx* ctx, int32_t* n_launches, double* flops, ra_stream_t stream) {
+  if (!ctx) return RA_ERR_ARG;
+  if (!ctx->W) return fail(ctx, RA_ERR_STATE, "ra_bind_memory first");
+  CU(cudaSetDevice(ctx->device));
+  double fl = 0.0;
+  for (const GemmArgs& g : ctx->gemm_log) {
+    CU(gemm(g, (cudaStream_t)stream));
+    fl += 2.0 * g.M * g.N * g.K;
+  }
+  if (n_launches) *n_launches = (int32_t)ctx->gemm_log.size();
+  if (flops) *flops = fl;
+  ctx->k_fwd = ctx->k_bwd = -1;  // the replay overwrote the saved activations
+  ctx->bwd_since_update = false;
+  return RA_OK;
+}
 
 // ---- stand-alone kernels -----------------------------------------------------------------
 ra_status ra_gemm_bf16(const void* A_dev, const void* B_dev, void* C_dev, int32_t M, int32_t N,

@@ -140,5 +140,26 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
 }
 
 
+// byte offset of 16-byte chunk j of row r in a 128-byte-row, 128-byte-swizzled tile
+__device__ __forceinline__ uint32_t swz(int r, int j) { return (uint32_t)(r * 128 + ((j ^ (r & 7)) << 4)); }
+
+// Descriptor of a [rows x 64] 128-byte-swizzled block read as an MN-major operand: the
+// product's K runs along the block's rows and its N (or M) = 64 along the 128-byte rows, a
+// single swizzle atom wide.  Eight-row K groups are 1024 bytes apart; the leading and stride
+// byte offsets are both set to 1024, which is the K-group stride and leaves no second atom
+// along N to address.  A K step of 16 rows advances the start address by 2048 bytes.
+__device__ __forceinline__ uint64_t sdesc_mn_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)(1024 >> 4) << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Instruction descriptor of kind::f16 with B read MN-major (bit 16)
+__host__ __device__ constexpr uint32_t idesc_bf16_bmn(int M, int N) { return idesc_bf16(M, N) | (1u << 16); }
+
 }  // namespace tc
 }  // namespace ra
