@@ -305,6 +305,18 @@ ra_status ra_profile_records(ra_ctx* ctx, ra_profile_record* out, int32_t max, i
 /* Kernels this library has launched in this process so far (every entry point). */
 int64_t ra_kernel_launches(void);
 
+/* GEMM timing without per-kernel events (measurement support, no counterpart in the paper).
+ * With ra_profile_gemm_log(ctx, 1) every GEMM launch of the following calls (forward,
+ * backward) is also recorded: shapes, operands, epilogue and buffers.  ra_profile_gemm_replay
+ * enqueues the recorded launches again, in order, back to back on stream (capturable in a
+ * CUDA graph), and returns their count and algorithmic flops (2 M N K summed).  Timing that
+ * replay gives the GEMM kernels' duration with the launch overlap they have in the step,
+ * which an event pair around each kernel removes.  The replay overwrites the step's
+ * activations: the next backward needs a new ra_forward (ra_backward_truncated returns
+ * RA_ERR_STATE until then). */
+ra_status ra_profile_gemm_log(ra_ctx* ctx, int32_t on);
+ra_status ra_profile_gemm_replay(ra_ctx* ctx, int32_t* n_launches, double* flops, ra_stream_t stream);
+
 /* ---------------------------------------------------------------------------------------
  * Stand-alone kernels, for testing each piece of the step in isolation.  No context.
  * ------------------------------------------------------------------------------------- */

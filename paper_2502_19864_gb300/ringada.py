@@ -136,6 +136,9 @@ _SIGS = {
     "ra_profile_enable": (C.c_int, [C.c_void_p, C.c_int32]),
     "ra_profile_read": (C.c_int, [C.c_void_p, C.c_void_p]),
     "ra_kernel_launches": (C.c_int64, []),
+    "ra_profile_gemm_log": (C.c_int, [C.c_void_p, C.c_int32]),
+    "ra_profile_gemm_replay": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32), C.POINTER(C.c_double),
+                                         C.c_void_p]),
     "ra_profile_records": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_int32)]),
 }
 
@@ -330,6 +333,17 @@ def ra_profile_records(ctx, max_records=4096):
     n = C.c_int32()
     _check(lib().ra_profile_records(ctx, arr, max_records, C.byref(n)), ctx)
     return [(PROF_CATS[r.cat], r.ms, r.flops, r.bytes) for r in arr[:min(n.value, max_records)]]
+
+
+def ra_profile_gemm_log(ctx, on: bool):
+    _check(lib().ra_profile_gemm_log(ctx, 1 if on else 0), ctx)
+
+
+def ra_profile_gemm_replay(ctx, stream=None):
+    """Re-launches the recorded GEMMs back to back; returns (launches, flops)."""
+    n, fl = C.c_int32(), C.c_double()
+    _check(lib().ra_profile_gemm_replay(ctx, C.byref(n), C.byref(fl), _stream_ptr(stream)), ctx)
+    return n.value, fl.value
 
 
 def ra_kernel_launches() -> int:
