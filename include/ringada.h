@@ -337,11 +337,13 @@ ra_status ra_gemm_bf16(const void* A_dev, const void* B_dev, void* C_dev, int32_
  *   RA_EPI_BIAS_GELU_G u = acc + bias: C = GELU'(u) (nullable), C2 = GELU(u) (bf16)
  *   RA_EPI_MUL         C = acc * aux                     (aux bf16 [M, N], C c_dtype)
  *   RA_EPI_RESID       C = acc + aux                     (aux f32 [M, N], C f32)
- * Outputs are [M, N] row-major with leading dimension N.  bias: nullable f32 [N].  Device
+ * Outputs are [M, N] row-major with leading dimension N.  bias: nullable f32 [N].  With
+ * RA_EPI_B_KN or-ed into epi, B is given as stored [K, N] (N contiguous, leading dimension N),
+ * the layout of a forward weight [out, in] that the backward's dX GEMMs multiply by.  Device
  * pointers, 16-byte aligned; N and K multiples of 8.  Enqueued on stream.  RA_ERR_SHAPE
  * for a combination the kernel does not take, RA_ERR_UNSUPPORTED without sm_103. */
 enum { RA_EPI_STORE = 0, RA_EPI_BIAS_GELU = 1, RA_EPI_MUL = 2, RA_EPI_RESID = 3,
-       RA_EPI_BIAS_GELU_G = 6 };
+       RA_EPI_BIAS_GELU_G = 6, RA_EPI_B_KN = 0x100 };
 ra_status ra_gemm_bf16_epi(const void* A_dev, const void* B_dev, int32_t M, int32_t N, int32_t K,
                            int32_t epi, const float* bias_dev, const void* aux_dev, void* C_dev,
                            int32_t c_dtype, void* C2_dev, ra_stream_t stream);

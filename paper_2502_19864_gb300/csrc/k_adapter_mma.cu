@@ -436,7 +436,7 @@ struct BwdArgs {
   const float* z;     // [T, m]
   const bf16* Wu;     // [m, H]
   const bf16* Wd;     // [H, m]
-  float* dz;          // [T, m]
+  float* dz;          // [T, m] f32 of scratch, used as [T, m] bf16 GELU(z) then [T, m] bf16 dz
   void* dh;           // [T, H] or null: bf16, or f32 when DH_F32
 };
 
@@ -459,16 +459,25 @@ __global__ void RA_ROWS_BOUNDS(SZ) adapter_bwd_rows_mma_kernel(BwdArgs p) {
   __syncthreads();
   if (warp < W1) phase1_store<MB>(Gs, ldg, p.Wu, H, warp * KS, KS, part + (size_t)warp * R * (MB + 8), lane);
   __syncthreads();
+  // the weight-gradient kernel reads GELU(z) and dz as the bf16 operands it multiplies: both
+  // leave here rounded once, in the dz buffer ([T][m] GELU(z), then [T][m] dz)
+  bf16* sz = reinterpret_cast<bf16*>(p.dz);
+  bf16* dzb = sz + (size_t)p.T * MB;
   for (int e = threadIdx.x; e < R * MB; e += blockDim.x) {
     const int r = e / MB, j = e % MB;
     float ds = 0.f;
     for (int w = 0; w < W1; ++w) ds += part[((size_t)w * R + r) * (MB + 8) + j];
     float dz = 0.f;
+    const bf16 d16 = __float2bfloat16_rn(0.f);
+    bf16 dzr = d16;
     if (t0 + r < p.T) {
-      dz = ds * gelu_grad_f(p.z[(size_t)(t0 + r) * MB + j]);
-      p.dz[(size_t)(t0 + r) * MB + j] = dz;
+      const float zz = p.z[(size_t)(t0 + r) * MB + j];
+      dz = ds * gelu_grad_f(zz);
+      dzr = __float2bfloat16_rn(dz);
+      sz[(size_t)(t0 + r) * MB + j] = __float2bfloat16_rn(gelu_f(zz));
+      dzb[(size_t)(t0 + r) * MB + j] = dzr;
     }
-    Ds[r * lds + j] = __float2bfloat16_rn(dz);
+    Ds[r * lds + j] = dzr;
   }
   if (!p.dh) return;
   __syncthreads();
@@ -517,8 +526,8 @@ struct DwArgs {
   int T, H, m, chunk;
   const float* g;
   const bf16* h;
-  const float* z;
-  const float* dz;
+  const bf16* s;    // GELU(z) [T, m], bf16
+  const bf16* dz;   // dz [T, m], bf16
   float* partials;
 };
 
@@ -550,19 +559,19 @@ __global__ void __launch_bounds__(256) adapter_dw_mma_kernel(DwArgs p) {
       for (int i = 0; i < 4; ++i) acc[a][nt][i] = 0.f;
   const bf16* X = which ? Dsm : Ssm;
   const bf16* Y = which ? Hsm : Gsm;
-  // each thread's share of one 32-row tile: (z, dz) pairs and (g, h) quads
+  // each thread's share of one 32-row tile: (GELU(z), dz) pairs and (g, h) quads
   constexpr int NZ = DWR * (MB / 2) / 256, NG = DWR * (DWC / 4) / 256;
-  float2 zr[NZ], dr[NZ];
+  uint32_t zr[NZ], dr[NZ];
   float4 gr[NG];
   uint2 hr[NG];
   auto fetch = [&](int r0) {
 #pragma unroll
     for (int q = 0; q < NZ; ++q) {
       const int e = threadIdx.x + q * 256, r = e / (MB / 2), j = (e % (MB / 2)) * 2, tt = r0 + r;
-      zr[q] = dr[q] = make_float2(0.f, 0.f);
+      zr[q] = dr[q] = 0u;
       if (tt < te) {
-        zr[q] = *reinterpret_cast<const float2*>(p.z + (size_t)tt * MB + j);
-        dr[q] = *reinterpret_cast<const float2*>(p.dz + (size_t)tt * MB + j);
+        zr[q] = *reinterpret_cast<const uint32_t*>(p.s + (size_t)tt * MB + j);
+        dr[q] = *reinterpret_cast<const uint32_t*>(p.dz + (size_t)tt * MB + j);
       }
     }
 #pragma unroll
@@ -582,8 +591,8 @@ __global__ void __launch_bounds__(256) adapter_dw_mma_kernel(DwArgs p) {
 #pragma unroll
     for (int q = 0; q < NZ; ++q) {
       const int e = threadIdx.x + q * 256, r = e / (MB / 2), j = (e % (MB / 2)) * 2;
-      *reinterpret_cast<uint32_t*>(Ssm + r * LDJ + j) = pack2(gelu_f(zr[q].x), gelu_f(zr[q].y));
-      *reinterpret_cast<uint32_t*>(Dsm + r * LDJ + j) = pack2(dr[q].x, dr[q].y);
+      *reinterpret_cast<uint32_t*>(Ssm + r * LDJ + j) = zr[q];
+      *reinterpret_cast<uint32_t*>(Dsm + r * LDJ + j) = dr[q];
     }
 #pragma unroll
     for (int q = 0; q < NG; ++q) {
@@ -734,7 +743,9 @@ cudaError_t adapter_bwd_mma(const AdapterBwdArgs& a, const void* Wu_b, const voi
   // weight-gradient partials on the tensor cores, then the fixed-order sum
   DwArgs d;
   d.T = a.T; d.H = a.H; d.m = a.m; d.g = a.g; d.h = reinterpret_cast<const bf16*>(a.h);
-  d.z = a.z; d.dz = a.dz; d.partials = a.partials;
+  d.s = reinterpret_cast<const bf16*>(a.dz);
+  d.dz = d.s + (size_t)a.T * a.m;
+  d.partials = a.partials;
   const int nchunk = adapter_dw_chunks(a.T, a.H);
   d.chunk = (a.T + nchunk - 1) / nchunk;
   dim3 grid(a.H / DWC, nchunk);

@@ -82,9 +82,15 @@ __global__ void __launch_bounds__(NT) gemm_simt_kernel(GemmArgs g) {
     for (int r = 0; r < 4; ++r) {
       int e = tid + r * NT;
       int row = e >> 4, kk = e & 15;
-      int gm = m0 + row, gn = n0 + row, gk = k0 + kk;
+      int gm = m0 + row, gk = k0 + kk;
       As[kk][row] = (gm < g.M && gk < g.K) ? to_f(A[(int64_t)gm * g.lda + gk]) : 0.f;
-      Bs[kk][row] = (gn < g.N && gk < g.K) ? to_f(B[(int64_t)gn * g.ldb + gk]) : 0.f;
+      if (g.b_kn) {  // B stored [K, N]: n fastest for coalescing
+        int n = e & 63, k = e >> 6, gn = n0 + n, gk2 = k0 + k;
+        Bs[k][n] = (gn < g.N && gk2 < g.K) ? to_f(B[(int64_t)gk2 * g.ldb + gn]) : 0.f;
+      } else {
+        int gn = n0 + row;
+        Bs[kk][row] = (gn < g.N && gk < g.K) ? to_f(B[(int64_t)gn * g.ldb + gk]) : 0.f;
+      }
     }
     __syncthreads();
 #pragma unroll

@@ -75,6 +75,7 @@ struct TileCfg {
 
 struct TcParams {
   int M, N, K;
+  int b_kn;  // B stored [K, N]: BN / 64 TMA boxes of 64 x 64 per stage, read MN-major
   int n_tiles_n, m_tiles, num_tiles, k_blocks;
   int epi;
   void* C; int ldc; int c_dtype;
@@ -397,7 +398,14 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
           mbar_expect_tx(&full_bar[stage], Cfg::STAGE_BYTES);
           const uint32_t sa = smem_base + stage * Cfg::STAGE_BYTES;
           tma_load_2d(&tmA, sa, &full_bar[stage], kb * BK, m0);
-          tma_load_2d(&tmB, sa + Cfg::A_BYTES, &full_bar[stage], kb * BK, n0);
+          if (p.b_kn) {
+            // rows kb*BK.. of B [K, N]: one 64-column swizzle atom (8 KB) per 64 columns
+#pragma unroll
+            for (int a = 0; a < BN / 64; ++a)
+              tma_load_2d(&tmB, sa + Cfg::A_BYTES + a * 8192, &full_bar[stage], n0 + 64 * a, kb * BK);
+          } else {
+            tma_load_2d(&tmB, sa + Cfg::A_BYTES, &full_bar[stage], kb * BK, n0);
+          }
           pending_phase[stage] = (int)phase;
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
@@ -411,7 +419,7 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16(BM, BN);
+      const uint32_t idesc = p.b_kn ? idesc_bf16_bmn(BM, BN) : idesc_bf16(BM, BN);
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
@@ -425,10 +433,14 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
           if (!mbar_wait(&full_bar[stage], phase, &abort_sh, p.err)) { ok = false; break; }
           tc_fence_after();
           const uint32_t sa = smem_base + stage * Cfg::STAGE_BYTES;
-          const uint64_t adesc = sdesc_sw128(sa), bdesc = sdesc_sw128(sa + Cfg::A_BYTES);
+          const uint64_t adesc = sdesc_sw128(sa);
+          // K-major B: advance 16 elements = 32 bytes inside the swizzle atom; [K, N] B
+          // (MN-major): advance 16 rows = 2048 bytes, atoms along N 8 KB apart
+          const uint64_t bdesc = p.b_kn ? sdesc_mn_sw128_lbo(sa + Cfg::A_BYTES, 8192) : sdesc_sw128(sa + Cfg::A_BYTES);
+          const uint64_t bstep = p.b_kn ? 128u : 2u;
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)  // advance 16 elements = 32 bytes inside the swizzle atom
-            umma_bf16(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k), idesc,
+          for (int k = 0; k < BK / 16; ++k)
+            umma_bf16(d_tmem, adesc + (uint64_t)(2 * k), bdesc + bstep * (uint64_t)k, idesc,
                       (kb | k) != 0);
           umma_commit(&empty_bar[stage]);
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -837,7 +849,11 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   memset(&mc2, 0, sizeof mc2);
   memset(&mx, 0, sizeof mx);
   if (!make_map(&ma, g.A, g.M, g.K, g.lda, 64, BM, DT_BF16)) return cudaErrorNotSupported;
-  if (!make_map(&mb, g.B, g.N, g.K, g.ldb, 64, BNsel, DT_BF16)) return cudaErrorNotSupported;
+  if (g.b_kn) {
+    if (!make_map(&mb, g.B, g.K, g.N, g.ldb, 64, BK, DT_BF16)) return cudaErrorNotSupported;
+  } else if (!make_map(&mb, g.B, g.N, g.K, g.ldb, 64, BNsel, DT_BF16)) {
+    return cudaErrorNotSupported;
+  }
   // output maps: C is [M, N] except the packed d(gate|up) output of the SwiGLU' epilogue,
   // [M, 2N]; C2 is [M, N] (bias+GELU) or [M, N / 2] (h of the SwiGLU epilogue)
   if (has_c) {
@@ -861,6 +877,7 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   }
   TcParams p;
   p.M = g.M; p.N = g.N; p.K = g.K;
+  p.b_kn = g.b_kn ? 1 : 0;
   p.n_tiles_n = (g.N + BNsel - 1) / BNsel;
   p.m_tiles = m_tiles;
   p.num_tiles = m_tiles * p.n_tiles_n;

@@ -53,7 +53,11 @@ enum EpiKind : int {
 
 struct GemmArgs {
   const void* A = nullptr; int lda = 0;
+  // B is [N, K] (K contiguous) by default; with b_kn it is read as stored [K, N] (N
+  // contiguous, ldb = its row stride): the dX GEMMs multiply by a forward weight [out, in]
+  // without a transposed copy
   const void* B = nullptr; int ldb = 0;
+  bool b_kn = false;
   int M = 0, N = 0, K = 0;
   int in_dtype = DT_F32;
   int epi = EPI_STORE;

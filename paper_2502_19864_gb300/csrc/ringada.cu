@@ -40,7 +40,7 @@ struct Carve {
 };
 
 struct LayerWOff {  // offsets into the weights region
-  size_t Wqkv, WqkvT, bqkv, Wo, WoT, bo, W1, W1T, b1, W2, W2T, b2, g1, be1, g2, be2;
+  size_t Wqkv, bqkv, Wo, bo, W1, b1, W2, b2, g1, be1, g2, be2;
 };
 typedef uint16_t bf16_t;  // storage of the bf16 adapter shadows (host side never reads them)
 
@@ -67,7 +67,7 @@ struct ra_ctx {
   // region sizes and layouts
   size_t w_bytes = 0, t_bytes = 0, ws_bytes = 0;
   std::vector<LayerWOff> lw;
-  size_t head_W = 0, head_WT = 0, head_rmsf = 0;  // decoder frozen head (weights region)
+  size_t head_W = 0, head_rmsf = 0;  // decoder frozen head (weights region)
   // trainable region
   size_t n_train = 0;       // floats in P (= G = M = V)
   size_t n_head = 0;        // encoder head floats at the end of P
@@ -224,17 +224,13 @@ void plan(ra_ctx* c) {
   for (size_t l = 0; l < L; ++l) {
     LayerWOff& o = c->lw[l];
     o.Wqkv = w.take(3 * H * H * es);
-    o.WqkvT = w.take(3 * H * H * es);
     o.bqkv = c->dec ? 0 : w.take(3 * H * 4);
     o.Wo = w.take(H * H * es);
-    o.WoT = w.take(H * H * es);
     o.bo = c->dec ? 0 : w.take(H * 4);
     size_t f1 = c->dec ? 2 * F : F;  // decoder: packed gate|up
     o.W1 = w.take(f1 * H * es);
-    o.W1T = w.take(f1 * H * es);
     o.b1 = c->dec ? 0 : w.take(F * 4);
     o.W2 = w.take(H * F * es);
-    o.W2T = w.take(H * F * es);
     o.b2 = c->dec ? 0 : w.take(H * 4);
     o.g1 = w.take(H * 4);
     o.be1 = c->dec ? 0 : w.take(H * 4);
@@ -243,7 +239,6 @@ void plan(ra_ctx* c) {
   }
   if (c->dec) {
     c->head_W = w.take((size_t)c->C * H * es);
-    c->head_WT = w.take((size_t)c->C * H * es);
     c->head_rmsf = w.take(H * 4);
   }
   c->w_bytes = w.off;
@@ -489,7 +484,6 @@ ra_status ra_set_weights(ra_ctx* ctx, const ra_tensor_desc* list, int32_t n, ra_
         CU(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, st));
       } else if (d.param == RA_P_HEAD_W) {
         CU(convert_f32(src, ctx->w(ctx->head_W), act, d.numel, st));
-        CU(transpose_f32(src, ctx->w(ctx->head_WT), act, ctx->C, H, ctx->C, st));
       } else {
         CU(cudaMemcpyAsync(ctx->w(ctx->head_rmsf), src, bytes, cudaMemcpyDeviceToDevice, st));
       }
@@ -505,29 +499,23 @@ ra_status ra_set_weights(ra_ctx* ctx, const ra_tensor_desc* list, int32_t n, ra_
         } break;
         case RA_P_WQKV:
           CU(convert_f32(src, ctx->w(o.Wqkv), act, d.numel, st));
-          CU(transpose_f32(src, ctx->w(o.WqkvT), act, 3 * H, H, 3 * H, st));
           break;
         case RA_P_WQ: case RA_P_WK: case RA_P_WV: {
           int part = d.param - RA_P_WQ;
           CU(convert_f32(src, ctx->w<char>(o.Wqkv) + (size_t)part * H * H * es, act, d.numel, st));
-          CU(transpose_f32(src, ctx->w<char>(o.WqkvT) + (size_t)part * H * es, act, H, H, 3 * H, st));
         } break;
         case RA_P_WO:
           CU(convert_f32(src, ctx->w(o.Wo), act, d.numel, st));
-          CU(transpose_f32(src, ctx->w(o.WoT), act, H, H, H, st));
           break;
         case RA_P_W1:
           CU(convert_f32(src, ctx->w(o.W1), act, d.numel, st));
-          CU(transpose_f32(src, ctx->w(o.W1T), act, F, H, F, st));
           break;
         case RA_P_WG: case RA_P_WU: {
           int part = d.param == RA_P_WU;
           CU(pack_rows(src, ctx->w(o.W1), act, F, H, part, false, st));
-          CU(pack_rows(src, ctx->w(o.W1T), act, F, H, part, true, st));
         } break;
         case RA_P_W2: case RA_P_WD:
           CU(convert_f32(src, ctx->w(o.W2), act, d.numel, st));
-          CU(transpose_f32(src, ctx->w(o.W2T), act, H, F, H, st));
           break;
         case RA_P_BQKV: CU(cudaMemcpyAsync(ctx->w(o.bqkv), src, bytes, cudaMemcpyDeviceToDevice, st)); break;
         case RA_P_BO: CU(cudaMemcpyAsync(ctx->w(o.bo), src, bytes, cudaMemcpyDeviceToDevice, st)); break;
@@ -653,6 +641,15 @@ GemmArgs gemm_args(const ra_ctx* c, const void* A, int lda, const void* B, int l
 // their saved set, layers < k keep nothing).  Scratch comes from the set fs; the block
 // outputs ping-pong through fs.X, except that the last block writes last_out when given.
 // *y_out receives the last block's output.
+// dX GEMMs: C[M, N] = A[M, K] W[K, N] with the forward weight W [out = K, in = N] read as
+// stored (row stride ldw), no transposed copy
+GemmArgs gemm_kn(const ra_ctx* c, const void* A, int lda, const void* W, int ldw, int M, int N,
+                 int K) {
+  GemmArgs g = gemm_args(c, A, lda, W, ldw, M, N, K);
+  g.b_kn = true;
+  return g;
+}
+
 ra_status encoder_blocks(ra_ctx* ctx, const void* x, int B, int S, int l0, int l1, int k,
                          const ra_ctx::FwdScratch& fs, void* last_out, const void** y_out,
                          cudaStream_t st) {
@@ -1008,7 +1005,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
     }));
   } else {
     float* dn = ctx->ws<float>(ctx->b_ds2);
-    GemmArgs g = gemm_args(ctx, ctx->ws(ctx->h_logits), ctx->C, ctx->w(ctx->head_WT), ctx->C, T,
+    GemmArgs g = gemm_kn(ctx, ctx->ws(ctx->h_logits), ctx->C, ctx->w(ctx->head_W), H, T,
                            H, ctx->C);
     g.C = dn; g.ldc = H; g.c_dtype = DT_F32;
     CU(P_gemm(ctx, g, st));
@@ -1048,12 +1045,12 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
         return layernorm_bwd(dy2, nullptr, sb + so.xhat2, (float*)(sb + so.rstd2), ctx->w<float>(o.g2), ds2,
                              T, H, act, st, ctx->ws(ctx->b_df));
       }));
-      GemmArgs g = gemm_args(ctx, ctx->ws(ctx->b_df), H, ctx->w(o.W2T), H, T, F, H);
+      GemmArgs g = gemm_kn(ctx, ctx->ws(ctx->b_df), H, ctx->w(o.W2), F, T, F, H);
       g.epi = EPI_MUL; g.C = ctx->ws(ctx->b_du); g.ldc = F; g.c_dtype = act;
       g.aux = sb + so.gp; g.ldaux = F; g.aux_dtype = act;
       CU(P_gemm(ctx, g, st));
       float* dy1 = ctx->ws<float>(ctx->b_dy1);
-      g = gemm_args(ctx, ctx->ws(ctx->b_du), F, ctx->w(o.W1T), F, T, H, F);
+      g = gemm_kn(ctx, ctx->ws(ctx->b_du), F, ctx->w(o.W1), H, T, H, F);
       g.C = dy1; g.ldc = H; g.c_dtype = DT_F32;
       CU(P_gemm(ctx, g, st));
       float* ds1 = ctx->ws<float>(ctx->b_ds1);
@@ -1061,7 +1058,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
         return layernorm_bwd(dy1, ds2, sb + so.xhat1, (float*)(sb + so.rstd1), ctx->w<float>(o.g1), ds1,
                              T, H, act, st, ctx->ws(ctx->b_da));
       }));
-      g = gemm_args(ctx, ctx->ws(ctx->b_da), H, ctx->w(o.WoT), H, T, H, H);
+      g = gemm_kn(ctx, ctx->ws(ctx->b_da), H, ctx->w(o.Wo), H, T, H, H);
       g.C = ctx->ws(ctx->b_dO); g.ldc = H; g.c_dtype = act;
       CU(P_gemm(ctx, g, st));
       AttnArgs at;
@@ -1072,7 +1069,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       CU(P_attn_bwd(ctx, at, st));
       // dX = ds1 + dqkv Wqkv, the residual joined in the GEMM's epilogue (the next layer's
       // adapter backward reads dX whole)
-      g = gemm_args(ctx, ctx->ws(ctx->b_dqkv), 3 * H, ctx->w(o.WqkvT), 3 * H, T, H, 3 * H);
+      g = gemm_kn(ctx, ctx->ws(ctx->b_dqkv), 3 * H, ctx->w(o.Wqkv), H, T, H, 3 * H);
       g.epi = EPI_RESID; g.C = dX; g.ldc = H; g.c_dtype = DT_F32;
       g.aux = ds1; g.ldaux = H; g.aux_dtype = DT_F32;
       CU(P_gemm(ctx, g, st));
@@ -1088,13 +1085,13 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       ab.dWd = Gl + (size_t)2 * H * m; ab.dWu = Gl + (size_t)3 * H * m;
       CU(P_adapter_bwd(ctx, ab, st));
       // du = (df W2) * GELU'(u), the factor saved by the forward's FFN-up epilogue
-      GemmArgs g = gemm_args(ctx, ctx->ws(ctx->b_df), H, ctx->w(o.W2T), H, T, F, H);
+      GemmArgs g = gemm_kn(ctx, ctx->ws(ctx->b_df), H, ctx->w(o.W2), F, T, F, H);
       g.epi = EPI_MUL; g.C = ctx->ws(ctx->b_du); g.ldc = F; g.c_dtype = act;
       g.aux = sb + so.gp; g.ldaux = F; g.aux_dtype = act;
       CU(P_gemm(ctx, g, st));
       // dy1 = ds2 + du W1: the GEMM writes du W1, the LayerNorm backward adds ds2
       float* dy1 = ctx->ws<float>(ctx->b_dy1);
-      g = gemm_args(ctx, ctx->ws(ctx->b_du), F, ctx->w(o.W1T), F, T, H, F);
+      g = gemm_kn(ctx, ctx->ws(ctx->b_du), F, ctx->w(o.W1), H, T, H, F);
       g.C = dy1; g.ldc = H; g.c_dtype = DT_F32;
       CU(P_gemm(ctx, g, st));
       float* ds1 = ctx->ws<float>(ctx->b_ds1);
@@ -1108,7 +1105,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       ab.dWd = Gl; ab.dWu = Gl + (size_t)H * m;
       CU(P_adapter_bwd(ctx, ab, st));
       if (lowest) break;
-      g = gemm_args(ctx, ctx->ws(ctx->b_da), H, ctx->w(o.WoT), H, T, H, H);
+      g = gemm_kn(ctx, ctx->ws(ctx->b_da), H, ctx->w(o.Wo), H, T, H, H);
       g.C = ctx->ws(ctx->b_dO); g.ldc = H; g.c_dtype = act;
       CU(P_gemm(ctx, g, st));
       AttnArgs at;
@@ -1119,7 +1116,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       CU(P_attn_bwd(ctx, at, st));
       // dX = ds1 + dqkv Wqkv: the GEMM writes dqkv Wqkv; the next layer's LayerNorm backward
       // adds ds1
-      g = gemm_args(ctx, ctx->ws(ctx->b_dqkv), 3 * H, ctx->w(o.WqkvT), 3 * H, T, H, 3 * H);
+      g = gemm_kn(ctx, ctx->ws(ctx->b_dqkv), 3 * H, ctx->w(o.Wqkv), H, T, H, 3 * H);
       g.C = dX; g.ldc = H; g.c_dtype = DT_F32;
       CU(P_gemm(ctx, g, st));
       dY2 = ds1;
@@ -1132,12 +1129,12 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       ab.dWd = Gl + (size_t)2 * H * m; ab.dWu = Gl + (size_t)3 * H * m;
       CU(P_adapter_bwd(ctx, ab, st));
       // d(gate), d(up) from d h = df Wd
-      GemmArgs g = gemm_args(ctx, ctx->ws(ctx->b_df), H, ctx->w(o.W2T), H, T, F, H);
+      GemmArgs g = gemm_kn(ctx, ctx->ws(ctx->b_df), H, ctx->w(o.W2), F, T, F, H);
       g.epi = EPI_DSWIGLU; g.C = ctx->ws(ctx->b_du); g.ldc = 2 * F; g.c_dtype = act;
       g.aux = sb + so.gu; g.ldaux = 2 * F; g.aux_dtype = act;
       CU(P_gemm(ctx, g, st));
       float* dn2 = ctx->ws<float>(ctx->b_ds2);
-      g = gemm_args(ctx, ctx->ws(ctx->b_du), 2 * F, ctx->w(o.W1T), 2 * F, T, H, 2 * F);
+      g = gemm_kn(ctx, ctx->ws(ctx->b_du), 2 * F, ctx->w(o.W1), H, T, H, 2 * F);
       g.C = dn2; g.ldc = H; g.c_dtype = DT_F32;
       CU(P_gemm(ctx, g, st));
       float* dx1 = ctx->ws<float>(ctx->b_dy1);
@@ -1150,7 +1147,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       ab.dWd = Gl; ab.dWu = Gl + (size_t)H * m;
       CU(P_adapter_bwd(ctx, ab, st));
       if (lowest) break;
-      g = gemm_args(ctx, ctx->ws(ctx->b_da), H, ctx->w(o.WoT), H, T, H, H);
+      g = gemm_kn(ctx, ctx->ws(ctx->b_da), H, ctx->w(o.Wo), H, T, H, H);
       g.C = ctx->ws(ctx->b_dO); g.ldc = H; g.c_dtype = act;
       CU(P_gemm(ctx, g, st));
       AttnArgs at;
@@ -1162,7 +1159,7 @@ ra_status ra_backward_truncated(ra_ctx* ctx, int32_t k, ra_stream_t stream) {
       at.dqkv = ctx->ws(ctx->b_dqkv); at.err = ctx->ws<unsigned>(ctx->ws_err);
       CU(P_attn_bwd(ctx, at, st));
       float* dn1 = ctx->ws<float>(ctx->b_ds1);
-      g = gemm_args(ctx, ctx->ws(ctx->b_dqkv), 3 * H, ctx->w(o.WqkvT), 3 * H, T, H, 3 * H);
+      g = gemm_kn(ctx, ctx->ws(ctx->b_dqkv), 3 * H, ctx->w(o.Wqkv), H, T, H, 3 * H);
       g.C = dn1; g.ldc = H; g.c_dtype = DT_F32;
       CU(P_gemm(ctx, g, st));
       CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * 16, st,
@@ -1448,8 +1445,11 @@ ra_status ra_gemm_bf16_epi(const void* A_dev, const void* B_dev, int32_t M, int3
   if (!A_dev || !B_dev || M < 0 || N <= 0 || K <= 0) return RA_ERR_ARG;
   if (c_dtype != RA_F32 && c_dtype != RA_BF16) return RA_ERR_ARG;
   if (K % 8 || N % 8) return RA_ERR_SHAPE;
+  const bool b_kn = (epi & RA_EPI_B_KN) != 0;
+  epi &= ~RA_EPI_B_KN;
   GemmArgs g;
-  g.A = A_dev; g.lda = K; g.B = B_dev; g.ldb = K; g.M = M; g.N = N; g.K = K;
+  g.A = A_dev; g.lda = K; g.B = B_dev; g.ldb = b_kn ? N : K; g.b_kn = b_kn;
+  g.M = M; g.N = N; g.K = K;
   g.in_dtype = DT_BF16;
   g.C = C_dev; g.ldc = N; g.c_dtype = c_dtype == RA_BF16 ? DT_BF16 : DT_F32;
   switch (epi) {

@@ -158,6 +158,19 @@ __device__ __forceinline__ uint64_t sdesc_mn_sw128(uint32_t saddr) {
   return d;
 }
 
+// The same MN-major form for an operand several 64-wide swizzle atoms wide along N (or M):
+// consecutive atoms lbo bytes apart (the leading byte offset), eight-row K groups 1024 bytes
+// apart (the stride byte offset)
+__device__ __forceinline__ uint64_t sdesc_mn_sw128_lbo(uint32_t saddr, uint32_t lbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
 // Instruction descriptor of kind::f16 with B read MN-major (bit 16)
 __host__ __device__ constexpr uint32_t idesc_bf16_bmn(int M, int N) { return idesc_bf16(M, N) | (1u << 16); }
 

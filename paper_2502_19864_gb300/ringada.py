@@ -288,6 +288,7 @@ def ra_gemm_bf16(A_ptr, B_ptr, C_ptr, M, N, K, bias_ptr=None, gelu_ptr=None, str
 
 
 RA_EPI_STORE, RA_EPI_BIAS_GELU, RA_EPI_MUL, RA_EPI_RESID, RA_EPI_BIAS_GELU_G = 0, 1, 2, 3, 6
+RA_EPI_B_KN = 0x100
 
 
 def ra_gemm_bf16_epi(A_ptr, B_ptr, M, N, K, epi, bias_ptr=None, aux_ptr=None, C_ptr=None,

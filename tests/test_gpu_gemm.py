@@ -158,3 +158,32 @@ def test_gemm_f32_store_epilogue():
     ref = acc.cuda()
     assert not bool(C.isnan().any())
     assert (C - ref).abs().max().item() <= 1e-4 * ref.abs().max().item()
+
+
+# B given as stored [K, N] (a forward weight read by a dX GEMM, no transposed copy): tile
+# widths 256 (N 1024), 192 (N 768 at 4096 rows), 128 (N 128), ragged N and K, and a
+# multiply epilogue
+@pytest.mark.parametrize("M,N,K,epi", [(8192, 1024, 4096, "store"), (4096, 768, 3072, "store"),
+                                       (256, 128, 192, "store"), (300, 264, 136, "store"),
+                                       (1000, 520, 72, "mul")])
+def test_gemm_b_given_as_k_by_n(M, N, K, epi):
+    import torch
+    A, _, _, g = _operands(M, N, K, 9)
+    Wkn = (torch.randn(K, N, generator=g) * 0.05).to(torch.bfloat16)
+    acc = A.float().cpu() @ Wkn.float()
+    aux = (torch.rand(M, N, generator=g) * 1.2).to(torch.bfloat16)
+    Wd, auxd = Wkn.cuda(), aux.cuda()
+    if epi == "mul":  # bf16 output, as the step's dH GEMM writes it
+        C = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda")
+        R.ra_gemm_bf16_epi(A.data_ptr(), Wd.data_ptr(), M, N, K, R.RA_EPI_MUL | R.RA_EPI_B_KN, None,
+                           auxd.data_ptr(), C.data_ptr(), R.RA_BF16)
+        torch.cuda.synchronize()
+        _check(C, (acc * aux.float()).cuda())
+        return
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    R.ra_gemm_bf16_epi(A.data_ptr(), Wd.data_ptr(), M, N, K, R.RA_EPI_STORE | R.RA_EPI_B_KN, None,
+                       None, C.data_ptr(), R.RA_F32)
+    torch.cuda.synchronize()
+    ref = acc.cuda()
+    assert not bool(C.isnan().any())
+    assert (C - ref).abs().max().item() <= 1e-4 * ref.abs().max().item()
