@@ -341,12 +341,21 @@ ra_status ra_gemm_bf16(const void* A_dev, const void* B_dev, void* C_dev, int32_
  * RA_EPI_B_KN or-ed into epi, B is given as stored [K, N] (N contiguous, leading dimension N),
  * the layout of a forward weight [out, in] that the backward's dX GEMMs multiply by.  Device
  * pointers, 16-byte aligned; N and K multiples of 8.  Enqueued on stream.  RA_ERR_SHAPE
- * for a combination the kernel does not take, RA_ERR_UNSUPPORTED without sm_103. */
+ * for a combination the kernel does not take, RA_ERR_UNSUPPORTED without sm_103.
+ * scratch_dev (nullable; 256-byte aligned, scratch_bytes >= ra_gemm_scratch_bytes(),
+ * caller-owned, zero-filled before its first use; every call leaves it zeroed): lets the
+ * STORE and GELU epilogues spread the k-blocks of a last, partial round of output tiles over
+ * all CTAs (stream-K), each such tile summed from its CTAs' fp32 partials in a fixed order,
+ * so results are deterministic.  Calls that may run at the same time need different
+ * scratch.  Without it every tile is accumulated by one CTA.  RA_ERR_ARG for a scratch
+ * that is too small or misaligned. */
 enum { RA_EPI_STORE = 0, RA_EPI_BIAS_GELU = 1, RA_EPI_MUL = 2, RA_EPI_RESID = 3,
        RA_EPI_BIAS_GELU_G = 6, RA_EPI_B_KN = 0x100 };
+size_t ra_gemm_scratch_bytes(void);
 ra_status ra_gemm_bf16_epi(const void* A_dev, const void* B_dev, int32_t M, int32_t N, int32_t K,
                            int32_t epi, const float* bias_dev, const void* aux_dev, void* C_dev,
-                           int32_t c_dtype, void* C2_dev, ra_stream_t stream);
+                           int32_t c_dtype, void* C2_dev, void* scratch_dev, size_t scratch_bytes,
+                           ra_stream_t stream);
 
 /* Adapter backward of Eq. 1 for T rows (the in-kernel weight-gradient reduction of the
  * step), float32 throughout.  g_dev [T, H] = dLoss/d(adapter output); h_dev [T, H] the

@@ -24,6 +24,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cstring>
 #include <mutex>
 #include <unordered_map>
@@ -52,6 +53,8 @@ struct EpiTraits {
   static constexpr int WARPS = (EPI == EPI_BIAS_GELU || EPI == EPI_BIAS_GELU_G) ? 12 : 8;
   static constexpr int THREADS = (2 + WARPS) * 32;
   static constexpr bool AUX = EPI == EPI_MUL || EPI == EPI_RESID || EPI == EPI_DSWIGLU;
+  // stream-K partial and finisher units (the plain store epilogue only)
+  static constexpr bool SK = EPI == EPI_STORE;
 };
 
 // Every epilogue stages through 4 KB per warp, which keeps the full operand ring.  AUX
@@ -75,7 +78,10 @@ struct TileCfg {
 
 struct TcParams {
   int M, N, K;
-  int b_kn;  // B stored [K, N]: BN / 64 TMA boxes of 64 x 64 per stage, read MN-major
+  // B stored [K, N], read MN-major: 1 = BN / 64 TMA boxes of 64 x 64 per stage; 2 = one
+  // box of a 3-D view (64 columns, K rows, N / 64 column blocks) that lands as the same
+  // BN / 64 swizzle atoms (N a multiple of 64)
+  int b_kn;
   int n_tiles_n, m_tiles, num_tiles, k_blocks;
   int epi;
   void* C; int ldc; int c_dtype;
@@ -83,6 +89,76 @@ struct TcParams {
   void* C2; int ldc2; int c2_dtype;
   const void* aux; int ldaux; int aux_dtype;
   unsigned* err;
+  // stream-K (sk_iters > 0): tiles [0, dp_tiles) go one per CTA and round; the k-blocks of
+  // the tiles after them, numbered tile by tile, are split evenly over CTAs 0 .. sk_ctas - 1
+  int dp_tiles, sk_ctas, sk_iters;
+  float* sk_ws;         // one partial accumulator slot (SK_SLOT_FLOATS) per CTA
+  unsigned* sk_flags;   // per (CTA, epilogue warp): 1 while that warp's partial is published
+};
+
+// A partial accumulator slot holds a whole 128 x 256 tile in fp32: for output column chunk
+// c (32 columns) and column group q (4 columns), the 128 rows' float4s are contiguous, so a
+// warp moves 512 consecutive bytes per access.
+constexpr int SK_SLOT_FLOATS = BM * 256;
+constexpr int SK_MAX_WARPS = 12;
+
+// One CTA's work as an ordered list of units (tile, k-blocks [kb0, kb1), kind):
+//   kind 0  a whole tile;
+//   kind 1  partial: the accumulator of k-blocks [kb0, kb1) of a stream-K tile goes to this
+//           CTA's slot; a CTA with a higher index finishes the tile;
+//   kind 2  finisher: the last k-blocks of a stream-K tile; the epilogue first adds the
+//           partials of the lower-indexed CTAs that did the tile's first k-blocks, in
+//           ascending CTA order (a fixed order: the result does not depend on timing).
+// Order within a CTA: the partial first, so that a finisher only ever waits for work its
+// source CTAs do before anything else (and sources have lower indexes, so they were
+// dispatched first); then the finisher, whose wait for the partials and whose reads of them
+// then overlap the main loops of the tiles that follow; then the whole stream-K tiles and
+// the data-parallel tiles.
+struct Sched {
+  int c, K, stride, dp_tiles, n_dp, n_p, n_mid, n_fin, t_first, t_last, b, e;
+  __device__ void init(const TcParams& p, int cta, int grid) {
+    c = cta; K = p.k_blocks; stride = grid; dp_tiles = p.dp_tiles;
+    n_dp = dp_tiles > c ? (dp_tiles - c + grid - 1) / grid : 0;
+    n_p = n_mid = n_fin = 0;
+    t_first = 0; t_last = -1; b = e = 0;
+    if (p.sk_iters > 0 && c < p.sk_ctas) {
+      b = (int)((long long)c * p.sk_iters / p.sk_ctas);
+      e = (int)((long long)(c + 1) * p.sk_iters / p.sk_ctas);
+      if (b < e) {
+        t_first = b / K;
+        t_last = (e - 1) / K;
+        n_fin = (b % K != 0 && (t_first + 1) * K <= e) ? 1 : 0;
+        n_p = e % K != 0 ? 1 : 0;
+        n_mid = t_last - t_first + 1 - n_p - n_fin;
+      }
+    }
+  }
+  __device__ int count() const { return n_p + n_dp + n_mid + n_fin; }
+  __device__ void unit(int u, int& tile, int& kb0, int& kb1, int& kind) const {
+    if (u < n_p) {
+      const int base = t_last * K;
+      tile = dp_tiles + t_last; kb0 = max(b, base) - base; kb1 = e - base; kind = 1;
+      return;
+    }
+    u -= n_p;
+    if (u < n_fin) {
+      tile = dp_tiles + t_first; kb0 = b - t_first * K; kb1 = K; kind = 2;
+      return;
+    }
+    u -= n_fin;
+    if (u < n_mid) {  // whole tiles
+      tile = dp_tiles + t_first + n_fin + u; kb0 = 0; kb1 = K; kind = 0;
+      return;
+    }
+    u -= n_mid;
+    tile = c + u * stride; kb0 = 0; kb1 = K; kind = 0;
+  }
+  // first CTA that holds k-blocks of stream-K tile t: the owner of its first iteration,
+  // the largest cc with floor(cc * I / G) <= t * K
+  __device__ static int first_source(const TcParams& p, int t) {
+    const long long i = (long long)t * p.k_blocks;
+    return (int)(((i + 1) * p.sk_ctas - 1) / p.sk_iters);
+  }
 };
 
 // ---- TMA and bulk-copy helpers ------------------------------------------------------------
@@ -92,6 +168,14 @@ __device__ __forceinline__ void tma_load_2d(const CUtensorMap* tm, uint32_t dst,
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_3d(const CUtensorMap* tm, uint32_t dst, uint64_t* bar,
+                                            int c0, int c1, int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar))
       : "memory");
 }
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, uint32_t src, int c0, int c1) {
@@ -202,6 +286,49 @@ __device__ __forceinline__ void store_chunk(const CUtensorMap* tm, uint8_t* stag
       bulk_commit();
     }
     ++slot_i;
+  }
+}
+
+// ---- stream-K partials ---------------------------------------------------------------------
+// This thread's row (TMEM lane) of tile rows 32 quad.., output chunk cidx (columns 32 cidx..):
+// float4 q of the row at ((cidx * 8 + q) * 128 + row) * 4.  L2 only (st.cg / ld.cg): the
+// slot is written and read within the launch, by different SMs.
+__device__ __forceinline__ void sk_put(float* slot, int cidx, int row, const float* v) {
+  float4* d = reinterpret_cast<float4*>(slot) + (size_t)cidx * 8 * BM + row;
+#pragma unroll
+  for (int q = 0; q < 8; ++q)
+    __stcg(d + q * BM, make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+}
+__device__ __forceinline__ void sk_add(const float* slot, int cidx, int row, float* v) {
+  const float4* s = reinterpret_cast<const float4*>(slot) + (size_t)cidx * 8 * BM + row;
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const float4 x = __ldcg(s + q * BM);
+    v[4 * q] += x.x; v[4 * q + 1] += x.y; v[4 * q + 2] += x.z; v[4 * q + 3] += x.w;
+  }
+}
+__device__ __forceinline__ void flag_release(unsigned* f) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(f), "r"(1u) : "memory");
+}
+__device__ __forceinline__ unsigned flag_acquire(const unsigned* f) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(f) : "memory");
+  return v;
+}
+// Bounded wait (global timer) for a published partial; false on expiry or abort.
+__device__ __noinline__ bool sk_wait(const unsigned* f, volatile int* abort_flag, unsigned* err) {
+  if (flag_acquire(f) != 0u) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (flag_acquire(f) != 0u) return true;
+    if ((it & 63) == 0) {
+      if (*abort_flag) return false;
+      if (global_ns() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        set_dev_error(err, RA_DEVERR_TIMEOUT);
+        return false;
+      }
+    }
   }
 }
 
@@ -380,6 +507,8 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
   // the set-up above overlaps the previous kernel's tail; operands are read only after it
   pdl_wait();
   pdl_trigger();
+  Sched sch;
+  sch.init(p, blockIdx.x, gridDim.x);
 
   if (warp == 0) {
     // ------------------------------------------------------------------ TMA producer
@@ -389,16 +518,20 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
       int pending_phase[STAGES];
       for (int s = 0; s < STAGES; ++s) pending_phase[s] = -1;
       bool ok = true;
-      for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+      for (int u = 0; ok && u < sch.count(); ++u) {
+        int tile, kb0, kb1, kind;
+        sch.unit(u, tile, kb0, kb1, kind);
         int mt, nt;
         tile_coords(tile, p.m_tiles, p.n_tiles_n, mt, nt);
         const int m0 = mt * BM, n0 = nt * BN;
-        for (int kb = 0; kb < p.k_blocks; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, &abort_sh, p.err)) { ok = false; break; }
           mbar_expect_tx(&full_bar[stage], Cfg::STAGE_BYTES);
           const uint32_t sa = smem_base + stage * Cfg::STAGE_BYTES;
           tma_load_2d(&tmA, sa, &full_bar[stage], kb * BK, m0);
-          if (p.b_kn) {
+          if (p.b_kn == 2) {
+            tma_load_3d(&tmB, sa + Cfg::A_BYTES, &full_bar[stage], 0, kb * BK, n0 / 64);
+          } else if (p.b_kn) {
             // rows kb*BK.. of B [K, N]: one 64-column swizzle atom (8 KB) per 64 columns
 #pragma unroll
             for (int a = 0; a < BN / 64; ++a)
@@ -425,11 +558,13 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+      for (int u = 0; ok && u < sch.count(); ++u) {
+        int tile, kb0, kb1, kind;
+        sch.unit(u, tile, kb0, kb1, kind);
         if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, &abort_sh, p.err)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
-        for (int kb = 0; kb < p.k_blocks; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&full_bar[stage], phase, &abort_sh, p.err)) { ok = false; break; }
           tc_fence_after();
           const uint32_t sa = smem_base + stage * Cfg::STAGE_BYTES;
@@ -441,7 +576,7 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             umma_bf16(d_tmem, adesc + (uint64_t)(2 * k), bdesc + bstep * (uint64_t)k, idesc,
-                      (kb | k) != 0);
+                      (kb != kb0 || k != 0) ? 1u : 0u);
           umma_commit(&empty_bar[stage]);
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
@@ -490,7 +625,10 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
       ++aux_i;
     };
     bool ok = true;
-    for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+    const int ew = warp - 2;
+    for (int u = 0; ok && u < sch.count(); ++u) {
+      int tile, kb0, kb1, kind;
+      sch.unit(u, tile, kb0, kb1, kind);
       int mt, nt;
       tile_coords(tile, p.m_tiles, p.n_tiles_n, mt, nt);
       const int m0 = mt * BM, n0 = nt * BN;
@@ -508,6 +646,16 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
       if (!mbar_wait(&tfull_bar[acc], acc_phase, &abort_sh, p.err)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
+      // finisher: the partials of CTAs src0 .. blockIdx.x - 1 (this warp's rows and columns)
+      // must be published before they are added
+      const int src0 = (EpiTraits<EPI>::SK && kind == 2) ? Sched::first_source(p, tile - p.dp_tiles) : 0;
+      if (EpiTraits<EPI>::SK && kind == 2) {
+        bool got = true;
+        if (lane == 0)
+          for (int cc = src0; got && cc < (int)blockIdx.x; ++cc)
+            got = sk_wait(p.sk_flags + cc * SK_MAX_WARPS + ew, &abort_sh, p.err);
+        if (!__shfl_sync(0xffffffffu, got ? 1 : 0, 0)) break;
+      }
       if (EPI == EPI_SWIGLU) {
         // per 128-column block: gate columns [0, 64), up columns [64, 128); the two warps of
         // a quadrant split each block's 64 gate columns
@@ -591,9 +739,18 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
           if (lane == 0) mbar_arrive(&tempty_bar[acc]);
         };
         auto chunk = [&](int c0, uint32_t* r) {
+          if (EpiTraits<EPI>::SK && kind == 1) {  // partial: the fp32 accumulator goes to this CTA's slot
+            sk_put(p.sk_ws + (size_t)blockIdx.x * SK_SLOT_FLOATS, c0 / 32, quad * 32 + lane,
+                   reinterpret_cast<const float*>(r));
+            return;
+          }
           // chunks entirely right of N or below M are skipped (warp-uniform); partial ones
           // are clipped by the tensor store
           if (n0 + c0 < p.N && row0 < p.M) {
+            if (EpiTraits<EPI>::SK && kind == 2)
+              for (int cc = src0; cc < (int)blockIdx.x; ++cc)
+                sk_add(p.sk_ws + (size_t)cc * SK_SLOT_FLOATS, c0 / 32, quad * 32 + lane,
+                       reinterpret_cast<float*>(r));
             EpiIn<EPI> in;
             // (N is a multiple of 8: a group of 8 that starts below N ends below it)
 #pragma unroll
@@ -628,6 +785,19 @@ __global__ void __launch_bounds__(EpiTraits<EPI>::THREADS, 1)
         }
       }
       if (EPI == EPI_STORE || EPI == EPI_BIAS_GELU || EPI == EPI_BIAS_GELU_G) {  // released above
+        if (EpiTraits<EPI>::SK && kind == 1) {
+          // publish this warp's part of the partial: every lane's stores are ordered before
+          // the flag by the fence and the warp barrier, the flag store releases them
+          __threadfence();
+          __syncwarp();
+          if (lane == 0) flag_release(p.sk_flags + blockIdx.x * SK_MAX_WARPS + ew);
+        } else if (EpiTraits<EPI>::SK && kind == 2) {
+          // the partials are consumed: clear their flags for the next launch (which reads
+          // them only after this grid has completed)
+          __syncwarp();
+          if (lane == 0)
+            for (int cc = src0; cc < (int)blockIdx.x; ++cc) p.sk_flags[cc * SK_MAX_WARPS + ew] = 0u;
+        }
         if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
         continue;
       }
@@ -695,18 +865,18 @@ EncodeTiledFn encode_fn() {
 struct MapKey {
   const void* ptr;
   int64_t rows, cols, ld;
-  int box_cols, box_rows, dtype;
+  int box_cols, box_rows, dtype, blocks;
   bool operator==(const MapKey& o) const {
     return ptr == o.ptr && rows == o.rows && cols == o.cols && ld == o.ld &&
-           box_cols == o.box_cols && box_rows == o.box_rows && dtype == o.dtype;
+           box_cols == o.box_cols && box_rows == o.box_rows && dtype == o.dtype && blocks == o.blocks;
   }
 };
 struct MapKeyHash {
   size_t operator()(const MapKey& k) const {
     size_t h = std::hash<const void*>()(k.ptr);
     h ^= std::hash<int64_t>()(k.rows * 1000003 + k.cols) + 0x9e3779b9 + (h << 6) + (h >> 2);
-    h ^= std::hash<int64_t>()(k.ld * 31 + k.box_rows * 7 + k.box_cols * 131 + k.dtype) + 0x9e3779b9 +
-         (h << 6) + (h >> 2);
+    h ^= std::hash<int64_t>()(k.ld * 31 + k.box_rows * 7 + k.box_cols * 131 + k.dtype + k.blocks * 1009) +
+         0x9e3779b9 + (h << 6) + (h >> 2);
     return h;
   }
 };
@@ -716,11 +886,14 @@ struct MapKeyHash {
 // MMA descriptors expect; output stores (32 bf16 or 16 f32 columns: 64-byte rows) and operand
 // loads of the epilogues (32 columns) use the swizzle whose span is one box row, matching
 // stage_row, stage_half and unstage_row.
+// blocks > 0: the matrix (cols a multiple of box_cols) seen in 3-D as (box_cols columns, rows,
+// cols / box_cols column blocks); one box of box_cols x box_rows x blocks then lands as
+// `blocks` consecutive box_cols x box_rows tiles (the MN-major B operand atoms).
 bool make_map(CUtensorMap* out, const void* ptr, int64_t rows, int64_t cols, int64_t ld,
-              int box_cols, int box_rows, int dtype) {
+              int box_cols, int box_rows, int dtype, int blocks = 0) {
   static std::mutex mu;
   static std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
-  MapKey key{ptr, rows, cols, ld, box_cols, box_rows, dtype};
+  MapKey key{ptr, rows, cols, ld, box_cols, box_rows, dtype, blocks};
   std::lock_guard<std::mutex> lock(mu);
   auto it = cache.find(key);
   if (it != cache.end()) {
@@ -734,12 +907,14 @@ bool make_map(CUtensorMap* out, const void* ptr, int64_t rows, int64_t cols, int
   CUtensorMapSwizzle sw = row_bytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
                         : row_bytes == 64  ? CU_TENSOR_MAP_SWIZZLE_64B
                                            : CU_TENSOR_MAP_SWIZZLE_NONE;
-  cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-  cuuint64_t gstride[1] = {(cuuint64_t)ld * es};
-  cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
-  cuuint32_t estride[2] = {1, 1};
+  const bool b3 = blocks > 0;
+  if (b3 && cols % box_cols) return false;
+  cuuint64_t gdim[3] = {(cuuint64_t)(b3 ? box_cols : cols), (cuuint64_t)rows, (cuuint64_t)(b3 ? cols / box_cols : 1)};
+  cuuint64_t gstride[2] = {(cuuint64_t)ld * es, (cuuint64_t)box_cols * es};
+  cuuint32_t box[3] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows, (cuuint32_t)(b3 ? blocks : 1)};
+  cuuint32_t estride[3] = {1, 1, 1};
   CUresult r = fn(out, dtype == DT_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
-                  2, const_cast<void*>(ptr), gdim, gstride, box, estride,
+                  b3 ? 3 : 2, const_cast<void*>(ptr), gdim, gstride, box, estride,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return false;
@@ -792,6 +967,9 @@ cudaError_t dispatch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorM
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 }  // namespace
+
+size_t gemm_sk_slot_bytes() { return (size_t)SK_SLOT_FLOATS * 4; }
+int gemm_sk_flags_per_slot() { return SK_MAX_WARPS; }
 
 cudaError_t selftest_wait(unsigned* err, uint64_t limit_ns, cudaStream_t st) {
   selftest_wait_kernel<<<1, 32, 0, st>>>(err, limit_ns);
@@ -849,11 +1027,12 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   memset(&mc2, 0, sizeof mc2);
   memset(&mx, 0, sizeof mx);
   if (!make_map(&ma, g.A, g.M, g.K, g.lda, 64, BM, DT_BF16)) return cudaErrorNotSupported;
-  if (g.b_kn) {
-    if (!make_map(&mb, g.B, g.K, g.N, g.ldb, 64, BK, DT_BF16)) return cudaErrorNotSupported;
-  } else if (!make_map(&mb, g.B, g.N, g.K, g.ldb, 64, BNsel, DT_BF16)) {
-    return cudaErrorNotSupported;
-  }
+  // stored [K, N] B: one 3-D box per stage where N is a multiple of 64 (and the driver takes
+  // the view), else BN / 64 boxes
+  int b_kn = !g.b_kn ? 0 : g.N % 64 == 0 ? 2 : 1;
+  if (b_kn == 2 && !make_map(&mb, g.B, g.K, g.N, g.ldb, 64, BK, DT_BF16, BNsel / 64)) b_kn = 1;
+  if (b_kn == 1 && !make_map(&mb, g.B, g.K, g.N, g.ldb, 64, BK, DT_BF16)) return cudaErrorNotSupported;
+  if (b_kn == 0 && !make_map(&mb, g.B, g.N, g.K, g.ldb, 64, BNsel, DT_BF16)) return cudaErrorNotSupported;
   // output maps: C is [M, N] except the packed d(gate|up) output of the SwiGLU' epilogue,
   // [M, 2N]; C2 is [M, N] (bias+GELU) or [M, N / 2] (h of the SwiGLU epilogue)
   if (has_c) {
@@ -877,7 +1056,7 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   }
   TcParams p;
   p.M = g.M; p.N = g.N; p.K = g.K;
-  p.b_kn = g.b_kn ? 1 : 0;
+  p.b_kn = b_kn;
   p.n_tiles_n = (g.N + BNsel - 1) / BNsel;
   p.m_tiles = m_tiles;
   p.num_tiles = m_tiles * p.n_tiles_n;
@@ -889,6 +1068,29 @@ cudaError_t gemm_tc(const GemmArgs& g, cudaStream_t st) {
   p.aux = g.aux; p.ldaux = g.ldaux; p.aux_dtype = g.aux_dtype;
   p.err = g.err;
   const int grid = p.num_tiles < sms ? p.num_tiles : sms;
+  // Stream-K for the last, partial round of tiles (e.g. 256 tiles on 152 SMs: 104 tiles
+  // would keep 104 SMs busy for a whole tile while 48 idle): their k-blocks are spread over
+  // the CTAs.  Only after at least one full round (a single round stays one tile per CTA),
+  // only where the round is not nearly full, only for the plain store epilogue, and only
+  // where each CTA's share is at least 24 k-blocks: writing and reading back a tile's fp32
+  // partials costs about as much as 8 to 12 k-blocks of MMA (measured on the BERT-large
+  // shapes: 8192 x 1024 with K = 3072 or 4096 gain 3 to 4 us a launch, K = 1024 loses 4 us).
+  p.dp_tiles = p.num_tiles;
+  p.sk_ctas = 0;
+  p.sk_iters = 0;
+  p.sk_ws = g.sk_ws;
+  p.sk_flags = g.sk_flags;
+  const bool sk_epi = g.epi == EPI_STORE;
+  if (sk_epi && g.sk_ws && g.sk_flags && grid <= g.sk_slots && p.num_tiles > grid) {
+    const int rem = p.num_tiles % grid;
+    const long long iters = (long long)rem * p.k_blocks;
+    const int ctas = (int)std::min<long long>(grid, iters / 8);
+    if (rem > 0 && rem * 100 < 85 * grid && ctas > rem && iters >= 24LL * ctas) {
+      p.dp_tiles = p.num_tiles - rem;
+      p.sk_ctas = ctas;
+      p.sk_iters = (int)iters;
+    }
+  }
   return BNsel == 256 ? dispatch<256>(ma, mb, mc, mc2, mx, p, grid, st)
        : BNsel == 192 ? dispatch<192>(ma, mb, mc, mc2, mx, p, grid, st)
                       : dispatch<128>(ma, mb, mc, mc2, mx, p, grid, st);

@@ -66,7 +66,17 @@ struct GemmArgs {
   void* C2 = nullptr; int ldc2 = 0; int c2_dtype = DT_F32;
   const void* aux = nullptr; int ldaux = 0; int aux_dtype = DT_F32;
   unsigned* err = nullptr;
+  // stream-K scratch of the tcgen05 path (nullable: then every tile is done by one CTA):
+  // sk_slots partial-accumulator slots of gemm_sk_slot_bytes() and sk_slots * 12 flags,
+  // zero before the first launch (every launch leaves them zero).  GEMMs that may run at the
+  // same time (different streams) need different scratch.
+  float* sk_ws = nullptr;
+  unsigned* sk_flags = nullptr;
+  int sk_slots = 0;
 };
+// bytes of one stream-K slot, flags per slot
+size_t gemm_sk_slot_bytes();
+int gemm_sk_flags_per_slot();
 
 // Returns a cudaError_t from the launch (cudaSuccess if enqueued).
 cudaError_t gemm(const GemmArgs& a, cudaStream_t st);

@@ -26,6 +26,8 @@ using namespace ra;
 namespace {
 
 constexpr size_t kAlign = 256;
+// stream-K slots per GEMM scratch set: at least the SM count (one CTA per SM)
+constexpr int kSkSlots = 160;
 constexpr unsigned RA_DEVERR_TIMEOUT_BIT = 1u;  // matches the device-side flag bits
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
@@ -76,6 +78,10 @@ struct ra_ctx {
   // workspace
   SlotOff so{};
   size_t ws_err = 0, ws_arena = 0;
+  // GEMM stream-K scratch (bf16 models): flags, then partial slots; set 1 serves the
+  // next-batch prefix, which may run on another stream at the same time as set 0
+  size_t ws_skf[2]{}, ws_sks[2]{};
+  size_t ws_zero_end = 256;  // bytes from the start of the workspace zeroed at binding
   size_t s_X[2]{}, s_qkv = 0, s_O = 0, s_a = 0, s_y1 = 0, s_h = 0, s_f = 0, s_u = 0, s_gu = 0;
   size_t s_n = 0;  // decoder normalised input of the next GEMM
   size_t s_rstd = 0;
@@ -104,7 +110,7 @@ struct ra_ctx {
   // next-batch prefix (ra_forward_prefix / ra_forward_suffix, encoders): a second set of
   // forward scratch buffers, so that the prefix of one batch can run on another stream while
   // the previous batch's suffix, backward and update run, and two buffers for its output
-  struct FwdScratch { size_t X[2], qkv, O, a, y1, h, f; };
+  struct FwdScratch { size_t X[2], qkv, O, a, y1, h, f; int sk; };
   FwdScratch fs[2]{};
   bool prefix_bufs = false;
   size_t pbuf[2]{};
@@ -302,6 +308,12 @@ void plan(ra_ctx* c) {
 
   Carve ws;
   c->ws_err = ws.take(256);
+  const bool sk = c->act == DT_BF16;
+  if (sk) {
+    for (int i = 0; i < 2; ++i) c->ws_skf[i] = ws.take((size_t)kSkSlots * gemm_sk_flags_per_slot() * 4);
+    c->ws_zero_end = ws.off;
+    for (int i = 0; i < 2; ++i) c->ws_sks[i] = ws.take((size_t)kSkSlots * gemm_sk_slot_bytes());
+  }
   c->ws_arena = ws.take((size_t)c->max_depth * s.slot_bytes);
   // forward scratch (layers below k)
   if (!c->dec) {
@@ -321,10 +333,11 @@ void plan(ra_ctx* c) {
   c->s_f = ws.take(T * H * es);
   c->s_u = c->dec ? 0 : ws.take(T * F * es);
   c->s_gu = c->dec ? ws.take(T * 2 * F * es) : 0;
-  c->fs[0] = {{c->s_X[0], c->s_X[1]}, c->s_qkv, c->s_O, c->s_a, c->s_y1, c->s_h, c->s_f};
+  c->fs[0] = {{c->s_X[0], c->s_X[1]}, c->s_qkv, c->s_O, c->s_a, c->s_y1, c->s_h, c->s_f, 0};
   c->prefix_bufs = !c->dec && c->cfg.prefix_buffers != 0;
   if (c->prefix_bufs) {
     ra_ctx::FwdScratch& f1 = c->fs[1];
+    f1.sk = 1;
     f1.X[0] = ws.take(T * H * es);
     f1.X[1] = ws.take(T * H * es);
     f1.qkv = ws.take(T * 3 * H * es);
@@ -449,7 +462,7 @@ ra_status ra_bind_memory(ra_ctx* ctx, void* weights_dev, size_t weights_bytes,
   ctx->Tr = (char*)trainable_dev;
   ctx->WS = (char*)workspace_dev;
   CU(cudaMemset(ctx->Tr, 0, ctx->t_bytes));
-  CU(cudaMemset(ctx->WS, 0, 256));
+  CU(cudaMemset(ctx->WS, 0, ctx->ws_zero_end));
   CU(cudaDeviceSynchronize());
   ctx->n_updates = 0;
   ctx->k_fwd = ctx->k_bwd = -1;
@@ -628,12 +641,18 @@ extern "C" {
 // ---- forward -----------------------------------------------------------------------------
 namespace {
 
+// sk: the stream-K scratch set (1 for GEMMs of the next-batch prefix, 0 otherwise)
 GemmArgs gemm_args(const ra_ctx* c, const void* A, int lda, const void* B, int ldb, int M, int N,
-                   int K) {
+                   int K, int sk = 0) {
   GemmArgs g;
   g.A = A; g.lda = lda; g.B = B; g.ldb = ldb; g.M = M; g.N = N; g.K = K;
   g.in_dtype = c->act;
   g.err = c->ws<unsigned>(c->ws_err);
+  if (c->act == DT_BF16) {
+    g.sk_ws = c->ws<float>(c->ws_sks[sk]);
+    g.sk_flags = c->ws<unsigned>(c->ws_skf[sk]);
+    g.sk_slots = kSkSlots;
+  }
   return g;
 }
 
@@ -678,7 +697,7 @@ ra_status encoder_blocks(ra_ctx* ctx, const void* x, int B, int S, int l0, int l
     void* xout = (last_out && l + 1 == l1) ? last_out : ctx->ws<char>(fs.X[out_idx]);
     const float* Pl = ctx->P() + (size_t)l * 4 * H * m;
 
-    GemmArgs g = gemm_args(ctx, xin, H, ctx->w(o.Wqkv), H, T, 3 * H, H);
+    GemmArgs g = gemm_args(ctx, xin, H, ctx->w(o.Wqkv), H, T, 3 * H, H, fs.sk);
     g.C = qkv; g.ldc = 3 * H; g.c_dtype = act; g.bias = ctx->w<float>(o.bqkv);
     CU(P_gemm(ctx, g, st));
     AttnArgs at;
@@ -690,21 +709,21 @@ ra_status encoder_blocks(ra_ctx* ctx, const void* x, int B, int S, int l0, int l
     if (ctx->post_ffn) {
       // Fig. 1 placement: y1 = LN1(x + a); y2 = LN2(y1 + f); out = y2 + GELU(y2 Wd) Wu
       void* a_s = ctx->ws<char>(fs.a);
-      g = gemm_args(ctx, O, H, ctx->w(o.Wo), H, T, H, H);
+      g = gemm_args(ctx, O, H, ctx->w(o.Wo), H, T, H, H, fs.sk);
       g.C = a_s; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.bo);
       CU(P_gemm(ctx, g, st));
       CU(prof(ctx, RA_PROF_NORM, 0, (double)T * H * ((full ? 4 : 3) * dtype_size(act)), st, [&] {
         return add_layernorm_fwd(xin, a_s, ctx->w<float>(o.g1), ctx->w<float>(o.be1), ctx->cfg.norm_eps,
                                  y1, full ? xhat1 : nullptr, full ? rstd1 : nullptr, T, H, act, st);
       }));
-      g = gemm_args(ctx, y1, H, ctx->w(o.W1), H, T, F, H);
+      g = gemm_args(ctx, y1, H, ctx->w(o.W1), H, T, F, H, fs.sk);
       // layers above k keep GELU'(u) for the FFN backward; layer k stops at its adapter
       g.epi = full ? EPI_BIAS_GELU_G : EPI_BIAS_GELU;
       g.C = full ? gp : nullptr; g.ldc = F; g.c_dtype = act; g.bias = ctx->w<float>(o.b1);
       g.C2 = hbuf; g.ldc2 = F; g.c2_dtype = act;
       CU(P_gemm(ctx, g, st));
       void* f_s = ctx->ws<char>(fs.f);
-      g = gemm_args(ctx, hbuf, F, ctx->w(o.W2), F, T, H, F);
+      g = gemm_args(ctx, hbuf, F, ctx->w(o.W2), F, T, H, F, fs.sk);
       g.C = f_s; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.b2);
       CU(P_gemm(ctx, g, st));
       // the adapter's input: saved for layers >= k, else scratch (a is consumed by now)
@@ -723,7 +742,7 @@ ra_status encoder_blocks(ra_ctx* ctx, const void* x, int B, int S, int l0, int l
       out_idx ^= 1;
       continue;
     }
-    g = gemm_args(ctx, O, H, ctx->w(o.Wo), H, T, H, H);
+    g = gemm_args(ctx, O, H, ctx->w(o.Wo), H, T, H, H, fs.sk);
     g.C = a; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.bo);
     CU(P_gemm(ctx, g, st));
     AdapterFwdArgs ad;
@@ -733,13 +752,13 @@ ra_status encoder_blocks(ra_ctx* ctx, const void* x, int B, int S, int l0, int l
     ad.gamma = ctx->w<float>(o.g1); ad.beta = ctx->w<float>(o.be1); ad.eps = ctx->cfg.norm_eps;
     ad.y = y1; ad.xhat = xhat1; ad.rstd = rstd1;
     CU(P_adapter_fwd(ctx, ad, st));
-    g = gemm_args(ctx, y1, H, ctx->w(o.W1), H, T, F, H);
+    g = gemm_args(ctx, y1, H, ctx->w(o.W1), H, T, F, H, fs.sk);
     // saved layers also keep GELU'(u) for the backward; frozen layers need GELU(u) only
     g.epi = gp ? EPI_BIAS_GELU_G : EPI_BIAS_GELU;
     g.C = gp; g.ldc = F; g.c_dtype = act; g.bias = ctx->w<float>(o.b1);
     g.C2 = hbuf; g.ldc2 = F; g.c2_dtype = act;
     CU(P_gemm(ctx, g, st));
-    g = gemm_args(ctx, hbuf, F, ctx->w(o.W2), F, T, H, F);
+    g = gemm_args(ctx, hbuf, F, ctx->w(o.W2), F, T, H, F, fs.sk);
     g.C = f; g.ldc = H; g.c_dtype = act; g.bias = ctx->w<float>(o.b2);
     CU(P_gemm(ctx, g, st));
     ad.a = f; ad.Wd = Pl + (size_t)2 * H * m; ad.Wu = Pl + (size_t)3 * H * m; ad.z = zF;
@@ -1439,10 +1458,17 @@ ra_status ra_gemm_bf16(const void* A_dev, const void* B_dev, void* C_dev, int32_
   return e == cudaSuccess ? RA_OK : RA_ERR_CUDA;
 }
 
+size_t ra_gemm_scratch_bytes(void) {
+  return align_up((size_t)kSkSlots * gemm_sk_flags_per_slot() * 4) + (size_t)kSkSlots * gemm_sk_slot_bytes();
+}
+
 ra_status ra_gemm_bf16_epi(const void* A_dev, const void* B_dev, int32_t M, int32_t N, int32_t K,
                            int32_t epi, const float* bias_dev, const void* aux_dev, void* C_dev,
-                           int32_t c_dtype, void* C2_dev, ra_stream_t stream) {
+                           int32_t c_dtype, void* C2_dev, void* scratch_dev, size_t scratch_bytes,
+                           ra_stream_t stream) {
   if (!A_dev || !B_dev || M < 0 || N <= 0 || K <= 0) return RA_ERR_ARG;
+  if (scratch_dev && (scratch_bytes < ra_gemm_scratch_bytes() || (uintptr_t)scratch_dev % kAlign))
+    return RA_ERR_ARG;
   if (c_dtype != RA_F32 && c_dtype != RA_BF16) return RA_ERR_ARG;
   if (K % 8 || N % 8) return RA_ERR_SHAPE;
   const bool b_kn = (epi & RA_EPI_B_KN) != 0;
@@ -1472,6 +1498,11 @@ ra_status ra_gemm_bf16_epi(const void* A_dev, const void* B_dev, int32_t M, int3
       g.epi = EPI_RESID; g.aux = aux_dev; g.ldaux = N; g.aux_dtype = DT_F32;
       break;
     default: return RA_ERR_ARG;
+  }
+  if (scratch_dev) {
+    g.sk_flags = (unsigned*)scratch_dev;
+    g.sk_ws = (float*)((char*)scratch_dev + align_up((size_t)kSkSlots * gemm_sk_flags_per_slot() * 4));
+    g.sk_slots = kSkSlots;
   }
   if (!tc_available()) return RA_ERR_UNSUPPORTED;
   cudaError_t e = gemm_tc(g, (cudaStream_t)stream);

@@ -124,7 +124,8 @@ _SIGS = {
                                C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p]),
     "ra_gemm_bf16_epi": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
                                    C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
-                                   C.c_void_p, C.c_void_p]),
+                                   C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]),
+    "ra_gemm_scratch_bytes": (C.c_size_t, []),
     "ra_adapter_backward": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                       C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
                                       C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]),
@@ -291,10 +292,14 @@ RA_EPI_STORE, RA_EPI_BIAS_GELU, RA_EPI_MUL, RA_EPI_RESID, RA_EPI_BIAS_GELU_G = 0
 RA_EPI_B_KN = 0x100
 
 
+def ra_gemm_scratch_bytes() -> int:
+    return int(lib().ra_gemm_scratch_bytes())
+
+
 def ra_gemm_bf16_epi(A_ptr, B_ptr, M, N, K, epi, bias_ptr=None, aux_ptr=None, C_ptr=None,
-                     c_dtype=RA_BF16, C2_ptr=None, stream=None):
+                     c_dtype=RA_BF16, C2_ptr=None, scratch_ptr=None, scratch_bytes=0, stream=None):
     _check(lib().ra_gemm_bf16_epi(A_ptr, B_ptr, M, N, K, epi, bias_ptr, aux_ptr, C_ptr, c_dtype,
-                                  C2_ptr, _stream_ptr(stream)))
+                                  C2_ptr, scratch_ptr, scratch_bytes, _stream_ptr(stream)))
 
 
 def ra_adapter_backward_scratch_bytes(T, H, m) -> int:

@@ -187,3 +187,54 @@ def test_gemm_b_given_as_k_by_n(M, N, K, epi):
     ref = acc.cuda()
     assert not bool(C.isnan().any())
     assert (C - ref).abs().max().item() <= 1e-4 * ref.abs().max().item()
+
+
+# Stream-K: the k-blocks of the last, partial round of output tiles spread over all CTAs,
+# their fp32 partials summed in a fixed order by the CTA that finishes each tile.  It applies
+# where each CTA's share is at least 24 k-blocks: the BERT-large FFN-down / dY1 (K = 4096)
+# and dX (K = 3072) shapes, 256 tiles of 128 x 256 on the SMs (1.7 rounds), with B as given
+# or as stored [K, N], and ragged M, N and K; bias; bf16 and f32 outputs.  The K = 1024
+# shapes (attention output, QKV) stay one tile per CTA, bitwise the result without scratch.
+@pytest.mark.parametrize("M,N,K,bias,cdt,kn,sk", [
+    (8192, 1024, 4096, False, "f32", False, True), (8192, 1024, 4096, False, "f32", True, True),
+    (8192, 1024, 3072, False, "f32", True, True), (8192, 1024, 4096, True, "bf16", False, True),
+    (8000, 1000, 4000, True, "f32", False, True), (8192, 1024, 1024, True, "f32", False, False),
+    (8192, 3072, 1024, True, "f32", False, False)])
+def test_gemm_stream_k(M, N, K, bias, cdt, kn, sk):
+    import torch
+    A, B, acc, g = _operands(M, N, K, 11)
+    if kn:  # the same product with B handed over as stored [K, N]
+        B = B.T.contiguous()
+    b = (torch.randn(N, generator=g) * 0.1).float()
+    ref = (acc + b if bias else acc).cuda()
+    bd = b.cuda() if bias else None
+    nbytes = R.ra_gemm_scratch_bytes()
+    ws = torch.zeros(nbytes // 4, dtype=torch.int32, device="cuda")
+    dt, rdt = (torch.bfloat16, R.RA_BF16) if cdt == "bf16" else (torch.float32, R.RA_F32)
+    epi = R.RA_EPI_STORE | (R.RA_EPI_B_KN if kn else 0)
+
+    def run(scratch, A_=A):
+        C = torch.full((M, N), float("nan"), dtype=dt, device="cuda")
+        R.ra_gemm_bf16_epi(A_.data_ptr(), B.data_ptr(), M, N, K, epi,
+                           bd.data_ptr() if bias else None, None, C.data_ptr(), rdt, None,
+                           ws.data_ptr() if scratch else None, nbytes if scratch else 0)
+        torch.cuda.synchronize()
+        return C
+
+    # another product through the same scratch first: the flags it leaves must be clear
+    # (160 slots x 12 epilogue warps of u32 flags at the start of the scratch)
+    run(True, A_=torch.flip(A, [0]))
+    assert int(ws[: 160 * 12].abs().sum().item()) == 0
+    C1 = run(True)
+    C2 = run(True)
+    C0 = run(False)
+    assert torch.equal(C1, C2), "stream-K result depends on timing"
+    assert int(ws[: 160 * 12].abs().sum().item()) == 0
+    if cdt == "bf16":
+        _check(C1, ref)
+    else:
+        assert not bool(C1.isnan().any())
+        assert (C1 - ref).abs().max().item() <= 1e-4 * ref.abs().max().item()
+        # a split tile sums its k-blocks in another order than one accumulator does: some
+        # fp32 outputs differ in their last bits where stream-K ran, none where it did not
+        assert torch.equal(C1, C0) != sk
