@@ -2,18 +2,19 @@
 // with TMEM accumulators) for the encoder's short sequences: bf16, head_dim 64, no mask, no
 // RoPE, S <= 256.  CTA = 128 queries of one (batch, head), 8 warps (two per TMEM lane
 // quadrant; each query row is shared by two threads, each taking half of the keys):
-//   - q (128 x 64) and k (NK x 64; NK = S rounded up to 64) are copied (cp.async) into shared
-//     memory in the 128-byte-swizzled K-major layout the MMA reads, v in its own layout;
-//   - one thread issues S = q k^T (M 128, N NK, K 64) into TMEM columns [0, NK) while the
-//     others transpose v into v^T (64 x NK, K-major, swizzled);
+//   - one thread loads q (128 x 64), k and v (NK x 64; NK = S rounded up to 64) with three
+//     TMA boxes into 128-byte-swizzled tiles, completion on an mbarrier;
+//   - it issues S = q k^T (M 128, N NK, K 64) into TMEM columns [0, NK);
 //   - each pair of threads reads its row of S from TMEM: row max, p = exp((s - max) * scale),
 //     row sum (halves combined in a fixed order), and writes p (bf16) as the A operand of the
 //     second product;
-//   - O = p v (M 128, N 64, K NK) into TMEM columns [0, 64) (S is consumed by then); O / sum
-//     and the log-sum-exp (natural log of the scaled scores) go to memory.
-// p reuses the shared memory of k and the staged v, so two or more CTAs fit per SM.
-// All keys fit in one tile, so the softmax is exact in one pass (no running rescale).  Keys
-// at or beyond S are zero-filled and get p = 0.
+//   - O = p v (M 128, N 64, K NK) into TMEM columns [0, 64) (S is consumed by then), v read
+//     as stored, MN-major through the descriptor (no transposed copy); O / sum and the
+//     log-sum-exp (natural log of the scaled scores) go to memory.
+// p reuses the shared memory of q and k, so two CTAs fit per SM.  All keys fit in one tile,
+// so the softmax is exact in one pass (no running rescale).  Key rows at or beyond S hold
+// the next sequence's keys (or, past the last token, the copy's zero fill): they get p = 0,
+// and query rows beyond S are not stored.
 #include "common.cuh"
 #include "kernels.h"
 #include "tcgen05.cuh"
@@ -27,10 +28,6 @@ constexpr float kLog2eT = 1.4426950408889634f;
 constexpr int QT = 128;        // queries per CTA
 constexpr int DH = 64;         // head dim (one 128-byte swizzle atom of K)
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
-               : "memory");
-}
 __device__ __forceinline__ uint32_t pack_bf16x2_tc(float a, float b) {
   __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<uint32_t*>(&h);
@@ -40,43 +37,52 @@ __device__ __forceinline__ uint32_t sw128(int r, int j) { return (uint32_t)(r * 
 
 template <int NK>
 struct AttnTcPlan {
-  // K and the staged v are dead once S = q k^T is done and v^T is built; p reuses them
-  static constexpr int Q_OFF = 0;                      // [128][64]   16 KB
-  static constexpr int K_OFF = QT * 128;               // [NK][64]
-  static constexpr int V_OFF = K_OFF + NK * 128;       // [NK][64] as loaded (128-byte rows)
-  static constexpr int P_OFF = K_OFF;                  // NK / 64 atoms of [128][64]
-  static constexpr int VT_OFF = K_OFF + NK * 256;      // NK / 64 atoms of [64][64]
-  static constexpr int RED_OFF = Q_OFF;                // [2][128] f32 row partials, once q is consumed
-  static constexpr int BYTES = VT_OFF + NK * 128;
+  // v stays until O = p v; q and k are dead once S = q k^T is done, and p reuses them
+  static constexpr int V_OFF = 0;                      // [NK][64] swizzled, MN-major B
+  static constexpr int Q_OFF = NK * 128;               // [128][64] 16 KB
+  static constexpr int K_OFF = Q_OFF + QT * 128;       // [NK][64]
+  static constexpr int P_OFF = Q_OFF;                  // NK / 64 atoms of [128][64]
+  static constexpr int BYTES = (K_OFF + NK * 128 > P_OFF + NK * 256) ? K_OFF + NK * 128 : P_OFF + NK * 256;
   static constexpr int SMEM = BYTES;                   // the extern array is 1024-byte aligned
   static constexpr uint32_t TMEM_COLS = NK;            // S; O reuses columns [0, 64)
 };
 
+__device__ __forceinline__ void tma_load_2d_at(const CUtensorMap* tm, uint32_t dst, uint64_t* bar, int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
+      : "memory");
+}
+
 template <int NK>
-__global__ void __launch_bounds__(256) attn_fwd_tc_kernel(AttnArgs a) {
+__global__ void __launch_bounds__(256) attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
+                                                          const __grid_constant__ CUtensorMap tmKV, AttnArgs a) {
   using Pl = AttnTcPlan<NK>;
-  constexpr int NT = 256, HALF = NK / 2;
+  constexpr int HALF = NK / 2;
   extern __shared__ __align__(1024) uint8_t smem[];
-  __shared__ __align__(8) uint64_t mma_bar;
+  __shared__ __align__(8) uint64_t mma_bar, load_bar;
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_sh;
+  __shared__ float red[2][QT];  // per-row partials of the two halves
   const uint32_t sbase = smem_u32(smem);
   if (sbase & 1023u) {  // the swizzled operand tiles need 1024-byte alignment
     if (threadIdx.x == 0) set_dev_error(a.err, RA_DEVERR_BOUNDS);
     return;
   }
-  float (*red)[QT] = reinterpret_cast<float (*)[QT]>(smem + Pl::RED_OFF);  // per-row partials
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int quad = warp & 3, half = warp >> 2;  // TMEM lane quadrant, column half
   const int bh = blockIdx.y, b = bh / a.n_heads, hh = bh % a.n_heads;
-  const int H = a.n_heads * DH, ldq = 3 * H, S = a.S;
+  const int H = a.n_heads * DH, S = a.S;
   const int q0 = blockIdx.x * QT;
-  const bf16* qkv = reinterpret_cast<const bf16*>(a.qkv);
 
   if (tid == 0) {
     mbar_init(&mma_bar, 1);
+    mbar_init(&load_bar, 1);
     abort_sh = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKV)) : "memory");
   }
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -84,52 +90,34 @@ __global__ void __launch_bounds__(256) attn_fwd_tc_kernel(AttnArgs a) {
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  pdl_wait();
-  pdl_trigger();
-
-  // q, k (swizzled) and v (as loaded) by cp.async; rows beyond S read as zero
-  for (int e = tid; e < QT * 8; e += NT) {
-    const int r = e >> 3, j = e & 7, q = q0 + r;
-    const bool ok = q < S;
-    cp_async16(sbase + Pl::Q_OFF + sw128(r, j), qkv + (size_t)(b * S + (ok ? q : 0)) * ldq + hh * DH + 8 * j, ok);
-  }
-  for (int e = tid; e < NK * 8; e += NT) {
-    const int r = e >> 3, j = e & 7;
-    const bool ok = r < S;
-    const bf16* src = qkv + (size_t)(b * S + (ok ? r : 0)) * ldq + hh * DH + 8 * j;
-    cp_async16(sbase + Pl::K_OFF + sw128(r, j), src + H, ok);
-    cp_async16(sbase + Pl::V_OFF + r * 128 + 16 * j, src + 2 * H, ok);
-  }
-  asm volatile("cp.async.commit_group;" ::: "memory");
-  asm volatile("cp.async.wait_group 0;" ::: "memory");
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic writes -> MMA reads
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base_sh;
+  pdl_wait();
+  pdl_trigger();
+
+  // q, k and v: one box each from the [B S, 3 H] qkv matrix (x = the head's columns)
+  if (tid == 0) {
+    mbar_expect_tx(&load_bar, (uint32_t)(QT + 2 * NK) * 128);
+    tma_load_2d_at(&tmQ, sbase + Pl::Q_OFF, &load_bar, hh * DH, b * S + q0);
+    tma_load_2d_at(&tmKV, sbase + Pl::K_OFF, &load_bar, H + hh * DH, b * S);
+    tma_load_2d_at(&tmKV, sbase + Pl::V_OFF, &load_bar, 2 * H + hh * DH, b * S);
+  }
+  bool ok = mbar_wait(&load_bar, 0, &abort_sh, a.err);
+  tc_fence_after();
 
   // S = q k^T
-  if (tid == 0) {
+  if (tid == 0 && ok) {
     constexpr uint32_t idesc = idesc_bf16(QT, NK);
     const uint64_t ad = sdesc_sw128(sbase + Pl::Q_OFF), bd = sdesc_sw128(sbase + Pl::K_OFF);
 #pragma unroll
     for (int k = 0; k < DH / 16; ++k) umma_bf16(tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, k > 0);
     umma_commit(&mma_bar);
   }
-  // meanwhile v -> v^T: item (dim d, 8 keys) gathers a column segment (lanes take consecutive
-  // dims of the same keys: conflict-free) and writes one 16-byte chunk of v^T row d
-  for (int e = tid; e < DH * (NK / 8); e += NT) {
-    const int d = e & 63, kc = e >> 6;  // keys 8 kc .. 8 kc + 7
-    const uint16_t* src = reinterpret_cast<const uint16_t*>(smem + Pl::V_OFF) + (size_t)(8 * kc) * DH + d;
-    uint32_t w[4];
-#pragma unroll
-    for (int t = 0; t < 4; ++t) w[t] = (uint32_t)src[(2 * t) * DH] | ((uint32_t)src[(2 * t + 1) * DH] << 16);
-    uint8_t* atom = smem + Pl::VT_OFF + (kc >> 3) * (DH * 128);
-    *reinterpret_cast<uint4*>(atom + sw128(d, kc & 7)) = make_uint4(w[0], w[1], w[2], w[3]);
-  }
-  bool ok = mbar_wait(&mma_bar, 0, &abort_sh, a.err);
+  if (ok) ok = mbar_wait(&mma_bar, 0, &abort_sh, a.err);
   tc_fence_before();
-  __syncthreads();  // q, k and the staged v are no longer read: red and p may overwrite them
+  __syncthreads();  // q and k are no longer read: p may overwrite them
   tc_fence_after();
 
   // softmax of row `row` over this thread's half of the keys
@@ -183,12 +171,11 @@ __global__ void __launch_bounds__(256) attn_fwd_tc_kernel(AttnArgs a) {
 
   // O = p v into TMEM columns [0, 64) (S is no longer read)
   if (tid == 0 && ok) {
-    constexpr uint32_t idesc = idesc_bf16(QT, DH);
+    constexpr uint32_t idesc = idesc_bf16_bmn(QT, DH);
 #pragma unroll
     for (int kk = 0; kk < NK / 16; ++kk) {
       const uint32_t pa = sbase + Pl::P_OFF + (kk >> 2) * (QT * 128) + (kk & 3) * 32;
-      const uint32_t vb = sbase + Pl::VT_OFF + (kk >> 2) * (DH * 128) + (kk & 3) * 32;
-      umma_bf16(tmem, sdesc_sw128(pa), sdesc_sw128(vb), idesc, kk > 0);
+      umma_bf16(tmem, sdesc_sw128(pa), sdesc_mn_sw128(sbase + Pl::V_OFF + kk * 2048), idesc, kk > 0);
     }
     umma_commit(&mma_bar);
   }
@@ -212,9 +199,11 @@ __global__ void __launch_bounds__(256) attn_fwd_tc_kernel(AttnArgs a) {
       }
       if (a.lse && half == 0) a.lse[(size_t)bh * S + q] = mx * a.scale + logf(sum);
     }
-  } else {
-    // a wait gave up: let an issued product finish before TMEM is released
+  } else if (tid == 0) {
+    // a wait gave up: the copies and any issued product finish before the shared memory and
+    // TMEM are released (bounded waits)
     volatile int no_abort = 0;
+    mbar_wait(&load_bar, 0, &no_abort, nullptr);
     mbar_wait(&mma_bar, 1, &no_abort, nullptr);
   }
   tc_fence_before();
@@ -235,8 +224,14 @@ cudaError_t launch_tc(const AttnArgs& a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     attr = true;
   }
+  // the qkv matrix [B S, 3 H]: q boxes of 64 columns x 128 rows, k and v boxes of NK rows
+  const int H = a.n_heads * DH;
+  CUtensorMap mq, mkv;
+  if (!tma_map_bf16(&mq, a.qkv, (int64_t)a.B * a.S, 3LL * H, 3LL * H, DH, QT) ||
+      !tma_map_bf16(&mkv, a.qkv, (int64_t)a.B * a.S, 3LL * H, 3LL * H, DH, NK))
+    return cudaErrorNotSupported;
   cudaError_t e = launch_pdl(k, dim3((a.S + QT - 1) / QT, a.B * a.n_heads), dim3(256),
-                             (size_t)AttnTcPlan<NK>::SMEM, st, a);
+                             (size_t)AttnTcPlan<NK>::SMEM, st, mq, mkv, a);
   note_launch(1);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
@@ -244,7 +239,9 @@ cudaError_t launch_tc(const AttnArgs& a, cudaStream_t st) {
 }  // namespace
 
 bool attention_tc_ok(const AttnArgs& a) {
-  return a.dtype == DT_BF16 && a.head_dim == DH && !a.causal && !a.rope && a.S >= 1 && a.S <= 256;
+  // the TMA boxes start on 16-byte boundaries of the qkv rows
+  return a.dtype == DT_BF16 && a.head_dim == DH && !a.causal && !a.rope && a.S >= 1 && a.S <= 256 &&
+         (reinterpret_cast<uintptr_t>(a.qkv) & 15) == 0;
 }
 
 cudaError_t attention_fwd_tc(const AttnArgs& a, cudaStream_t st) {

@@ -968,6 +968,11 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 
 
 }  // namespace
 
+bool tma_map_bf16(CUtensorMap* out, const void* ptr, int64_t rows, int64_t cols, int64_t ld, int box_cols,
+                  int box_rows) {
+  return make_map(out, ptr, rows, cols, ld, box_cols, box_rows, DT_BF16);
+}
+
 size_t gemm_sk_slot_bytes() { return (size_t)SK_SLOT_FLOATS * 4; }
 int gemm_sk_flags_per_slot() { return SK_MAX_WARPS; }
 

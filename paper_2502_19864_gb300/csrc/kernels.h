@@ -1,6 +1,7 @@
 // kernels.h -- host-side launchers of the libringada kernels (internal, not ABI).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -89,6 +90,11 @@ cudaError_t selftest_wait(unsigned* err, uint64_t limit_ns, cudaStream_t st);
 // Whether the tcgen05 path is usable on the current device (sm_103).
 bool tc_available();
 int device_sm_count();
+// TMA map of a row-major bf16 [rows, cols] matrix (row stride ld elements), boxes of
+// box_cols x box_rows with the swizzle whose span is one box row (128-byte rows: the
+// 128-byte swizzle the tcgen05 operand descriptors read); false if the driver refuses it.
+bool tma_map_bf16(CUtensorMap* out, const void* ptr, int64_t rows, int64_t cols, int64_t ld, int box_cols,
+                  int box_rows);
 
 // ---------------------------------------------------------------------------------------
 // Attention (per (batch, head); token t = b*S + s; head hh at columns hh*dh of q/k/v).
