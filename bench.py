@@ -581,6 +581,17 @@ def gpu_main(args):
                                "step graph: adds the launch gap and prologue that programmatic "
                                "dependent launch hides in the step (lower bound)"},
     }
+    if cfg.dtype != "bf16":
+        # fp32 models run the SIMT GEMM (FFMA): against the FFMA peak of 152 SMs x 128 lanes x
+        # 2 flops x 2.07 GHz, not the tensor-core peak
+        ffma_peak = 152 * 128 * 2 * 2.07e9 / 1e12
+        roof.update({"kernel": "frozen-weight and dX GEMMs (SIMT fp32, FFMA), all launches of one step",
+                     "bound": "alu", "peak": ffma_peak,
+                     "peak_kind": "FFMA issue rate: 152 SMs x 128 lanes x 2 flops x 2070 MHz",
+                     "frac": replay_tf / ffma_peak if replay_tf else None,
+                     "frac_of_sustained": None, "peak_sustained": None, "traffic": None,
+                     "traffic_note": "the DRAM capture covers the tensor-core GEMM"})
+        roof["event_pair"]["frac"] = (gr["tflops"] / ffma_peak) if gr and gr["tflops"] else None
     phases = {k: {"ms": v["ms"], "calls": v["calls"],
                   "tflops": (v["flops"] / v["ms"] / 1e9) if v["ms"] > 0 and v["flops"] else None,
                   "gbs": (v["bytes"] / v["ms"] / 1e6) if v["ms"] > 0 and v["bytes"] else None}
