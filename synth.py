@@ -92,6 +92,10 @@ CONFIGS: Dict[str, ModelCfg] = {
     "small_paper_bf16": _paper(3, 256, 4, 1024, 32, 3, 100, "bf16"),
     # two 128-row key/query blocks with a ragged second block (S = 250)
     "small_enc_s250_bf16": _enc(2, 256, 4, 1024, 32, 2, 250, "bf16"),
+    # m = 64 and H = 512: the fused tcgen05 adapter forward over clusters of two CTAs, with a
+    # ragged last 128-row tile (T = 300), in both placements
+    "small_enc_m64_bf16": _enc(2, 512, 8, 1024, 64, 3, 100, "bf16"),
+    "small_paper_m64_bf16": _paper(2, 512, 8, 1024, 64, 3, 100, "bf16"),
     # the bench workloads' shapes with the other heads / placement (per-kernel profiles)
     "base_span": _span(12, 768, 12, 3072, 64, 32, 128, "bf16"),
     "large_paper": _paper(24, 1024, 16, 4096, 64, 32, 256, "bf16"),

@@ -41,12 +41,14 @@ def test_fp32_parity_every_depth(name):
 
 
 @pytest.mark.parametrize("name", ["small_enc_bf16", "small_dec_bf16", "small_span_bf16",
-                                  "small_paper_bf16", "small_enc_s250_bf16"])
+                                  "small_paper_bf16", "small_enc_s250_bf16", "small_enc_m64_bf16",
+                                  "small_paper_m64_bf16"])
 def test_bf16_parity_every_depth(name):
     _parity_all_depths(name)
 
 
-@pytest.mark.parametrize("name", ["mid_enc_f32", "tiny_paper", "small_enc_bf16", "small_paper_bf16"])
+@pytest.mark.parametrize("name", ["mid_enc_f32", "tiny_paper", "small_enc_bf16", "small_paper_bf16",
+                                  "small_enc_m64_bf16"])
 def test_truncated_equals_full_and_nothing_below_k(name):
     import torch
     cfg = synth.CONFIGS[name]
