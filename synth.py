@@ -96,6 +96,9 @@ CONFIGS: Dict[str, ModelCfg] = {
     # ragged last 128-row tile (T = 300), in both placements
     "small_enc_m64_bf16": _enc(2, 512, 8, 1024, 64, 3, 100, "bf16"),
     "small_paper_m64_bf16": _paper(2, 512, 8, 1024, 64, 3, 100, "bf16"),
+    # the BERT-large layer shapes on 2 layers: its FFN-down and dX GEMMs run stream-K, on two
+    # streams at once when the next batch's prefix overlaps
+    "large_2l": _enc(2, 1024, 16, 4096, 64, 32, 256, "bf16"),
     # the bench workloads' shapes with the other heads / placement (per-kernel profiles)
     "base_span": _span(12, 768, 12, 3072, 64, 32, 128, "bf16"),
     "large_paper": _paper(24, 1024, 16, 4096, 64, 32, 256, "bf16"),

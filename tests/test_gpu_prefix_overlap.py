@@ -74,13 +74,15 @@ def test_split_forward_is_bitwise_the_forward(name):
         run.close()
 
 
-def test_prefix_on_a_second_stream_overlapping_the_backward_matches_sequential_steps():
+@pytest.mark.parametrize("name", ["small_enc_bf16", "large_2l"])
+def test_prefix_on_a_second_stream_overlapping_the_backward_matches_sequential_steps(name):
     """Four Adam steps on distinct batches with the unfreezing depth growing from 1 to 2:
     the prefix of batch s + 1 is enqueued on stream B while batch s's suffix, backward and
     update run on stream A (events order the shared buffers), against the same steps run
-    one after the other through ra_forward."""
+    one after the other through ra_forward.  With the BERT-large layer shapes the stream-K
+    GEMMs of both streams run at the same time, each on its own scratch."""
     import torch
-    cfg = synth.CONFIGS["small_enc_bf16"]
+    cfg = synth.CONFIGS[name]
     w = synth.make_workload(cfg, 2)
     batches = [synth.make_batch(cfg, 50 + i) for i in range(4)]
     depths = [1, 1, 2, 2]
