@@ -99,6 +99,14 @@ __device__ __forceinline__ float2 gelu_grad2(float2 x) {
   const float2 ex = make_float2(__expf(q.x), __expf(q.y));
   return __fadd2_rn(Phi, __fmul2_rn(__fmul2_rn(x, ex), f2(0.39894228040143268f)));
 }
+// 2^x on the special function unit (ex2.approx): about 2 ulp, results below 2^-126 flushed to
+// zero -- the softmax probabilities it serves are rounded to bf16, and one below 2^-126
+// contributes nothing
+__device__ __forceinline__ float ex2_fast(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
 __device__ __forceinline__ float silu_grad_f(float x) {
   float s = 1.0f / (1.0f + expf(-x));

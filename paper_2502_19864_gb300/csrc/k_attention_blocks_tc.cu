@@ -208,7 +208,7 @@ __global__ void __launch_bounds__(NTHR, DH == 64 ? 2 : 1) attn_bwd_tc_kernel(Att
             bool live = rg < S && cg < S;
             // causal: key <= query
             if (CAUSAL) live = live && (keys ? rg <= cg : cg <= rg);
-            pp[u] = live ? exp2f(s[e] * sl2 - (keys ? LSE[c] : LSE[row])) : 0.f;
+            pp[u] = live ? ex2_fast(s[e] * sl2 - (keys ? LSE[c] : LSE[row])) : 0.f;
           }
           w[t] = pk2(pp[0], pp[1]);
         }
@@ -530,7 +530,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_blocks_tc_kernel(AttnArgs a)
       if (m > -INFINITY) {
 #pragma unroll
         for (int e = 0; e < 32; ++e)
-          if (live(k0 + e)) l += exp2f(s[e] * sl2 - m);
+          if (live(k0 + e)) l += ex2_fast(s[e] * sl2 - m);
       }
     }
   }
@@ -567,8 +567,8 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_blocks_tc_kernel(AttnArgs a)
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
           const int e = 8 * g + 2 * t;
-          const float p0 = live(k0 + e) ? exp2f(s[e] * sl2 - lse2) : 0.f;
-          const float p1 = live(k0 + e + 1) ? exp2f(s[e + 1] * sl2 - lse2) : 0.f;
+          const float p0 = live(k0 + e) ? ex2_fast(s[e] * sl2 - lse2) : 0.f;
+          const float p1 = live(k0 + e + 1) ? ex2_fast(s[e + 1] * sl2 - lse2) : 0.f;
           w[t] = pk2(p0, p1);
         }
         *reinterpret_cast<uint4*>(xrow + swz(row, 4 * h2 + g)) = make_uint4(w[0], w[1], w[2], w[3]);

@@ -151,8 +151,8 @@ __global__ void __launch_bounds__(256) attn_fwd_tc_kernel(const __grid_constant_
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
           const int i = 8 * q + 2 * t;
-          const float p0 = c + i < S ? exp2f((s[i] - mx) * sl2) : 0.f;
-          const float p1 = c + i + 1 < S ? exp2f((s[i + 1] - mx) * sl2) : 0.f;
+          const float p0 = c + i < S ? ex2_fast((s[i] - mx) * sl2) : 0.f;
+          const float p1 = c + i + 1 < S ? ex2_fast((s[i + 1] - mx) * sl2) : 0.f;
           sum += p0 + p1;
           __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
           w[t] = *reinterpret_cast<uint32_t*>(&h2);
