@@ -107,9 +107,12 @@ __device__ __forceinline__ float ex2_fast(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
-__device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
+// SiLU and its derivative with the special-function exponential and the fast division (a few
+// ulp; they run per element in the SwiGLU epilogues).  For x below about -88 the denominator
+// overflows and the sigmoid is 0, its limit.
+__device__ __forceinline__ float silu_f(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
 __device__ __forceinline__ float silu_grad_f(float x) {
-  float s = 1.0f / (1.0f + expf(-x));
+  const float s = __fdividef(1.0f, 1.0f + __expf(-x));
   return s * (1.0f + x * (1.0f - s));
 }
 
