@@ -606,8 +606,33 @@ __global__ void __launch_bounds__(HEAD_FWD_THREADS) encoder_head_fwd_kernel(cons
     float acc[CM];
 #pragma unroll
     for (int c = 0; c < CM; ++c) acc[c] = 0.f;
+    // bf16 rows: 8 columns per lane and load (16 bytes), so a row takes H / 256 round trips
+    int i0 = 0;
+    if (sizeof(T) == 2 && H % 256 == 0 && ((row * 2) & 15) == 0 &&
+        ((reinterpret_cast<uintptr_t>(y) | reinterpret_cast<uintptr_t>(Wh)) & 15) == 0) {
+      for (int i = 8 * lane; i < H; i += 256) {
+        const uint4 w = *reinterpret_cast<const uint4*>(reinterpret_cast<const T*>(y) + row + i);
+        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+        float x[8];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u[q]));
+          x[2 * q] = f.x;
+          x[2 * q + 1] = f.y;
+        }
+#pragma unroll
+        for (int c = 0; c < CM; ++c)
+          if (c < C) {
+            const float4 a0 = __ldg(reinterpret_cast<const float4*>(Wh + (int64_t)c * H + i));
+            const float4 a1 = __ldg(reinterpret_cast<const float4*>(Wh + (int64_t)c * H + i + 4));
+            acc[c] += x[0] * a0.x + x[1] * a0.y + x[2] * a0.z + x[3] * a0.w + x[4] * a1.x + x[5] * a1.y +
+                      x[6] * a1.z + x[7] * a1.w;
+          }
+      }
+      i0 = H;
+    }
 #pragma unroll 8
-    for (int i = lane; i < H; i += 32) {
+    for (int i = i0 + lane; i < H; i += 32) {
       const float x = ldf<T>(y, row + i);
 #pragma unroll
       for (int c = 0; c < CM; ++c)
@@ -902,21 +927,43 @@ __global__ void __launch_bounds__(256) mean_kernel(const float* v, int n, float*
 // ---------------------------------------------------------------------------------------
 // Adam
 // ---------------------------------------------------------------------------------------
+// The bias corrections depend only on the segment's step count: they are evaluated once for
+// the segments of a block's first and last element instead of per element (powf twice per
+// element dominated the kernel's instructions); only a segment shorter than a block, lying
+// strictly inside one, falls back to evaluating them per element.
 __global__ void adam_kernel(AdamArgs a) {
-  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  __shared__ float corr[2][2];  // [first / second segment of the block][lr / bc1, 1 / sqrt(bc2)]
+  __shared__ int segs[2];
+  const int64_t base = (int64_t)blockIdx.x * blockDim.x;
+  if (threadIdx.x < 2) {
+    const int64_t e = threadIdx.x == 0 ? base : min(a.n - 1, base + (int64_t)blockDim.x - 1);
+    const int64_t se = e / a.seg_len;
+    const int s = (int)(se < a.n_seg - 1 ? se : a.n_seg - 1);
+    const float t = (float)(a.steps[s] + 1);
+    corr[threadIdx.x][0] = a.lr / (1.f - powf(a.beta1, t));
+    corr[threadIdx.x][1] = 1.f / sqrtf(1.f - powf(a.beta2, t));
+    segs[threadIdx.x] = s;
+  }
+  __syncthreads();
+  const int64_t i = base + threadIdx.x;
   if (i >= a.n) return;
-  int s = (int)(i / a.seg_len);
-  if (s >= a.n_seg) s = a.n_seg - 1;
-  float t = (float)(a.steps[s] + 1);
-  float g = a.g[i];
-  float m = a.beta1 * a.m[i] + (1.f - a.beta1) * g;
-  float v = a.beta2 * a.v[i] + (1.f - a.beta2) * g * g;
+  const int64_t si = i / a.seg_len;
+  const int s = (int)(si < a.n_seg - 1 ? si : a.n_seg - 1);
+  float c[2];
+  if (s == segs[0] || s == segs[1]) {
+    c[0] = corr[s == segs[0] ? 0 : 1][0];
+    c[1] = corr[s == segs[0] ? 0 : 1][1];
+  } else {  // a segment shorter than the block, lying strictly inside it
+    const float t = (float)(a.steps[s] + 1);
+    c[0] = a.lr / (1.f - powf(a.beta1, t));
+    c[1] = 1.f / sqrtf(1.f - powf(a.beta2, t));
+  }
+  const float g = a.g[i];
+  const float m = a.beta1 * a.m[i] + (1.f - a.beta1) * g;
+  const float v = a.beta2 * a.v[i] + (1.f - a.beta2) * g * g;
   a.m[i] = m;
   a.v[i] = v;
-  float bc1 = 1.f - powf(a.beta1, t);
-  float bc2 = 1.f - powf(a.beta2, t);
-  float denom = sqrtf(v) / sqrtf(bc2) + a.eps;
-  a.p[i] -= (a.lr / bc1) * m / denom;
+  a.p[i] -= c[0] * m / (sqrtf(v) * c[1] + a.eps);
 }
 
 __global__ void bump_kernel(int32_t* steps, int n) {
