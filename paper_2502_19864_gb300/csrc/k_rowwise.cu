@@ -1032,18 +1032,83 @@ __device__ __forceinline__ int64_t tfrag_off(int n, int k, int C) {
 // layout [rows, cols]) and PTB (transposed [cols, rows]) in the tiled fragment layout; when
 // H or m is not a multiple of 32 (no tensor-core kernel reads them then) they are plain
 // row-major copies.
-__global__ void adapter_transpose_kernel(const float* P, float* PT, bf16* PB, bf16* PTB, int H, int m) {
-  int layer = blockIdx.z >> 2, mat = blockIdx.z & 3;
-  int64_t base = (int64_t)layer * 4 * H * m + (int64_t)mat * H * m;
-  int rows = (mat & 1) ? m : H, cols = (mat & 1) ? H : m;
-  int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (e >= (int64_t)rows * cols) return;
-  int r = (int)(e / cols), c = (int)(e % cols);
-  const float v = P[base + e];
-  PT[base + (int64_t)c * rows + r] = v;
+// One block per 32 x 32 tile of one matrix: the tile is read row-major (coalesced, and PB's
+// fragment offsets of a 32-column run stay inside one 64-byte span), staged in shared memory,
+// and written transposed with the same coalescing for PT and PTB.
+__global__ void __launch_bounds__(256) adapter_transpose_kernel(const float* P, float* PT, bf16* PB,
+                                                                bf16* PTB, int H, int m) {
+  __shared__ float tile[32][33];
+  const int layer = blockIdx.z >> 2, mat = blockIdx.z & 3;
+  const int64_t base = (int64_t)layer * 4 * H * m + (int64_t)mat * H * m;
+  const int rows = (mat & 1) ? m : H, cols = (mat & 1) ? H : m;
+  const int tiles_c = (cols + 31) >> 5;
+  const int r0 = (int)(blockIdx.x / tiles_c) * 32, c0 = (int)(blockIdx.x % tiles_c) * 32;
   const bool tiled = (H % 32 == 0) && (m % 32 == 0);
-  if (PB) PB[base + (tiled ? tfrag_off(r, c, cols) : e)] = __float2bfloat16_rn(v);
-  if (PTB) PTB[base + (tiled ? tfrag_off(c, r, rows) : (int64_t)c * rows + r)] = __float2bfloat16_rn(v);
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  for (int j = ty; j < 32; j += 8) {
+    const int r = r0 + j, c = c0 + tx;
+    if (r < rows && c < cols) {
+      const int64_t e = (int64_t)r * cols + c;
+      const float v = P[base + e];
+      tile[j][tx] = v;
+      if (PB) PB[base + (tiled ? tfrag_off(r, c, cols) : e)] = __float2bfloat16_rn(v);
+    }
+  }
+  __syncthreads();
+  for (int j = ty; j < 32; j += 8) {
+    const int c = c0 + j, r = r0 + tx;
+    if (r < rows && c < cols) {
+      const float v = tile[tx][j];
+      const int64_t t = (int64_t)c * rows + r;
+      PT[base + t] = v;
+      if (PTB) PTB[base + (tiled ? tfrag_off(c, r, rows) : t)] = __float2bfloat16_rn(v);
+    }
+  }
+}
+
+// Adam on the adapter matrices (Algorithm 1's adapter update, the same arithmetic as
+// adam_kernel) fused with the refresh of their transposed and bf16 copies: one block per
+// 32 x 32 tile of one matrix updates the tile's masters in place, then writes PB from the new
+// values and stages them in shared memory for PT and PTB, so P is read once per update
+// instead of twice. Every element of a layer shares the layer's step count, hence one bias
+// correction per block.
+__global__ void __launch_bounds__(256) adam_adapter_kernel(AdamArgs a, float* PT, bf16* PB, bf16* PTB,
+                                                           int H, int m) {
+  __shared__ float tile[32][33];
+  const int layer = blockIdx.z >> 2, mat = blockIdx.z & 3;
+  const int64_t base = (int64_t)layer * 4 * H * m + (int64_t)mat * H * m;
+  const int rows = (mat & 1) ? m : H, cols = (mat & 1) ? H : m;
+  const int tiles_c = (cols + 31) >> 5;
+  const int r0 = (int)(blockIdx.x / tiles_c) * 32, c0 = (int)(blockIdx.x % tiles_c) * 32;
+  const bool tiled = (H % 32 == 0) && (m % 32 == 0);
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const float t = (float)(a.steps[layer] + 1);
+  const float c_lr = a.lr / (1.f - powf(a.beta1, t)), c_v = 1.f / sqrtf(1.f - powf(a.beta2, t));
+  for (int j = ty; j < 32; j += 8) {
+    const int r = r0 + j, c = c0 + tx;
+    if (r < rows && c < cols) {
+      const int64_t e = (int64_t)r * cols + c, i = base + e;
+      const float g = a.g[i];
+      const float mo = a.beta1 * a.m[i] + (1.f - a.beta1) * g;
+      const float vo = a.beta2 * a.v[i] + (1.f - a.beta2) * g * g;
+      a.m[i] = mo;
+      a.v[i] = vo;
+      const float v = a.p[i] - c_lr * mo / (sqrtf(vo) * c_v + a.eps);
+      a.p[i] = v;
+      tile[j][tx] = v;
+      if (PB) PB[base + (tiled ? tfrag_off(r, c, cols) : e)] = __float2bfloat16_rn(v);
+    }
+  }
+  __syncthreads();
+  for (int j = ty; j < 32; j += 8) {
+    const int c = c0 + j, r = r0 + tx;
+    if (r < rows && c < cols) {
+      const float v = tile[tx][j];
+      const int64_t tt = (int64_t)c * rows + r;
+      PT[base + tt] = v;
+      if (PTB) PTB[base + (tiled ? tfrag_off(c, r, rows) : tt)] = __float2bfloat16_rn(v);
+    }
+  }
 }
 
 __global__ void activation_kernel(int which, const float* x, float* y, int64_t n) {
@@ -1319,9 +1384,20 @@ cudaError_t pack_rows(const float* src, void* dst, int dst_dtype, int R, int C, 
 cudaError_t adapter_transpose(const float* P, float* PT, void* PB, void* PTB, int n_layers,
                               int H, int m, cudaStream_t st) {
   if (n_layers <= 0) return cudaSuccess;
-  dim3 grid(blocks_for((int64_t)H * m, 256), 1, 4 * n_layers);
+  // both orientations of a matrix hold the same number of 32 x 32 tiles
+  dim3 grid((unsigned)(((H + 31) / 32) * ((m + 31) / 32)), 1, 4 * n_layers);
   adapter_transpose_kernel<<<grid, 256, 0, st>>>(P, PT, reinterpret_cast<bf16*>(PB),
                                                  reinterpret_cast<bf16*>(PTB), H, m);
+  note_launch(1);
+  return cudaGetLastError();
+}
+
+cudaError_t adam_adapter_update(const AdamArgs& a, float* PT, void* PB, void* PTB, int n_layers,
+                                int H, int m, cudaStream_t st) {
+  if (n_layers <= 0) return cudaSuccess;
+  dim3 grid((unsigned)(((H + 31) / 32) * ((m + 31) / 32)), 1, 4 * n_layers);
+  adam_adapter_kernel<<<grid, 256, 0, st>>>(a, PT, reinterpret_cast<bf16*>(PB), reinterpret_cast<bf16*>(PTB),
+                                            H, m);
   note_launch(1);
   return cudaGetLastError();
 }

@@ -268,6 +268,11 @@ struct AdamArgs {
 };
 cudaError_t adam_update(const AdamArgs& a, cudaStream_t st);
 cudaError_t adam_bump(int32_t* steps, int n, cudaStream_t st);
+// Adam over n_layers layers of adapters (a.p / a.g / a.m / a.v at the first layer's start,
+// a.steps[l] that layer's completed steps; a.n, a.seg_len and a.n_seg unused) fused with
+// the refresh adapter_transpose performs for the same layers.
+cudaError_t adam_adapter_update(const AdamArgs& a, float* PT, void* PB, void* PTB, int n_layers,
+                                int H, int m, cudaStream_t st);
 
 // Utilities
 cudaError_t convert_f32(const float* src, void* dst, int dst_dtype, int64_t n, cudaStream_t st);

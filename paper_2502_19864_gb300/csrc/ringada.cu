@@ -1215,12 +1215,25 @@ ra_status ra_adapter_update(ra_ctx* ctx, const ra_adam_cfg* adam, ra_stream_t st
   a.n_seg = (L - k) + (ctx->cfg.head_trainable ? 1 : 0);
   a.steps = ctx->steps() + k;
   a.lr = adam->lr; a.beta1 = adam->beta1; a.beta2 = adam->beta2; a.eps = adam->eps;
-  CU(prof(ctx, RA_PROF_UPDATE, 0, (double)a.n * 4 * 6 + (double)(L - k) * 4 * ctx->H * ctx->m * 8, st, [&] {
-    cudaError_t e = adam_update(a, st);
+  // adapters: Adam fused with the transposed / bf16 refresh; the encoder head (when trained)
+  // is one more segment through the plain kernel; the step counters advance last
+  AdamArgs h = a;
+  h.p = a.p + (size_t)(L - k) * per;
+  h.g = a.g + (size_t)(L - k) * per;
+  h.m = a.m + (size_t)(L - k) * per;
+  h.v = a.v + (size_t)(L - k) * per;
+  h.n = a.n - (int64_t)((L - k) * per);
+  h.seg_len = h.n > 0 ? h.n : 1;
+  h.n_seg = 1;
+  h.steps = a.steps + (L - k);
+  const size_t adapt = (size_t)(L - k) * per;
+  // per adapter element: g, m, v, p read and m, v, p written (28 B), PT (4 B), PB + PTB (4 B)
+  const double bytes = (double)adapt * (ctx->PB() ? 36 : 32) + (double)(h.n > 0 ? h.n : 0) * 28;
+  CU(prof(ctx, RA_PROF_UPDATE, 0, bytes, st, [&] {
+    cudaError_t e = adam_adapter_update(a, ctx->PT() + off, ctx->PB() ? ctx->PB() + off : nullptr,
+                                        ctx->PTB() ? ctx->PTB() + off : nullptr, L - k, ctx->H, ctx->m, st);
+    if (e == cudaSuccess && h.n > 0) e = adam_update(h, st);
     if (e == cudaSuccess) e = adam_bump(ctx->steps() + k, a.n_seg, st);
-    if (e == cudaSuccess)
-      e = adapter_transpose(ctx->P() + off, ctx->PT() + off, ctx->PB() ? ctx->PB() + off : nullptr,
-                            ctx->PTB() ? ctx->PTB() + off : nullptr, L - k, ctx->H, ctx->m, st);
     return e;
   }));
   ctx->bwd_since_update = false;
