@@ -126,24 +126,34 @@ __global__ void __launch_bounds__(256) attn_fwd_tc_kernel(const __grid_constant_
   const float sl2 = a.scale * kLog2eT;
   const int c0 = half * HALF;
   float mx = -INFINITY, sum = 0.f;
+  // a chunk of 32 keys all below S (every chunk when S is a multiple of 32) skips the
+  // per-key test: the softmax is issue-bound, so its instruction count sets its pace
   if (ok) {
 #pragma unroll 1
     for (int c = c0; c < c0 + HALF; c += 32) {
       float s[32];
       tmem_ld32(trow + c, s);
+      if (c + 32 <= S) {
 #pragma unroll
-      for (int i = 0; i < 32; ++i)
-        if (c + i < S) mx = fmaxf(mx, s[i]);
+        for (int i = 0; i < 32; ++i) mx = fmaxf(mx, s[i]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (c + i < S) mx = fmaxf(mx, s[i]);
+      }
     }
   }
   red[half][row] = mx;
   __syncthreads();
   mx = fmaxf(red[0][row], red[1][row]);
+  // p = 2^(s sl2 - mx sl2): one fused multiply-add per key
+  const float mxs = mx * sl2;
   if (ok) {
 #pragma unroll 1
     for (int c = c0; c < c0 + HALF; c += 32) {
       float s[32];
       tmem_ld32(trow + c, s);
+      const bool full = c + 32 <= S;
       uint8_t* atom = smem + Pl::P_OFF + (c >> 6) * (QT * 128);
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
@@ -151,8 +161,11 @@ __global__ void __launch_bounds__(256) attn_fwd_tc_kernel(const __grid_constant_
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
           const int i = 8 * q + 2 * t;
-          const float p0 = c + i < S ? ex2_fast((s[i] - mx) * sl2) : 0.f;
-          const float p1 = c + i + 1 < S ? ex2_fast((s[i + 1] - mx) * sl2) : 0.f;
+          float p0 = ex2_fast(fmaf(s[i], sl2, -mxs)), p1 = ex2_fast(fmaf(s[i + 1], sl2, -mxs));
+          if (!full) {
+            p0 = c + i < S ? p0 : 0.f;
+            p1 = c + i + 1 < S ? p1 : 0.f;
+          }
           sum += p0 + p1;
           __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
           w[t] = *reinterpret_cast<uint32_t*>(&h2);
