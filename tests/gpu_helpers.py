@@ -32,7 +32,7 @@ def ra_cfg(cfg, max_depth=0, max_batch=None, max_seq=None):
                       max_depth, cfg.norm_eps, cfg.rope_theta, placement)
 
 
-class GpuRun:
+class GpuStepper:
     """One context on cuda:0 loaded with a synthetic workload."""
 
     def __init__(self, cfg, w, max_depth=0, want_logits=True, max_batch=None, max_seq=None):

@@ -8,7 +8,7 @@ import numpy as np
 import pytest
 
 import synth
-from gpu_helpers import GpuRun, check_step, oracle_full
+from gpu_helpers import GpuStepper, check_step, oracle_full
 
 pytestmark = pytest.mark.gpu
 
@@ -21,7 +21,7 @@ def built():
 
 def _parity(cfg, w, depths, **kw):
     ref = oracle_full(cfg, w)
-    run = GpuRun(cfg, w, **kw)
+    run = GpuStepper(cfg, w, **kw)
     try:
         for d in depths:
             k = cfg.n_layers - d
@@ -60,7 +60,7 @@ def test_zero_up_projection_gives_exactly_zero_down_gradient(name):
         p["WuA"] = np.zeros_like(p["WuA"])
         p["WuF"] = np.zeros_like(p["WuF"])
     ref = oracle_full(cfg, w)
-    run = GpuRun(cfg, w)
+    run = GpuStepper(cfg, w)
     try:
         loss = run.step(cfg.n_layers)
         grads = run.grads(0)

@@ -7,7 +7,7 @@ import pytest
 import synth
 from oracle import ringada_oracle as O
 from paper_2502_19864_gb300 import ringada as R
-from gpu_helpers import GpuRun, check_step, oracle_full
+from gpu_helpers import GpuStepper, check_step, oracle_full
 
 pytestmark = pytest.mark.gpu
 
@@ -22,7 +22,7 @@ def _parity_all_depths(name, depths=None, seed=0):
     cfg = synth.CONFIGS[name]
     w = synth.make_workload(cfg, seed)
     ref = oracle_full(cfg, w)
-    run = GpuRun(cfg, w)
+    run = GpuStepper(cfg, w)
     reports = {}
     try:
         for d in depths or range(1, cfg.n_layers + 1):
@@ -53,7 +53,7 @@ def test_truncated_equals_full_and_nothing_below_k(name):
     import torch
     cfg = synth.CONFIGS[name]
     w = synth.make_workload(cfg, 3)
-    run = GpuRun(cfg, w)
+    run = GpuStepper(cfg, w)
     try:
         run.step(cfg.n_layers)
         full = run.grads(0)
@@ -81,7 +81,7 @@ def test_truncated_equals_full_and_nothing_below_k(name):
 
 def test_backward_below_saved_depth_and_shape_errors():
     cfg = synth.CONFIGS["tiny"]
-    run = GpuRun(cfg, synth.make_workload(cfg, 0))
+    run = GpuStepper(cfg, synth.make_workload(cfg, 0))
     try:
         run.forward(1)
         with pytest.raises(R.RingAdaError) as e:
@@ -106,7 +106,7 @@ def test_backward_below_saved_depth_and_shape_errors():
 def test_frozen_weights_unchanged_and_only_unfrozen_updated():
     cfg = synth.CONFIGS["small_enc_bf16"]
     w = synth.make_workload(cfg, 0)
-    run = GpuRun(cfg, w)
+    run = GpuStepper(cfg, w)
     try:
         wbuf = run.model.buffers[0].clone()
         before = {l: {key: run.model.param(l, key).cpu() for key in synth.ADAPTER_KEYS}
@@ -125,8 +125,8 @@ def test_frozen_weights_unchanged_and_only_unfrozen_updated():
 def test_step_is_deterministic():
     cfg = synth.CONFIGS["small_dec_bf16"]
     w = synth.make_workload(cfg, 0)
-    a = GpuRun(cfg, w)
-    b = GpuRun(cfg, w)
+    a = GpuStepper(cfg, w)
+    b = GpuStepper(cfg, w)
     try:
         la, lb = a.step(2), b.step(2)
         assert la == lb
@@ -144,8 +144,8 @@ def test_checkpoint_resume_is_bitwise():
     w = synth.make_workload(cfg, 0)
     batches = [synth.make_batch(cfg, 100 + s) for s in range(5)]
     depths = [1, 1, 2, 2, 2]
-    a = GpuRun(cfg, w)
-    b = GpuRun(cfg, w)
+    a = GpuStepper(cfg, w)
+    b = GpuStepper(cfg, w)
     try:
         for (x, y), d in zip(batches, depths):
             a.set_batch(x, y)
@@ -155,7 +155,7 @@ def test_checkpoint_resume_is_bitwise():
             b.step(d, update=True)
         blob = R.ra_get_trainable(b.ctx)
         b.close()
-        c = GpuRun(cfg, w)
+        c = GpuStepper(cfg, w)
         R.ra_set_trainable(c.ctx, blob)
         for (x, y), d in zip(batches[3:], depths[3:]):
             c.set_batch(x, y)
@@ -175,7 +175,7 @@ def test_adam_trajectory_matches_oracle_tiny():
     w = synth.make_workload(cfg, 0)
     batches = [synth.make_batch(cfg, 200 + s) for s in range(5)]
     depths = [R.schedule_depth(s, interval=2, d0=1, d_max=cfg.n_layers) for s in range(5)]
-    run = GpuRun(cfg, w)
+    run = GpuStepper(cfg, w)
     layers, head = O.to_f64_params(w["layers"], w["head"])
     opt = O.Adam(lr=1e-4)
     ref_losses = O.train(cfg, layers, head, batches, depths, opt)
@@ -253,7 +253,7 @@ def test_schedule_first_five_steps_base():
     assert depths == [1] * 5
     layers, head = O.to_f64_params(w["layers"], w["head"])
     ref_losses = O.train(cfg, layers, head, batches, depths, O.Adam(lr=1e-4))
-    run = GpuRun(cfg, w, max_depth=12)
+    run = GpuStepper(cfg, w, max_depth=12)
     try:
         for (x, y), d, rl in zip(batches, depths, ref_losses):
             run.set_batch(x, y)
@@ -280,7 +280,7 @@ def test_bounded_wait_expiry_is_reported_and_the_context_survives():
     step on the same context is correct."""
     cfg = synth.CONFIGS["tiny"]
     w = synth.make_workload(cfg, 0)
-    run = GpuRun(cfg, w)
+    run = GpuStepper(cfg, w)
     try:
         R.ra_selftest_wait_timeout(run.ctx, 20000)
         with pytest.raises(R.RingAdaError) as e:

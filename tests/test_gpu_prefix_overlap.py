@@ -12,7 +12,7 @@ import pytest
 
 import synth
 from paper_2502_19864_gb300 import ringada as R
-from gpu_helpers import GpuRun, ra_cfg
+from gpu_helpers import GpuStepper, ra_cfg
 
 pytestmark = pytest.mark.gpu
 
@@ -23,8 +23,8 @@ def built():
     __graft_entry__.build()
 
 
-class PrefixRun(GpuRun):
-    """A GpuRun whose context reserves the prefix buffers."""
+class PrefixRun(GpuStepper):
+    """A GpuStepper whose context reserves the prefix buffers."""
 
     def __init__(self, cfg, w):
         import torch
@@ -87,7 +87,7 @@ def test_prefix_on_a_second_stream_overlapping_the_backward_matches_sequential_s
     batches = [synth.make_batch(cfg, 50 + i) for i in range(4)]
     depths = [1, 1, 2, 2]
     # sequential reference
-    ref = GpuRun(cfg, w)
+    ref = GpuStepper(cfg, w)
     ref_losses = []
     try:
         for (x, y), d in zip(batches, depths):
@@ -156,7 +156,7 @@ def test_split_calls_reject_out_of_order_use():
     finally:
         run.close()
     # a context without prefix buffers
-    plain = GpuRun(cfg, synth.make_workload(cfg, 0))
+    plain = GpuStepper(cfg, synth.make_workload(cfg, 0))
     try:
         with pytest.raises(R.RingAdaError) as e:
             R.ra_forward_prefix(plain.ctx, plain.x.data_ptr(), cfg.batch, cfg.seq, 0)
