@@ -519,15 +519,25 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_blocks_tc_kernel(AttnArgs a)
       float s[32];
       tmem_ld32(trow + Pl::C_S + c0 + 32 * h2, s);
       const int k0 = j * BR + c0 + 32 * h2;
+      // a chunk whose 32 keys are all live for this row skips the per-key test
+      const bool all_live = live(k0) && live(k0 + 31);
       float bm = -INFINITY;
+      if (all_live) {
 #pragma unroll
-      for (int e = 0; e < 32; ++e)
-        if (live(k0 + e)) bm = fmaxf(bm, s[e] * sl2);
+        for (int e = 0; e < 32; ++e) bm = fmaxf(bm, s[e] * sl2);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+          if (live(k0 + e)) bm = fmaxf(bm, s[e] * sl2);
+      }
       if (bm > m) {
         l *= exp2f(m - bm);
         m = bm;
       }
-      if (m > -INFINITY) {
+      if (all_live) {
+#pragma unroll
+        for (int e = 0; e < 32; ++e) l += ex2_fast(s[e] * sl2 - m);
+      } else if (m > -INFINITY) {
 #pragma unroll
         for (int e = 0; e < 32; ++e)
           if (live(k0 + e)) l += ex2_fast(s[e] * sl2 - m);
@@ -561,14 +571,18 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_blocks_tc_kernel(AttnArgs a)
       float s[32];
       tmem_ld32(trow + Pl::C_S + c0 + 32 * h2, s);
       const int k0 = j * BR + c0 + 32 * h2;
+      const bool all_live = live(k0) && live(k0 + 31);
 #pragma unroll
       for (int g = 0; g < 4; ++g) {
         uint32_t w[4];
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
           const int e = 8 * g + 2 * t;
-          const float p0 = live(k0 + e) ? ex2_fast(s[e] * sl2 - lse2) : 0.f;
-          const float p1 = live(k0 + e + 1) ? ex2_fast(s[e + 1] * sl2 - lse2) : 0.f;
+          float p0 = ex2_fast(s[e] * sl2 - lse2), p1 = ex2_fast(s[e + 1] * sl2 - lse2);
+          if (!all_live) {
+            p0 = live(k0 + e) ? p0 : 0.f;
+            p1 = live(k0 + e + 1) ? p1 : 0.f;
+          }
           w[t] = pk2(p0, p1);
         }
         *reinterpret_cast<uint4*>(xrow + swz(row, 4 * h2 + g)) = make_uint4(w[0], w[1], w[2], w[3]);
